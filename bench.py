@@ -1,0 +1,384 @@
+#!/usr/bin/env python3
+"""Benchmark: decoded queries/s of the neural-texture decode on one GB300.
+
+Workload (one "step" = one ntc_decode over one batch): 16 texture sets of
+1024^2 (latents 512^2x8 + 256^2x8 fp16 each), 16 decoders 16->64->64->8 (the
+non-shared baseline, one decoder per set), 4,194,304 queries with a uniform
+random set id, uniform UV in [0,1)^2 and lod 0 -- fully divergent (about 14
+distinct decoders per 32-query warp).  Inputs are resident in HBM; L2 is
+flushed (a 256 MiB write) before every timed step and the flush is outside the
+step's CUDA events.
+
+Prints one JSON line.  ``--impl reference`` times the CPU oracle instead (the
+only other code that computes the same result) on a bounded query sample.
+
+Multi-GPU (torchrun): every rank decodes its own 4M-query batch against a full
+replica of the assets -- queries are independent, so there is no collective on
+the data path (weak scaling); the step time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decoded queries/sec on 1 GB300 vs distinct decoders per warp; % of roofline"
+UNIT = "queries/s"
+WORKLOAD = ("config2: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16), 16 decoders "
+            "16->64->64->8 (one per set), 4,194,304 queries: uniform set id, uniform UV, lod 0")
+BYTES_PER_QUERY = 16 + 8 * 16 + 8 * 4  # query record + 8 taps of 16 B + 8 fp32 outputs
+FLOPS_PER_QUERY = 2 * (16 * 64 + 64 * 64 + 64 * 8)
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ntc", choices=["ntc", "reference"])
+    p.add_argument("--mode", default="bucketed", choices=["bucketed", "bucketed_mma", "divergent"])
+    p.add_argument("--precision", default="fp16", choices=["fp16", "bf16", "fp32"])
+    p.add_argument("--no-sweep", action="store_true", help="skip the decoders-per-warp sweep")
+    p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
+    return p.parse_args()
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """Polls NVML (read-only) for SM clock and clock-event reasons."""
+    REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+               0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+               0x100: "display_clock_setting"}
+
+    def __init__(self, index: int):
+        self.ok = False
+        self.samples = []
+        try:
+            self.nvml = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.nvml.nvmlInit_v2() != 0:
+                return
+            self.h = ctypes.c_void_p()
+            if self.nvml.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(index), ctypes.byref(self.h)) != 0:
+                return
+            mx = ctypes.c_uint()
+            self.nvml.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(mx))  # 1 = SM clock
+            self.max_mhz = int(mx.value)
+            self.ok = True
+        except OSError:
+            pass
+
+    def _poll(self):
+        clk, rs, pw = ctypes.c_uint(), ctypes.c_ulonglong(), ctypes.c_uint()
+        while not self._stop.is_set():
+            self.nvml.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(clk))
+            self.nvml.nvmlDeviceGetCurrentClocksEventReasons(self.h, ctypes.byref(rs))
+            self.nvml.nvmlDeviceGetPowerUsage(self.h, ctypes.byref(pw))
+            self.samples.append((int(clk.value), int(rs.value), pw.value / 1000.0))
+            time.sleep(0.002)
+
+    def start(self):
+        if not self.ok:
+            return
+        self._stop = threading.Event()
+        self._t = threading.Thread(target=self._poll, daemon=True)
+        self._t.start()
+
+    def stop(self):
+        if not self.ok:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvml unavailable"]}
+        self._stop.set()
+        self._t.join()
+        s = self.samples
+        bits = 0
+        for _, r, _ in s:
+            bits |= r
+        reasons = sorted(v for k, v in self.REASONS.items() if bits & k)
+        return {"sm_mhz": statistics.median(c for c, _, _ in s) if s else None,
+                "sm_max_mhz": self.max_mhz, "reasons": reasons, "samples": len(s),
+                "power_w_max": max((p for _, _, p in s), default=None)}
+
+
+# --------------------------------------------------------------- helpers
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha1()
+    for f in ("decode_tc.cu", "decode_mma.cu", "ntc_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_27888_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:12]
+
+
+def recorded_traffic(kernel_tag):
+    """DRAM bytes per decode launch from the committed ncu summary, if it was
+    taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "decode_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        r = rec.get(kernel_tag)
+        if r and r.get("source_hash") == kernel_source_hash():
+            return float(r["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def workload(small: bool, rank: int):
+    from paper_2608_27888_gb300 import workloads as W
+    if small:
+        w = W.config(2, "small")
+    else:
+        seed = W.BASE_SEED + 2
+        S, T, n = 16, 1024, 4_194_304
+        a = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
+        q = W.queries_uniform(seed + 1000 * rank, n, S)
+        w = W.Workload("config2-full", a, q, {})
+    return w
+
+
+def mean_distinct(q, assets):
+    d = assets.set_to_decoder[q["set_id"]]
+    nw = len(d) // 32
+    x = np.sort(d[:nw * 32].reshape(nw, 32), axis=1)
+    return float((1 + (np.diff(x, axis=1) != 0).sum(1)).mean())
+
+
+# -------------------------------------------------------------- reference arm
+
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return
+    import oracle
+    w = workload(args.small, 0)
+    n = len(w.queries)
+    cores = os.cpu_count() or 1
+    sample = min(n, 1 << 20)
+    q = w.queries[:sample]
+    for _ in range(max(0, args.warmup)):
+        oracle.decode(w.assets, q[:4096], nthreads=cores)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.decode(w.assets, q, nthreads=cores)
+        times.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.mean(times)
+    value = sample / (ms / 1e3)
+    desc = f"first {sample:,} queries of the workload per step, oracle on {cores} host threads"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample_queries": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# ------------------------------------------------------------------- GPU arm
+
+def main():
+    args = parse()
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2608_27888_gb300 import ntc
+
+    w = workload(args.small, rank)
+    n = len(w.queries)
+    C = w.assets.out_dim
+    dec = ntc.Decoder(w.assets, args.precision)
+    qd = ntc.queries_to_device(w.queries)
+    out = torch.empty((n, C), dtype=torch.float32, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    def timed_steps(mode, steps, warmup, stages=False):
+        dec.set_stage_timing(stages)
+        for _ in range(warmup):
+            dec.decode(qd, out, mode=mode)
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        st_times = []
+        l0 = dec.launches()
+        barrier()
+        torch.cuda.synchronize()
+        for i in range(steps):
+            flush.zero_()
+            ev[i][0].record(stream)
+            dec.decode(qd, out, mode=mode)
+            ev[i][1].record(stream)
+            if stages:
+                st_times.append(dec.stage_times())
+        torch.cuda.synchronize()
+        barrier()
+        launches = dec.launches() - l0
+        ms = [a.elapsed_time(b) for a, b in ev]
+        dec.set_stage_timing(False)
+        return ms, st_times, launches
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    ms, stages, launches = timed_steps(args.mode, args.steps, args.warmup, stages=True)
+    clocks = sampler.stop()
+    ms_step = statistics.mean(ms)
+    if dist is not None:
+        t = torch.tensor([ms_step], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_step = float(t.item())
+    value = n * ws / (ms_step / 1e3)
+    bucket_ms = statistics.mean(s[0] for s in stages)
+    decode_ms = statistics.mean(s[1] for s in stages)
+
+    # roofline of the dominant kernel (the gather-decode)
+    peak, peak_kind = peaks()
+    w_bytes = w.assets.num_decoders * (64 * 16 + 64 * 64 + 8 * 64) * 2
+    alg_bytes = n * BYTES_PER_QUERY + w_bytes
+    achieved = alg_bytes / (decode_ms / 1e3) / 1e9
+    kernel_tag = f"{args.mode}-{args.precision}"
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": recorded_traffic(kernel_tag),
+                "kernel": "gather-decode (" + ("tcgen05" if args.mode == "bucketed" and args.precision != "fp32"
+                                               else args.mode) + ")",
+                "kernel_ms": decode_ms, "bucketing_ms": bucket_ms,
+                "peak_kind": f"{peak_kind} HBM copy bandwidth",
+                "algorithmic_bytes_per_launch": alg_bytes}
+
+    # end to end through the public host-buffer call
+    hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
+    hout = torch.empty((n, C), dtype=torch.float32).pin_memory()
+    for _ in range(2):
+        dec.decode_host(hq, hout, mode=args.mode)
+    e2e_t = []
+    for _ in range(max(3, min(args.steps, 10))):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dec.decode_host(hq, hout, mode=args.mode)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_ms = 1e3 * statistics.mean(e2e_t)
+    e2e = {"value": n * ws / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": n * 16,
+           "d2h_bytes_per_step": n * C * 4, "ms_per_step": e2e_ms}
+
+    # the in-run comparison: the unsorted divergent kernel on the same batch
+    extra = {}
+    if args.mode != "divergent" and args.precision != "fp32":
+        dms, _, _ = timed_steps("divergent", max(5, args.steps // 2), 2)
+        extra["divergent"] = {"value": n * ws / (statistics.mean(dms) / 1e3), "unit": UNIT,
+                              "ms_per_step": statistics.mean(dms)}
+    dd = mean_distinct(w.queries, w.assets)
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f16" if args.precision == "fp16" else args.precision.replace("fp", "f"),
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD if not args.small else "config2-small", "queries_per_gpu": n,
+                   "decoders": w.assets.num_decoders, "mode": args.mode, "precision": args.precision,
+                   "mean_distinct_decoders_per_warp": dd,
+                   "l2": "flushed before every timed step (256 MiB write, outside the step events)",
+                   "parallelism": f"{ws} independent replicas (queries sharded, no collective)"},
+        "roofline": roofline, "e2e": e2e, "gpu_launches": launches, "clocks": clocks,
+        "flops_per_query": FLOPS_PER_QUERY,
+        **extra,
+    }
+
+    if not args.no_sweep and not args.small and rank == 0:
+        result["sweep"] = sweep(ntc, torch, args.precision)
+
+    if rank == 0 and not args.no_cpu and ws == 1:
+        result["cpu_baseline"] = cpu_baseline(w)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def sweep(ntc, torch, precision):
+    """Queries/s vs exactly d distinct decoders per warp (32 sets of 1024^2, 32
+    decoders, identity map, 4096^2 texel-centre raster), bucketed vs divergent."""
+    from paper_2608_27888_gb300 import workloads as W
+    rows = []
+    a = None
+    for d in (1, 2, 4, 8, 16, 32):
+        wl = W.sweep(d, 4096)
+        if a is None:
+            a = wl.assets
+            dec = ntc.Decoder(a, precision)
+        qd = ntc.queries_to_device(wl.queries)
+        out = torch.empty((len(wl.queries), a.out_dim), dtype=torch.float32, device="cuda")
+        flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+        row = {"d": d}
+        for mode in ("bucketed", "divergent"):
+            for _ in range(2):
+                dec.decode(qd, out, mode=mode)
+            ts = []
+            for _ in range(5):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                dec.decode(qd, out, mode=mode)
+                e1.record()
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            row[mode] = len(wl.queries) / (statistics.mean(ts) / 1e3)
+        row["bucketed_over_divergent"] = row["bucketed"] / row["divergent"]
+        rows.append(row)
+        del qd, out, flush
+    dec.close()
+    return rows
+
+
+def cpu_baseline(w):
+    import oracle
+    cores = os.cpu_count() or 1
+    n = len(w.queries)
+    t0 = time.perf_counter()
+    oracle.decode(w.assets, w.queries, nthreads=cores)
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"all {n:,} queries of one step (full workload), oracle on {cores} host threads, {dt:.1f} s"}
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,203 @@
+/*
+ * ntc.h -- C ABI of libntc, the GB300 (sm_103a) runtime decoder for
+ * neural-compressed textures with shared decoders.
+ *
+ * Problem (Sec. 2 and Sec. 3.3 of "Thread-Efficient Decoding for Neural
+ * Texture Compression"): every pixel of a rendering pass asks for a texel of
+ * some texture set i; the texel is x^_i = D_{c(i)}(z_i), the latents z_i of
+ * that set decoded by the MLP decoder D_g of the set's group g = c(i) (one
+ * decoder per set in the non-shared baseline, one per cluster, or one shared by
+ * all sets).  When one warp holds queries of several decoders it diverges
+ * (Sec. 2); libntc removes that divergence by bucketing the queries by decoder
+ * before the tensor-core decode, and keeps an unsorted "divergent" decode as
+ * the comparison the paper measures (Sec. 4.4, Tables 5-6).
+ *
+ * Reading of the decode (the paper leaves the sampling rule open):
+ *   - the MLP input is the concatenation of bilinear fetches from
+ *     `num_levels` latent grids (Sec. 1: "latent pyramids or grids"), each an
+ *     8-channel fp16 grid with its own box-filtered mip chain;
+ *   - texel-centre convention x = u*W - 0.5; address_mode 0 wraps u to [0,1)
+ *     and indices modulo W, 1 clamps indices to [0, W-1];
+ *   - mip: lambda = max(lod, 0), lo = min(floor(lambda), num_mips-1),
+ *     t = lambda - lo unless lo is the last mip (then t = 0); with t > 0 the
+ *     level feature is (1-t) f(lo) + t f(lo+1) (one MLP evaluation);
+ *   - address and weight arithmetic is fp32 round-to-nearest without
+ *     contraction, so texel indices and bilinear weights are reproducible
+ *     bit for bit;
+ *   - decoder: 3-layer MLP (Sec. 4: first two layers hidden), ReLU on the
+ *     hidden layers, sigmoid on the output, fp32 out.
+ *
+ * Memory: the context owns device copies of latents, weights and map.  Query
+ * and output buffers of ntc_decode are DEVICE pointers owned by the caller.
+ * Scratch (bucket counts, permutation, sorted queries) is owned by the context
+ * and grows on demand with cudaMallocAsync on the call's stream.  One context
+ * must not run two decodes concurrently (on different streams or threads).
+ *
+ * Errors: host-detectable problems return a status and enqueue nothing; the
+ * message is available from ntc_last_error().  A query whose set id is out of
+ * range or whose u or v is not finite decodes to NaN in every channel and is
+ * counted (ntc_get_error_count).  No kernel traps.
+ */
+#ifndef NTC_H
+#define NTC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define NTC_API __attribute__((visibility("default")))
+#else
+#define NTC_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct ntc_ctx ntc_ctx;
+
+typedef enum {
+  NTC_OK = 0,
+  NTC_ERR_INVALID_ARG = 1,   /* null pointer, inconsistent sizes, bad map entry */
+  NTC_ERR_UNSUPPORTED = 2,   /* a shape or mode this build does not implement  */
+  NTC_ERR_OUT_OF_MEMORY = 3, /* a device allocation failed                     */
+  NTC_ERR_CUDA = 4           /* any other CUDA runtime error                   */
+} ntc_status;
+
+/* One decode query, 16 bytes, in device memory: texture-set id, UV, lod. */
+typedef struct {
+  uint32_t set_id;
+  float u, v;
+  float lod;
+} ntc_query;
+
+/* Arithmetic of the MLP.  TC_*: tensor cores with fp16/bf16 operands and fp32
+ * accumulation; FP32: CUDA-core fp32 reference mode. Features, bilinear
+ * weights, bias, sigmoid and the output are fp32 in every mode. */
+typedef enum {
+  NTC_PREC_TC_FP16 = 0,
+  NTC_PREC_TC_BF16 = 1,
+  NTC_PREC_FP32 = 2
+} ntc_precision;
+
+/* Which decode path ntc_decode runs.
+ * BUCKETED:     stable counting sort of the queries by decoder id, then the
+ *               gather-decode over 128-query single-decoder tiles.  Tensor-core
+ *               precisions run the tcgen05/TMEM kernel; FP32 runs FFMA.
+ * DIVERGENT:    no sorting: each warp takes 32 consecutive queries and loops over
+ *               its distinct decoders (the non-shared setting of Sec. 4.4).
+ *               Tensor-core precisions only.
+ * BUCKETED_MMA: the bucketed path with the warp-level mma.sync decode kernel.
+ *               Tensor-core precisions only. */
+typedef enum {
+  NTC_MODE_BUCKETED = 0,
+  NTC_MODE_DIVERGENT = 1,
+  NTC_MODE_BUCKETED_MMA = 2
+} ntc_mode;
+
+/* Everything ntc_create needs.  All pointers are HOST memory owned by the
+ * caller; ntc_create copies them and keeps no reference. */
+typedef struct {
+  uint32_t num_sets;          /* texture sets, >= 1                            */
+  uint32_t num_decoders;      /* decoders (groups), 1 .. NTC_MAX_DECODERS       */
+  uint32_t latent_channels;   /* channels per latent texel; must be 8           */
+  uint32_t num_levels;        /* latent grids per set; must be 2                */
+  uint32_t num_mips;          /* mip-chain length of every grid, 1 .. 16        */
+  const uint32_t *level_dims; /* [num_sets][num_levels][2]: W, H of mip 0       */
+  const uint64_t *latent_offsets; /* [num_sets][num_levels][num_mips]: first
+                                 texel of each mip in `latents` (texel units);
+                                 mip m is max(1,W>>m) x max(1,H>>m) texels,
+                                 row-major, channel-last                       */
+  const uint16_t *latents;    /* IEEE fp16 bits, [num_texels][latent_channels] */
+  uint64_t num_texels;        /* length of `latents` in texels                  */
+  uint32_t in_dim;            /* = num_levels * latent_channels (16)            */
+  uint32_t hidden;            /* hidden width: 64 or 128                        */
+  uint32_t num_hidden_layers; /* must be 2 (a 3-layer MLP)                      */
+  uint32_t out_dim;           /* output channels, 1 .. 16                       */
+  const float *weights;       /* [num_decoders][P], per decoder W1[hidden][in],
+                                 b1[hidden], W2[hidden][hidden], b2[hidden],
+                                 W3[out][hidden], b3[out] (row-major [out][in]);
+                                 P = hidden*(in+1) + hidden*(hidden+1) +
+                                 out*(hidden+1)                                 */
+  const uint32_t *set_to_decoder; /* [num_sets]: c(i), each < num_decoders      */
+  ntc_precision precision;
+  uint32_t address_mode;      /* 0 = wrap, 1 = clamp                            */
+} ntc_desc;
+
+#define NTC_MAX_DECODERS 4095u
+#define NTC_TILE_ROWS 128u
+
+/* Validate `desc`, copy latents, weights and map to the current CUDA device
+ * and return a context in *out.  Synchronous.  On failure *out is NULL. */
+NTC_API ntc_status ntc_create(const ntc_desc *desc, ntc_ctx **out);
+
+/* Decode n queries: d_out[i][c] = channel c of D_{c(set_i)}(features of query
+ * i), for c < out_dim, in the queries' original order.  d_queries: device
+ * array of n records (16-byte aligned); d_out: device array of n*out_dim
+ * floats.  Asynchronous on `cuda_stream` (a cudaStream_t; NULL is the legacy
+ * default stream); no host synchronisation.  n = 0 is a no-op.  Output for a
+ * bad query is NaN in every channel. */
+NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_out,
+                      void *cuda_stream, ntc_mode mode);
+
+/* ntc_decode on HOST buffers: copies the queries to context-owned device
+ * memory, decodes, copies the outputs back into h_out and synchronises the
+ * stream before returning.  Pinned host memory makes the copies faster. */
+NTC_API ntc_status ntc_decode_host(ntc_ctx *ctx, const ntc_query *h_queries, size_t n, float *h_out,
+                           void *cuda_stream, ntc_mode mode);
+
+/* Free the context and everything it owns.  NULL is accepted. */
+NTC_API ntc_status ntc_destroy(ntc_ctx *ctx);
+
+/* --------------------------------------------------------------- debug / test */
+
+/* Taps of every query, as the decode computes them.  d_idx: [n][num_levels][2][4]
+ * uint64 texel indices into `latents`; d_w: same shape, fp32 bilinear weights;
+ * d_t: [n] fp32 mip blend factor.  Slot [k][0] holds mip lo, slot [k][1] mip
+ * lo+1 and is filled only when t > 0 (otherwise index UINT64_MAX, weight 0);
+ * a bad query reports UINT64_MAX / 0 everywhere.  Device pointers; async. */
+NTC_API ntc_status ntc_debug_taps(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, uint64_t *d_idx,
+                          float *d_w, float *d_t, void *cuda_stream);
+
+/* The fp32 MLP input of every query, d_feat[n][in_dim] (NaN rows for bad
+ * queries).  Device pointers; async. */
+NTC_API ntc_status ntc_debug_features(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_feat,
+                              void *cuda_stream);
+
+/* The bucketing stage alone.  d_perm[n]: query indices in (decoder, original
+ * index) order, where a query with an out-of-range set id counts as decoder
+ * num_decoders.  d_counts (may be NULL): [num_decoders+1] queries per decoder.
+ * d_tiles (may be NULL): [ntc_max_tiles(ctx, n)][3] = (decoder, first position
+ * in perm, length) of every 128-query tile, in decoder order; d_num_tiles (may
+ * be NULL): [1] the number of tiles written.  Device pointers; async. */
+NTC_API ntc_status ntc_debug_bucket(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, uint32_t *d_perm,
+                            uint32_t *d_counts, uint32_t *d_tiles, uint32_t *d_num_tiles,
+                            void *cuda_stream);
+
+/* Upper bound on the number of 128-query tiles of n queries. */
+NTC_API size_t ntc_max_tiles(const ntc_ctx *ctx, size_t n);
+
+/* Number of bad queries decoded since creation or the last reset.  Synchronises
+ * the device. */
+NTC_API ntc_status ntc_get_error_count(ntc_ctx *ctx, uint64_t *count);
+NTC_API ntc_status ntc_reset_error_count(ntc_ctx *ctx);
+
+/* Stage timing.  When enabled, ntc_decode records CUDA events on its stream
+ * before bucketing, between bucketing and the gather-decode, and after it.
+ * ntc_stage_times waits for the last decode and returns, in milliseconds,
+ * times[0] = bucketing (0 in divergent mode) and times[1] = gather-decode. */
+NTC_API ntc_status ntc_set_stage_timing(ntc_ctx *ctx, int enable);
+NTC_API ntc_status ntc_stage_times(ntc_ctx *ctx, float times[2]);
+
+/* Kernels this context has launched since creation (host-side counter). */
+NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
+
+/* Human-readable message of the last failed call on this host thread. */
+NTC_API const char *ntc_last_error(void);
+NTC_API const char *ntc_status_string(ntc_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NTC_H */

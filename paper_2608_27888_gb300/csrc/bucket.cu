@@ -1,0 +1,261 @@
+// Query bucketing: a stable counting sort of the queries by decoder id.
+//
+// Sec. 2 of the paper defines divergence as several decoders being needed by
+// the queries of one block; sorting the queries by decoder (stable, so each
+// bucket keeps the original order) turns the interleaved stream into runs of
+// single-decoder 128-query tiles.  Three kernels, no inter-CTA waiting:
+//   k_hist    per-chunk histogram; each warp of a chunk owns a contiguous range
+//             and counts it with __match_any_sync (one leader per decoder run)
+//   k_scan    one CTA per decoder scans that decoder's per-chunk counts; the last
+//             CTA to finish (atomic ticket) scans the decoder totals into the
+//             segment starts and the tile starts
+//   k_scatter recomputes each warp's counts, turns them into running bases and
+//             writes perm[] and the sorted query records
+// A query whose set id is out of range goes to the extra bucket D.
+#include "ntc_internal.cuh"
+
+namespace ntc {
+namespace {
+
+constexpr int kWarps = kBucketThreads / 32;
+
+__device__ __forceinline__ uint32_t decoder_of(const Assets &A, uint32_t set_id) {
+  return set_id < A.num_sets ? __ldg(A.map + set_id) : A.num_decoders;
+}
+
+__global__ void __launch_bounds__(kBucketThreads) k_hist(Assets A, const ntc_query *q, size_t n,
+                                                         uint32_t *counts, uint32_t chunks) {
+  extern __shared__ uint32_t cnt[];  // [kWarps][D+1]
+  const uint32_t D1 = A.num_decoders + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
+  __syncthreads();
+  const size_t base = (size_t)blockIdx.x * kBucketChunk + (size_t)warp * (kBucketItems * 32);
+  uint32_t dec[kBucketItems];
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) {
+    size_t i = base + (size_t)it * 32 + lane;
+    dec[it] = i < n ? decoder_of(A, __ldg(&q[i].set_id)) : 0xFFFFFFFFu;
+  }
+  uint32_t *my = cnt + warp * D1;
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) {
+    const uint32_t d = dec[it];
+    const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
+    if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
+    __syncwarp();
+  }
+  __syncthreads();
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
+    uint32_t s = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) s += cnt[w * D1 + d];
+    counts[(size_t)d * chunks + blockIdx.x] = s;
+  }
+}
+
+// Exclusive scan of one value per thread over a 1024-thread block.
+__device__ __forceinline__ uint32_t block_scan_1024(uint32_t v, uint32_t &total, uint32_t *ws) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) ws[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t s = ws[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint32_t y = __shfl_up_sync(0xFFFFFFFFu, s, o);
+      if (lane >= o) s += y;
+    }
+    ws[lane] = s;
+  }
+  __syncthreads();
+  uint32_t excl = x - v + (warp > 0 ? ws[warp - 1] : 0u);
+  total = ws[31];
+  __syncthreads();
+  return excl;
+}
+
+// Scan `len` values in place (exclusive) with 1024 threads, 4 per thread per
+// round; returns the total.
+__device__ uint32_t block_scan_inplace(uint32_t *a, uint32_t len, uint32_t *ws) {
+  uint32_t carry = 0;
+  for (uint32_t b = 0; b < len; b += 4096) {
+    uint32_t v[4], s = 0;
+    const uint32_t i0 = b + threadIdx.x * 4;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      v[j] = i0 + j < len ? a[i0 + j] : 0u;
+      s += v[j];
+    }
+    uint32_t tot;
+    uint32_t e = block_scan_1024(s, tot, ws) + carry;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (i0 + j < len) a[i0 + j] = e;
+      e += v[j];
+    }
+    carry += tot;
+  }
+  return carry;
+}
+
+// meta layout: [0] num_tiles, [1 .. D+2] seg_start, [D+3 .. 2D+4] tile_start;
+// ticket: one word, zero between calls.
+__global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks, uint32_t D,
+                                               uint32_t n, uint32_t *totals, uint32_t *meta,
+                                               uint32_t *ticket) {
+  __shared__ uint32_t ws[32];
+  __shared__ bool last;
+  const uint32_t d = blockIdx.x;
+  uint32_t tot = block_scan_inplace(counts + (size_t)d * chunks, chunks, ws);
+  if (threadIdx.x == 0) {
+    totals[d] = tot;
+    __threadfence();
+    last = atomicAdd(ticket, 1u) == D;  // gridDim.x == D + 1
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  uint32_t *seg = meta + 1, *tst = meta + 1 + (D + 2);
+  // segment starts and tile starts over the D+1 buckets
+  for (uint32_t i = threadIdx.x; i < D + 1; i += blockDim.x) {
+    uint32_t c = ((volatile uint32_t *)totals)[i];
+    seg[i] = c;
+    tst[i] = (c + kTile - 1) / kTile;
+  }
+  __syncthreads();
+  uint32_t ns = block_scan_inplace(seg, D + 1, ws);
+  __syncthreads();
+  uint32_t nt = block_scan_inplace(tst, D + 1, ws);
+  if (threadIdx.x == 0) {
+    seg[D + 1] = ns;  // == n
+    tst[D + 1] = nt;
+    meta[0] = nt;
+    *ticket = 0;
+  }
+  (void)n;
+}
+
+__global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_query *q, size_t n,
+                                                            const uint32_t *counts, uint32_t chunks,
+                                                            const uint32_t *meta, uint32_t *perm,
+                                                            ntc_query *sorted) {
+  extern __shared__ uint32_t cnt[];  // [kWarps][D+1]
+  const uint32_t D1 = A.num_decoders + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
+  __syncthreads();
+  const size_t base = (size_t)blockIdx.x * kBucketChunk + (size_t)warp * (kBucketItems * 32);
+  uint4 rec[kBucketItems];
+  uint32_t dec[kBucketItems];
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) {
+    size_t i = base + (size_t)it * 32 + lane;
+    if (i < n) {
+      rec[it] = __ldg(reinterpret_cast<const uint4 *>(q + i));
+      dec[it] = decoder_of(A, rec[it].x);
+    } else {
+      dec[it] = 0xFFFFFFFFu;
+    }
+  }
+  uint32_t *my = cnt + warp * D1;
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) {
+    const uint32_t d = dec[it];
+    const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
+    if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
+    __syncwarp();
+  }
+  __syncthreads();
+  // running base of (warp, decoder) = segment start + this chunk's offset in
+  // the decoder's segment + the counts of the earlier warps of this chunk
+  const uint32_t *seg = meta + 1;
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
+    uint32_t run = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      uint32_t c = cnt[w * D1 + d];
+      cnt[w * D1 + d] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+  const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) {
+    const uint32_t d = dec[it];
+    const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
+    if (d != 0xFFFFFFFFu) {
+      uint32_t pos = my[d] + __popc(m & lt);
+      size_t i = base + (size_t)it * 32 + lane;
+      perm[pos] = (uint32_t)i;
+      reinterpret_cast<uint4 *>(sorted)[pos] = rec[it];
+    }
+    __syncwarp();
+    if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
+    __syncwarp();
+  }
+}
+
+__global__ void k_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,
+                               uint32_t *counts, size_t max_tiles) {
+  const uint32_t T = meta[0];
+  const size_t stride = (size_t)gridDim.x * blockDim.x;
+  for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < max_tiles; t += stride) {
+    if (tiles && t < T) {
+      uint32_t dec, start, len;
+      tile_info(meta, D, (uint32_t)t, dec, start, len);
+      tiles[3 * t] = dec;
+      tiles[3 * t + 1] = start;
+      tiles[3 * t + 2] = len;
+    }
+    if (counts && t < D + 1) counts[t] = meta[1 + t + 1] - meta[1 + t];
+  }
+  if (num_tiles && blockIdx.x == 0 && threadIdx.x == 0) *num_tiles = T;
+}
+
+}  // namespace
+
+size_t bucket_scratch_counts(uint32_t D, size_t n) {
+  size_t chunks = (n + kBucketChunk - 1) / kBucketChunk;
+  return (size_t)(D + 1) * chunks;
+}
+
+cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
+                          cudaStream_t st, int *launches) {
+  const uint32_t chunks = (uint32_t)((n + kBucketChunk - 1) / kBucketChunk);
+  const uint32_t D = A.num_decoders;
+  const size_t smem = (size_t)kWarps * (D + 1) * sizeof(uint32_t);
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaFuncSetAttribute(k_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    cudaFuncSetAttribute(k_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    attr_done = true;
+  }
+  // totals[D+1] and the ticket live after meta
+  uint32_t *totals = s.meta + meta_words(D);
+  uint32_t *ticket = totals + (D + 1);
+  k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks);
+  k_scan<<<D + 1, 1024, 0, st>>>(s.counts, chunks, D, (uint32_t)n, totals, s.meta, ticket);
+  k_scatter<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks, s.meta, s.perm, s.sorted);
+  *launches += 3;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,
+                                uint32_t *counts, size_t max_tiles, cudaStream_t st, int *launches) {
+  size_t work = max_tiles > (size_t)D + 1 ? max_tiles : (size_t)D + 1;
+  unsigned blocks = (unsigned)((work + 255) / 256);
+  if (blocks > 4096) blocks = 4096;
+  k_tiles_export<<<blocks, 256, 0, st>>>(meta, D, tiles, num_tiles, counts, work);
+  *launches += 1;
+  return cudaGetLastError();
+}
+
+}  // namespace ntc

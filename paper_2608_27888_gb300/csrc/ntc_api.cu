@@ -1,0 +1,476 @@
+// The C ABI of libntc (declared in include/ntc.h): argument validation, device
+// copies of the assets, scratch management and the launch sequence of each
+// decode path.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <vector>
+
+#include "ntc_internal.cuh"
+
+using namespace ntc;
+
+struct ntc_ctx {
+  int device = 0;
+  int num_sms = 0;
+  uint32_t S = 0, D = 0, M = 0, H = 0, C = 0, address_mode = 0;
+  ntc_precision prec = NTC_PREC_TC_FP16;
+  uint64_t num_texels = 0;
+  uint4 *d_lat = nullptr;
+  GridDesc *d_grids = nullptr;
+  uint32_t *d_map = nullptr;
+  uint8_t *d_mma = nullptr;
+  float *d_f32 = nullptr;
+  uint8_t *d_tc = nullptr;
+  size_t mma_stride = 0, f32_stride = 0, tc_stride = 0;
+  unsigned long long *d_err = nullptr;
+  // bucketing scratch (grows on demand, stream-ordered)
+  size_t cap_n = 0, cap_counts = 0;
+  uint32_t *d_counts = nullptr, *d_perm = nullptr, *d_meta = nullptr;
+  ntc_query *d_sorted = nullptr;
+  // staging for ntc_decode_host
+  size_t cap_host = 0;
+  ntc_query *d_hq = nullptr;
+  float *d_hout = nullptr;
+  uint64_t launches = 0;
+  // optional stage timing
+  bool timing = false;
+  bool timed = false;
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+};
+
+static thread_local char g_err[512] = "";
+
+static ntc_status fail(ntc_status s, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof g_err, fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+static ntc_status cuda_fail(cudaError_t e, const char *what) {
+  if (e == cudaErrorMemoryAllocation)
+    return fail(NTC_ERR_OUT_OF_MEMORY, "%s: %s", what, cudaGetErrorString(e));
+  return fail(NTC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define CK(call, what)                            \
+  do {                                            \
+    cudaError_t e_ = (call);                      \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+namespace {
+
+// Keeps the caller's current device and restores it.
+struct DeviceGuard {
+  int prev = -1;
+  bool ok = true;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    int now = -1;
+    if (prev >= 0 && cudaGetDevice(&now) == cudaSuccess && now != prev) cudaSetDevice(prev);
+  }
+};
+
+Assets assets_of(const ntc_ctx *c) {
+  Assets A;
+  A.lat = c->d_lat;
+  A.grids = c->d_grids;
+  A.map = c->d_map;
+  A.num_sets = c->S;
+  A.num_decoders = c->D;
+  A.num_mips = c->M;
+  A.address_mode = c->address_mode;
+  return A;
+}
+
+WeightImages weights_of(const ntc_ctx *c) {
+  WeightImages W;
+  W.mma = c->d_mma;
+  W.mma_stride = c->mma_stride;
+  W.f32 = c->d_f32;
+  W.f32_stride = c->f32_stride;
+  W.tc = c->d_tc;
+  W.tc_stride = c->tc_stride;
+  W.hidden = c->H;
+  W.out_dim = c->C;
+  return W;
+}
+
+void release(ntc_ctx *c) {
+  for (auto &e : c->ev)
+    if (e) cudaEventDestroy(e);
+  cudaFree(c->d_lat);
+  cudaFree(c->d_grids);
+  cudaFree(c->d_map);
+  cudaFree(c->d_mma);
+  cudaFree(c->d_f32);
+  cudaFree(c->d_tc);
+  cudaFree(c->d_err);
+  cudaFree(c->d_counts);
+  cudaFree(c->d_perm);
+  cudaFree(c->d_sorted);
+  cudaFree(c->d_meta);
+  cudaFree(c->d_hq);
+  cudaFree(c->d_hout);
+}
+
+size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
+
+// Make sure the bucketing scratch holds n queries (stream-ordered allocation).
+ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
+  const size_t chunks = (n + kBucketChunk - 1) / kBucketChunk;
+  const size_t counts = (size_t)(c->D + 1) * (chunks ? chunks : 1);
+  if (!c->d_meta) {
+    const size_t words = meta_words(c->D) + (c->D + 1) + 1;
+    CK(cudaMallocAsync((void **)&c->d_meta, words * 4, st), "scratch allocation");
+    CK(cudaMemsetAsync(c->d_meta, 0, words * 4, st), "scratch clear");
+  }
+  if (counts > c->cap_counts) {
+    if (c->d_counts) CK(cudaFreeAsync(c->d_counts, st), "scratch free");
+    c->d_counts = nullptr;
+    c->cap_counts = 0;
+    CK(cudaMallocAsync((void **)&c->d_counts, counts * 4, st), "scratch allocation");
+    c->cap_counts = counts;
+  }
+  if (n > c->cap_n) {
+    if (c->d_perm) CK(cudaFreeAsync(c->d_perm, st), "scratch free");
+    if (c->d_sorted) CK(cudaFreeAsync(c->d_sorted, st), "scratch free");
+    c->d_perm = nullptr;
+    c->d_sorted = nullptr;
+    c->cap_n = 0;
+    CK(cudaMallocAsync((void **)&c->d_perm, n * 4, st), "scratch allocation");
+    CK(cudaMallocAsync((void **)&c->d_sorted, n * sizeof(ntc_query), st), "scratch allocation");
+    c->cap_n = n;
+  }
+  return NTC_OK;
+}
+
+Scratch scratch_of(const ntc_ctx *c) {
+  Scratch s;
+  s.counts = c->d_counts;
+  s.perm = c->d_perm;
+  s.sorted = c->d_sorted;
+  s.meta = c->d_meta;
+  return s;
+}
+
+ntc_status check_queries(const ntc_ctx *ctx, const void *q, size_t n) {
+  if (!ctx) return fail(NTC_ERR_INVALID_ARG, "null context");
+  if (n > 0xFFFFFF00ull) return fail(NTC_ERR_INVALID_ARG, "n = %zu exceeds 2^32 - 256 queries", n);
+  if (n && !q) return fail(NTC_ERR_INVALID_ARG, "null query pointer");
+  if (((uintptr_t)q & 15) != 0) return fail(NTC_ERR_INVALID_ARG, "query buffer is not 16-byte aligned");
+  return NTC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *ntc_last_error(void) { return g_err; }
+
+const char *ntc_status_string(ntc_status s) {
+  switch (s) {
+    case NTC_OK: return "ok";
+    case NTC_ERR_INVALID_ARG: return "invalid argument";
+    case NTC_ERR_UNSUPPORTED: return "unsupported";
+    case NTC_ERR_OUT_OF_MEMORY: return "out of memory";
+    case NTC_ERR_CUDA: return "CUDA error";
+  }
+  return "unknown status";
+}
+
+ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
+  if (!out) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
+  *out = nullptr;
+  if (!d) return fail(NTC_ERR_INVALID_ARG, "null descriptor");
+  if (!d->level_dims || !d->latent_offsets || !d->latents || !d->weights || !d->set_to_decoder)
+    return fail(NTC_ERR_INVALID_ARG, "null array in descriptor");
+  if (d->num_sets < 1) return fail(NTC_ERR_INVALID_ARG, "num_sets must be >= 1");
+  if (d->num_decoders < 1 || d->num_decoders > NTC_MAX_DECODERS)
+    return fail(NTC_ERR_INVALID_ARG, "num_decoders must be in 1..%u", NTC_MAX_DECODERS);
+  if (d->latent_channels != kChannels)
+    return fail(NTC_ERR_UNSUPPORTED, "latent_channels must be %d", kChannels);
+  if (d->num_levels != kLevels) return fail(NTC_ERR_UNSUPPORTED, "num_levels must be %d", kLevels);
+  if (d->num_mips < 1 || d->num_mips > kMaxMips)
+    return fail(NTC_ERR_INVALID_ARG, "num_mips must be in 1..%d", kMaxMips);
+  if (d->in_dim != kInDim) return fail(NTC_ERR_INVALID_ARG, "in_dim must be num_levels * latent_channels");
+  if (d->hidden != 64 && d->hidden != 128) return fail(NTC_ERR_UNSUPPORTED, "hidden must be 64 or 128");
+  if (d->num_hidden_layers != 2) return fail(NTC_ERR_UNSUPPORTED, "num_hidden_layers must be 2");
+  if (d->out_dim < 1 || d->out_dim > 16) return fail(NTC_ERR_UNSUPPORTED, "out_dim must be in 1..16");
+  if (d->precision != NTC_PREC_TC_FP16 && d->precision != NTC_PREC_TC_BF16 && d->precision != NTC_PREC_FP32)
+    return fail(NTC_ERR_INVALID_ARG, "unknown precision");
+  if (d->address_mode > 1) return fail(NTC_ERR_INVALID_ARG, "address_mode must be 0 (wrap) or 1 (clamp)");
+  if (d->num_texels < 1) return fail(NTC_ERR_INVALID_ARG, "num_texels must be >= 1");
+  const uint32_t S = d->num_sets, M = d->num_mips;
+  std::vector<GridDesc> grids((size_t)S * kLevels * M);
+  for (uint32_t s = 0; s < S; ++s)
+    for (uint32_t k = 0; k < kLevels; ++k) {
+      const uint32_t W0 = d->level_dims[((size_t)s * kLevels + k) * 2];
+      const uint32_t H0 = d->level_dims[((size_t)s * kLevels + k) * 2 + 1];
+      if (W0 < 1 || H0 < 1 || W0 > (1u << 24) || H0 > (1u << 24) || (uint64_t)W0 * H0 > 0xFFFFFFFFull)
+        return fail(NTC_ERR_INVALID_ARG, "set %u level %u: bad grid size %ux%u", s, k, W0, H0);
+      for (uint32_t m = 0; m < M; ++m) {
+        const uint32_t W = W0 >> m ? W0 >> m : 1, H = H0 >> m ? H0 >> m : 1;
+        const uint64_t base = d->latent_offsets[((size_t)s * kLevels + k) * M + m];
+        if (base > d->num_texels || (uint64_t)W * H > d->num_texels - base)
+          return fail(NTC_ERR_INVALID_ARG, "set %u level %u mip %u lies outside the latents", s, k, m);
+        GridDesc &g = grids[((size_t)s * kLevels + k) * M + m];
+        g.base = base;
+        g.W = W;
+        g.H = H;
+      }
+    }
+  for (uint32_t s = 0; s < S; ++s)
+    if (d->set_to_decoder[s] >= d->num_decoders)
+      return fail(NTC_ERR_INVALID_ARG, "set_to_decoder[%u] = %u is not a decoder", s, d->set_to_decoder[s]);
+
+  ntc_ctx *c = new ntc_ctx;
+  if (cudaGetDevice(&c->device) != cudaSuccess) {
+    delete c;
+    return fail(NTC_ERR_CUDA, "no CUDA device");
+  }
+  cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+  c->S = S;
+  c->D = d->num_decoders;
+  c->M = M;
+  c->H = d->hidden;
+  c->C = d->out_dim;
+  c->address_mode = d->address_mode;
+  c->prec = d->precision;
+  c->num_texels = d->num_texels;
+  const size_t P = (size_t)c->H * (kInDim + 1) + (size_t)c->H * (c->H + 1) + (size_t)c->C * (c->H + 1);
+  c->mma_stride = round16(mma_image_bytes(c->H));
+  c->f32_stride = (f32_image_floats(c->H, c->C) + 3) & ~(size_t)3;
+  c->tc_stride = round16(tc_image_bytes(c->H));
+  float *d_w32 = nullptr;
+  cudaError_t e = cudaSuccess;
+  auto step = [&](cudaError_t r) {
+    if (e == cudaSuccess) e = r;
+  };
+  step(cudaMalloc((void **)&c->d_lat, d->num_texels * 16));
+  step(cudaMalloc((void **)&c->d_grids, grids.size() * sizeof(GridDesc)));
+  step(cudaMalloc((void **)&c->d_map, (size_t)S * 4));
+  step(cudaMalloc((void **)&c->d_mma, c->mma_stride * c->D));
+  step(cudaMalloc((void **)&c->d_f32, c->f32_stride * 4 * c->D));
+  step(cudaMalloc((void **)&c->d_tc, c->tc_stride * c->D));
+  step(cudaMalloc((void **)&c->d_err, sizeof(unsigned long long)));
+  step(cudaMalloc((void **)&d_w32, P * 4 * c->D));
+  if (e == cudaSuccess) {
+    step(cudaMemcpy(c->d_lat, d->latents, d->num_texels * 16, cudaMemcpyHostToDevice));
+    step(cudaMemcpy(c->d_grids, grids.data(), grids.size() * sizeof(GridDesc), cudaMemcpyHostToDevice));
+    step(cudaMemcpy(c->d_map, d->set_to_decoder, (size_t)S * 4, cudaMemcpyHostToDevice));
+    step(cudaMemcpy(d_w32, d->weights, P * 4 * c->D, cudaMemcpyHostToDevice));
+    step(cudaMemset(c->d_err, 0, sizeof(unsigned long long)));
+    step(cudaMemset(c->d_tc, 0, c->tc_stride * c->D));
+    step(launch_pack_weights(d_w32, c->D, c->H, c->C, c->prec == NTC_PREC_TC_BF16, c->d_mma,
+                             c->mma_stride, c->d_f32, c->f32_stride, c->d_tc, c->tc_stride, 0));
+    step(cudaDeviceSynchronize());
+  }
+  cudaFree(d_w32);
+  if (e != cudaSuccess) {
+    release(c);
+    delete c;
+    return cuda_fail(e, "ntc_create");
+  }
+  *out = c;
+  return NTC_OK;
+}
+
+ntc_status ntc_destroy(ntc_ctx *c) {
+  if (!c) return NTC_OK;
+  DeviceGuard g(c->device);
+  cudaDeviceSynchronize();
+  release(c);
+  delete c;
+  return NTC_OK;
+}
+
+ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream,
+                      ntc_mode mode) {
+  ntc_status s = check_queries(c, q, n);
+  if (s != NTC_OK) return s;
+  if (n && !out) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
+  if (((uintptr_t)out & 3) != 0) return fail(NTC_ERR_INVALID_ARG, "output buffer is not 4-byte aligned");
+  if (mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT && mode != NTC_MODE_BUCKETED_MMA)
+    return fail(NTC_ERR_INVALID_ARG, "unknown mode");
+  const bool fp32 = c->prec == NTC_PREC_FP32;
+  if (fp32 && mode != NTC_MODE_BUCKETED)
+    return fail(NTC_ERR_UNSUPPORTED, "the fp32 precision has only the bucketed mode");
+  if (n == 0) return NTC_OK;
+  DeviceGuard g(c->device);
+  if (!g.ok) return fail(NTC_ERR_CUDA, "cannot select the context's device");
+  cudaStream_t st = (cudaStream_t)stream;
+  const Assets A = assets_of(c);
+  const WeightImages W = weights_of(c);
+  const bool bf16 = c->prec == NTC_PREC_TC_BF16;
+  int launches = 0;
+  cudaError_t e;
+  s = mode == NTC_MODE_DIVERGENT ? NTC_OK : ensure_scratch(c, n, st);
+  if (s != NTC_OK) return s;
+  if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
+  if (mode == NTC_MODE_DIVERGENT) {
+    if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
+    e = launch_decode_divergent(A, W, q, n, out, c->d_err, bf16, c->num_sms, st, &launches);
+    c->launches += launches;
+    if (e != cudaSuccess) return cuda_fail(e, "divergent decode launch");
+    if (c->timing) {
+      CK(cudaEventRecord(c->ev[2], st), "event record");
+      c->timed = true;
+    }
+    return NTC_OK;
+  }
+  e = launch_bucket(A, q, n, scratch_of(c), st, &launches);
+  if (e != cudaSuccess) {
+    c->launches += launches;
+    return cuda_fail(e, "bucketing launch");
+  }
+  Buckets B;
+  B.sorted = c->d_sorted;
+  B.perm = c->d_perm;
+  B.meta = c->d_meta;
+  if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
+  if (fp32)
+    e = launch_decode_fp32(A, W, B, n, out, c->d_err, c->num_sms, st, &launches);
+  else
+    e = launch_decode_mma(A, W, B, n, out, c->d_err, bf16, c->num_sms, st, &launches);
+  c->launches += launches;
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+  if (c->timing) {
+    CK(cudaEventRecord(c->ev[2], st), "event record");
+    c->timed = true;
+  }
+  return NTC_OK;
+}
+
+ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hout, void *stream,
+                           ntc_mode mode) {
+  ntc_status s = check_queries(c, hq, n);
+  if (s != NTC_OK) return s;
+  if (n && !hout) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
+  if (n == 0) return NTC_OK;
+  DeviceGuard g(c->device);
+  cudaStream_t st = (cudaStream_t)stream;
+  if (n > c->cap_host) {
+    CK(cudaStreamSynchronize(st), "staging resize");
+    cudaFree(c->d_hq);
+    cudaFree(c->d_hout);
+    c->d_hq = nullptr;
+    c->d_hout = nullptr;
+    c->cap_host = 0;
+    CK(cudaMalloc((void **)&c->d_hq, n * sizeof(ntc_query)), "staging allocation");
+    CK(cudaMalloc((void **)&c->d_hout, n * c->C * sizeof(float)), "staging allocation");
+    c->cap_host = n;
+  }
+  CK(cudaMemcpyAsync(c->d_hq, hq, n * sizeof(ntc_query), cudaMemcpyHostToDevice, st), "query upload");
+  s = ntc_decode(c, c->d_hq, n, c->d_hout, stream, mode);
+  if (s != NTC_OK) return s;
+  CK(cudaMemcpyAsync(hout, c->d_hout, n * c->C * sizeof(float), cudaMemcpyDeviceToHost, st), "output download");
+  CK(cudaStreamSynchronize(st), "decode");
+  return NTC_OK;
+}
+
+ntc_status ntc_debug_taps(ntc_ctx *c, const ntc_query *q, size_t n, uint64_t *idx, float *w,
+                          float *t, void *stream) {
+  ntc_status s = check_queries(c, q, n);
+  if (s != NTC_OK) return s;
+  if (n && (!idx || !w || !t)) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
+  if (n == 0) return NTC_OK;
+  DeviceGuard g(c->device);
+  int launches = 0;
+  cudaError_t e = launch_debug_taps(assets_of(c), q, n, (unsigned long long *)idx, w, t,
+                                    (cudaStream_t)stream, &launches);
+  c->launches += launches;
+  if (e != cudaSuccess) return cuda_fail(e, "debug taps launch");
+  return NTC_OK;
+}
+
+ntc_status ntc_debug_features(ntc_ctx *c, const ntc_query *q, size_t n, float *f, void *stream) {
+  ntc_status s = check_queries(c, q, n);
+  if (s != NTC_OK) return s;
+  if (n && !f) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
+  if (n == 0) return NTC_OK;
+  DeviceGuard g(c->device);
+  int launches = 0;
+  cudaError_t e = launch_debug_features(assets_of(c), q, n, f, (cudaStream_t)stream, &launches);
+  c->launches += launches;
+  if (e != cudaSuccess) return cuda_fail(e, "debug features launch");
+  return NTC_OK;
+}
+
+size_t ntc_max_tiles(const ntc_ctx *c, size_t n) {
+  if (!c) return 0;
+  return (n + kTile - 1) / kTile + c->D + 1;
+}
+
+ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *perm,
+                            uint32_t *counts, uint32_t *tiles, uint32_t *num_tiles, void *stream) {
+  ntc_status s = check_queries(c, q, n);
+  if (s != NTC_OK) return s;
+  if (n && !perm) return fail(NTC_ERR_INVALID_ARG, "null perm pointer");
+  DeviceGuard g(c->device);
+  cudaStream_t st = (cudaStream_t)stream;
+  int launches = 0;
+  if (n == 0) {
+    if (counts) CK(cudaMemsetAsync(counts, 0, (c->D + 1) * 4, st), "clear");
+    if (num_tiles) CK(cudaMemsetAsync(num_tiles, 0, 4, st), "clear");
+    return NTC_OK;
+  }
+  s = ensure_scratch(c, n, st);
+  if (s != NTC_OK) return s;
+  cudaError_t e = launch_bucket(assets_of(c), q, n, scratch_of(c), st, &launches);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(perm, c->d_perm, n * 4, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess && (counts || tiles || num_tiles))
+    e = launch_tiles_export(c->d_meta, c->D, tiles, num_tiles, counts, ntc_max_tiles(c, n), st, &launches);
+  c->launches += launches;
+  if (e != cudaSuccess) return cuda_fail(e, "bucketing");
+  return NTC_OK;
+}
+
+ntc_status ntc_get_error_count(ntc_ctx *c, uint64_t *count) {
+  if (!c || !count) return fail(NTC_ERR_INVALID_ARG, "null argument");
+  DeviceGuard g(c->device);
+  CK(cudaDeviceSynchronize(), "synchronize");
+  unsigned long long v = 0;
+  CK(cudaMemcpy(&v, c->d_err, sizeof v, cudaMemcpyDeviceToHost), "error counter read");
+  *count = v;
+  return NTC_OK;
+}
+
+ntc_status ntc_reset_error_count(ntc_ctx *c) {
+  if (!c) return fail(NTC_ERR_INVALID_ARG, "null context");
+  DeviceGuard g(c->device);
+  CK(cudaDeviceSynchronize(), "synchronize");
+  CK(cudaMemset(c->d_err, 0, sizeof(unsigned long long)), "error counter reset");
+  return NTC_OK;
+}
+
+uint64_t ntc_launch_count(const ntc_ctx *c) { return c ? c->launches : 0; }
+
+ntc_status ntc_set_stage_timing(ntc_ctx *c, int enable) {
+  if (!c) return fail(NTC_ERR_INVALID_ARG, "null context");
+  DeviceGuard g(c->device);
+  if (enable && !c->ev[0])
+    for (auto &e : c->ev) CK(cudaEventCreate(&e), "event create");
+  c->timing = enable != 0;
+  c->timed = false;
+  return NTC_OK;
+}
+
+ntc_status ntc_stage_times(ntc_ctx *c, float times[2]) {
+  if (!c || !times) return fail(NTC_ERR_INVALID_ARG, "null argument");
+  if (!c->timed) return fail(NTC_ERR_INVALID_ARG, "no timed decode since timing was enabled");
+  DeviceGuard g(c->device);
+  CK(cudaEventSynchronize(c->ev[2]), "event synchronize");
+  CK(cudaEventElapsedTime(&times[0], c->ev[0], c->ev[1]), "event elapsed");
+  CK(cudaEventElapsedTime(&times[1], c->ev[1], c->ev[2]), "event elapsed");
+  return NTC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,247 @@
+// Internal declarations of libntc: the context, device helpers shared by the
+// kernels (tap addressing, latent gather, mma.sync fragments) and launchers.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/ntc.h"
+
+namespace ntc {
+
+constexpr int kTile = NTC_TILE_ROWS;  // rows of one single-decoder tile
+constexpr int kLevels = 2;            // latent grids per set
+constexpr int kChannels = 8;          // fp16 channels per latent texel (16 B)
+constexpr int kInDim = kLevels * kChannels;
+constexpr int kMaxMips = 16;
+
+// Base texel and dimensions of one (set, level, mip) grid.
+struct alignas(16) GridDesc {
+  unsigned long long base;
+  uint32_t W, H;
+};
+
+// Device-side view of the assets, passed by value to kernels.
+struct Assets {
+  const uint4 *lat;         // latents, one uint4 (8 x fp16) per texel
+  const GridDesc *grids;    // [num_sets][kLevels][num_mips]
+  const uint32_t *map;      // [num_sets] set -> decoder
+  uint32_t num_sets, num_decoders, num_mips, address_mode;
+};
+
+// Per-decoder weight images.
+//  mma image (fp16/bf16 bits, rows padded by 8 elements so ldmatrix is
+//  conflict-free): W1[H][16+8], W2[H][H+8], W3[16][H+8] (rows >= C zero), then
+//  fp32 biases b1[H], b2[H], b3[16].
+//  fp32 image: W1[H][16], b1[H], W2[H][H], b2[H], W3[CP][H], b3[CP] (rows >= C
+//  zero), CP = 8 or 16.
+struct WeightImages {
+  const uint8_t *mma;       // [D][mma_stride] bytes
+  size_t mma_stride;
+  const float *f32;         // [D][f32_stride] floats
+  size_t f32_stride;
+  const uint8_t *tc;        // [D][tc_stride] bytes, tcgen05 shared-memory image
+  size_t tc_stride;
+  uint32_t hidden, out_dim;
+};
+
+inline __host__ __device__ size_t mma_image_bytes(uint32_t H) {
+  return (size_t)H * (16 + 8) * 2 + (size_t)H * (H + 8) * 2 + (size_t)16 * (H + 8) * 2 +
+         (size_t)(2 * H + 16) * 4;
+}
+inline __host__ __device__ uint32_t out_pad(uint32_t C) { return C <= 8 ? 8u : 16u; }
+inline __host__ __device__ size_t f32_image_floats(uint32_t H, uint32_t C) {
+  uint32_t CP = out_pad(C);
+  return (size_t)H * 16 + H + (size_t)H * H + H + (size_t)CP * H + CP;
+}
+
+// Bucketing results on the device.
+struct Buckets {
+  const ntc_query *sorted;  // queries in (decoder, index) order
+  const uint32_t *perm;     // original index of each sorted query
+  const uint32_t *meta;     // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
+};
+inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2); }
+
+// ------------------------------------------------------------- device helpers
+
+// One axis of the tap addressing, fp32 round-to-nearest with no contraction.
+__device__ __forceinline__ void axis_taps(float c, uint32_t n, uint32_t mode, uint32_t &i0,
+                                          uint32_t &i1, float &frac) {
+  float x;
+  if (mode == 0) {
+    float cw = __fsub_rn(c, floorf(c));
+    x = __fsub_rn(__fmul_rn(cw, (float)n), 0.5f);
+  } else {
+    x = __fsub_rn(__fmul_rn(c, (float)n), 0.5f);
+  }
+  float x0f = floorf(x);
+  frac = __fsub_rn(x, x0f);
+  if (mode == 0) {
+    int x0 = (int)x0f;  // in [-1, n-1]
+    i0 = x0 < 0 ? n - 1 : (uint32_t)x0;
+    uint32_t a1 = (uint32_t)(x0 + 1);
+    i1 = a1 >= n ? a1 - n : a1;
+  } else {
+    int x0 = (int)fminf(fmaxf(x0f, -1.0f), (float)n);
+    int hi = (int)n - 1;
+    i0 = (uint32_t)min(max(x0, 0), hi);
+    i1 = (uint32_t)min(max(x0 + 1, 0), hi);
+  }
+}
+
+// Texel indices and bilinear weights of one grid (tap order 00, 10, 01, 11).
+__device__ __forceinline__ void grid_taps(const GridDesc &g, float u, float v, uint32_t mode,
+                                          unsigned long long idx[4], float w[4]) {
+  uint32_t i0, i1, j0, j1;
+  float wx, wy;
+  axis_taps(u, g.W, mode, i0, i1, wx);
+  axis_taps(v, g.H, mode, j0, j1, wy);
+  unsigned long long r0 = g.base + (unsigned long long)j0 * g.W;
+  unsigned long long r1 = g.base + (unsigned long long)j1 * g.W;
+  idx[0] = r0 + i0;
+  idx[1] = r0 + i1;
+  idx[2] = r1 + i0;
+  idx[3] = r1 + i1;
+  float ax = __fsub_rn(1.0f, wx), ay = __fsub_rn(1.0f, wy);
+  w[0] = __fmul_rn(ax, ay);
+  w[1] = __fmul_rn(wx, ay);
+  w[2] = __fmul_rn(ax, wy);
+  w[3] = __fmul_rn(wx, wy);
+}
+
+__device__ __forceinline__ bool query_bad(const Assets &A, const ntc_query &q) {
+  return q.set_id >= A.num_sets || !isfinite(q.u) || !isfinite(q.v);
+}
+
+// Mip selection: lo and blend t (t > 0 only when mip lo+1 exists).
+__device__ __forceinline__ int select_mip(float lod, uint32_t num_mips, float &t) {
+  float lam = fmaxf(lod, 0.0f);
+  float lof = fminf(floorf(lam), (float)(num_mips - 1));
+  int lo = (int)lof;
+  t = (lo == (int)num_mips - 1) ? 0.0f : __fsub_rn(lam, lof);
+  return lo;
+}
+
+__device__ __forceinline__ void accum_tap(float f[kChannels], uint4 raw, float w) {
+  const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    float2 x = __half22float2(h[p]);
+    f[2 * p] = fmaf(w, x.x, f[2 * p]);
+    f[2 * p + 1] = fmaf(w, x.y, f[2 * p + 1]);
+  }
+}
+
+// The fp32 MLP input of a (good) query: f[0..7] level 0, f[8..15] level 1.
+// All tap loads of a query are issued before any is consumed.
+__device__ __forceinline__ void query_features(const Assets &A, const ntc_query &q,
+                                               float f[kInDim]) {
+  float t;
+  int lo = select_mip(q.lod, A.num_mips, t);
+  const GridDesc *g = A.grids + (size_t)q.set_id * kLevels * A.num_mips;
+#pragma unroll
+  for (int c = 0; c < kInDim; ++c) f[c] = 0.0f;
+  if (t == 0.0f) {
+    unsigned long long idx[kLevels][4];
+    float w[kLevels][4];
+    uint4 raw[kLevels][4];
+#pragma unroll
+    for (int k = 0; k < kLevels; ++k) grid_taps(g[k * A.num_mips + lo], q.u, q.v, A.address_mode, idx[k], w[k]);
+#pragma unroll
+    for (int k = 0; k < kLevels; ++k)
+#pragma unroll
+      for (int p = 0; p < 4; ++p) raw[k][p] = __ldg(A.lat + idx[k][p]);
+#pragma unroll
+    for (int k = 0; k < kLevels; ++k)
+#pragma unroll
+      for (int p = 0; p < 4; ++p) accum_tap(f + k * kChannels, raw[k][p], w[k][p]);
+  } else {
+    float s = __fsub_rn(1.0f, t);
+#pragma unroll
+    for (int k = 0; k < kLevels; ++k) {
+      unsigned long long idx[2][4];
+      float w[2][4];
+      uint4 raw[2][4];
+      grid_taps(g[k * A.num_mips + lo], q.u, q.v, A.address_mode, idx[0], w[0]);
+      grid_taps(g[k * A.num_mips + lo + 1], q.u, q.v, A.address_mode, idx[1], w[1]);
+#pragma unroll
+      for (int m = 0; m < 2; ++m)
+#pragma unroll
+        for (int p = 0; p < 4; ++p) raw[m][p] = __ldg(A.lat + idx[m][p]);
+#pragma unroll
+      for (int p = 0; p < 4; ++p) accum_tap(f + k * kChannels, raw[0][p], w[0][p] * s);
+#pragma unroll
+      for (int p = 0; p < 4; ++p) accum_tap(f + k * kChannels, raw[1][p], w[1][p] * t);
+    }
+  }
+}
+
+__device__ __forceinline__ ntc_query load_query(const ntc_query *q) {
+  uint4 r = __ldg(reinterpret_cast<const uint4 *>(q));
+  ntc_query out;
+  out.set_id = r.x;
+  out.u = __uint_as_float(r.y);
+  out.v = __uint_as_float(r.z);
+  out.lod = __uint_as_float(r.w);
+  return out;
+}
+
+// Tile t of the bucketed order: decoder, first sorted position and length.
+__device__ __forceinline__ void tile_info(const uint32_t *meta, uint32_t D, uint32_t t,
+                                          uint32_t &dec, uint32_t &start, uint32_t &len) {
+  const uint32_t *seg = meta + 1;           // seg_start[D+2]
+  const uint32_t *tst = meta + 1 + (D + 2); // tile_start[D+2]
+  // largest d in [0, D] with tile_start[d] <= t
+  uint32_t lo = 0, hi = D + 1;
+  while (hi - lo > 1) {
+    uint32_t mid = (lo + hi) >> 1;
+    if (__ldg(tst + mid) <= t) lo = mid; else hi = mid;
+  }
+  dec = lo;
+  start = __ldg(seg + lo) + (t - __ldg(tst + lo)) * kTile;
+  uint32_t end = __ldg(seg + lo + 1);
+  len = min((uint32_t)kTile, end - start);
+}
+
+// ---------------------------------------------------------------- launchers
+
+struct Scratch {
+  uint32_t *counts;   // [(D+1) * chunks]
+  uint32_t *perm;     // [n]
+  ntc_query *sorted;  // [n]
+  uint32_t *meta;     // meta_words(D)
+};
+
+constexpr int kBucketThreads = 256;
+constexpr int kBucketItems = 16;  // queries per thread
+constexpr int kBucketChunk = kBucketThreads * kBucketItems;
+
+cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
+                          cudaStream_t st, int *launches);
+cudaError_t launch_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,
+                                uint32_t *counts, size_t max_tiles, cudaStream_t st, int *launches);
+cudaError_t launch_decode_fp32(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
+                               float *out, unsigned long long *err, int num_sms, cudaStream_t st,
+                               int *launches);
+cudaError_t launch_decode_mma(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
+                              float *out, unsigned long long *err, bool bf16, int num_sms,
+                              cudaStream_t st, int *launches);
+cudaError_t launch_decode_divergent(const Assets &A, const WeightImages &W, const ntc_query *q,
+                                    size_t n, float *out, unsigned long long *err, bool bf16,
+                                    int num_sms, cudaStream_t st, int *launches);
+cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
+                             float *out, unsigned long long *err, bool bf16, int num_sms,
+                             cudaStream_t st, int *launches);
+cudaError_t launch_debug_taps(const Assets &A, const ntc_query *q, size_t n, unsigned long long *idx,
+                              float *w, float *t, cudaStream_t st, int *launches);
+cudaError_t launch_debug_features(const Assets &A, const ntc_query *q, size_t n, float *f,
+                                  cudaStream_t st, int *launches);
+cudaError_t launch_pack_weights(const float *w32, uint32_t D, uint32_t H, uint32_t C, bool bf16,
+                                uint8_t *mma, size_t mma_stride, float *f32, size_t f32_stride,
+                                uint8_t *tc, size_t tc_stride, cudaStream_t st);
+size_t tc_image_bytes(uint32_t H);
+
+}  // namespace ntc

@@ -1,0 +1,265 @@
+"""GPU parity: libntc (through the C ABI) against the CPU oracle.
+
+Bit-exact: bucketing permutation, counts and tile list; texel indices, bilinear
+weights and mip blend factors.  Floating point: fp32 mode within 1e-5 of the
+oracle; tensor-core modes within max-abs 2e-2 and mean-abs 2e-3 (outputs are in
+[0, 1]).  Small workloads are compared everywhere; full-size workloads in the
+launch configuration the benchmark times are compared on sampled queries.
+"""
+import functools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_27888_gb300 import workloads as W
+from tests.util import queries, tiny_assets
+
+pytestmark = pytest.mark.gpu
+
+FP32_TOL = 1e-5
+TC_MAX, TC_MEAN = 2e-2, 2e-3
+SMALL = [(1, None), (2, None), (3, "identity"), (3, "clustered4"), (3, "shared"), (4, "128"), (4, "16"),
+         (4, "8"), (4, "1"), (5, None)]
+
+
+def ntc():
+    from paper_2608_27888_gb300 import ntc as m
+    return m
+
+
+@functools.lru_cache(maxsize=None)
+def small(k, variant=None):
+    return W.config(k, "small", variant)
+
+
+@functools.lru_cache(maxsize=None)
+def oracle_out(k, variant=None):
+    w = small(k, variant)
+    return oracle.decode(w.assets, w.queries)
+
+
+@functools.lru_cache(maxsize=4)
+def decoder(k, variant, precision):
+    return ntc().Decoder(small(k, variant).assets, precision)
+
+
+def dq(q):
+    return ntc().queries_to_device(q)
+
+
+def check_tc(got, ref, what):
+    err = np.abs(got.astype(np.float64) - ref)
+    assert np.isfinite(got).all(), what
+    assert err.max() <= TC_MAX, f"{what}: max abs {err.max():.3e}"
+    assert err.mean() <= TC_MEAN, f"{what}: mean abs {err.mean():.3e}"
+
+
+# --------------------------------------------------------------- bucketing
+
+@pytest.mark.parametrize("k,variant", SMALL)
+def test_bucketing_bit_exact(k, variant):
+    w = small(k, variant)
+    dec = decoder(k, variant, "fp16")
+    perm, counts, tiles = dec.bucket(dq(w.queries))
+    p, c, o, t = oracle.bucket(w.queries["set_id"], w.assets.set_to_decoder, w.assets.num_decoders)
+    assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
+    assert np.array_equal(counts.cpu().numpy().astype(np.uint32), c)
+    assert np.array_equal(tiles.cpu().numpy().astype(np.uint32), t)
+
+
+@pytest.mark.parametrize("n", [1, 31, 32, 33, 127, 128, 129, 4095, 4096, 4097, 70001])
+@pytest.mark.parametrize("pattern", ["random", "same", "descending", "bad", "sparse"])
+def test_bucketing_edge_cases(n, pattern):
+    S, D = 40, 13
+    rng = np.random.default_rng(n)
+    m = rng.integers(0, D, S).astype(np.uint32)
+    m[:3] = [0, 5, 12]
+    if pattern == "random":
+        sets = rng.integers(0, S, n)
+    elif pattern == "same":
+        sets = np.full(n, 7)
+    elif pattern == "descending":
+        sets = (S - 1 - (np.arange(n) * S) // max(n, 1)).clip(0, S - 1)
+    elif pattern == "bad":
+        sets = rng.integers(0, S + 5, n)  # ids >= S land in the extra bucket
+    else:
+        sets = rng.choice([1, 2], n)  # most decoders empty
+    a = tiny_assets([[(8, 8), (4, 4)]] * S, num_sets=S, num_decoders=D, set_to_decoder=m, hidden=64, out_dim=8)
+    q = np.zeros(n, dtype=W.QUERY_DTYPE)
+    q["set_id"] = sets
+    q["u"] = rng.random(n)
+    q["v"] = rng.random(n)
+    dec = ntc().Decoder(a, "fp16")
+    perm, counts, tiles = dec.bucket(dq(q))
+    p, c, o, t = oracle.bucket(q["set_id"], m, D)
+    assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
+    assert np.array_equal(counts.cpu().numpy().astype(np.uint32), c)
+    assert np.array_equal(tiles.cpu().numpy().astype(np.uint32), t)
+    dec.close()
+
+
+# ----------------------------------------------------------------- taps
+
+def _taps_equal(dec, a, q):
+    idx, wt, t = dec.taps(dq(q))
+    ri, rw, rt = oracle.taps(a, q)
+    assert np.array_equal(idx.cpu().numpy().view(np.uint64), ri)
+    assert np.array_equal(wt.cpu().numpy().view(np.uint32), rw.view(np.uint32))
+    assert np.array_equal(t.cpu().numpy().view(np.uint32), rt.view(np.uint32))
+
+
+@pytest.mark.parametrize("k,variant", [(1, None), (2, None), (3, "identity"), (4, "128"), (5, None)])
+def test_taps_bit_exact(k, variant):
+    w = small(k, variant)
+    _taps_equal(decoder(k, variant, "fp16"), w.assets, w.queries)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("dims", [(1, 1), (2, 2), (3, 5), (7, 3), (16, 8)])
+def test_taps_tiny_grids_bit_exact(mode, dims):
+    W0, H0 = dims
+    a = tiny_assets([[(W0, H0), (max(1, W0 // 2), max(1, H0 // 2))]], num_mips=3, address_mode=mode,
+                    hidden=64, out_dim=8)
+    grid = np.arange(-40, 41) / 16.0
+    rng = np.random.default_rng(W0 * 7 + H0)
+    rows = [(0, float(u), float(v), float(l)) for u in grid[::3] for v in grid[::4]
+            for l in (0.0, 0.5, 1.25, 2.0, 5.0)]
+    rows += [(0, float(u), float(v), float(l)) for u, v, l in
+             zip(rng.uniform(-1e3, 1e3, 500), rng.uniform(-3, 3, 500), rng.uniform(-1, 4, 500))]
+    dec = ntc().Decoder(a, "fp32")
+    _taps_equal(dec, a, queries(rows))
+    dec.close()
+
+
+@pytest.mark.parametrize("k,variant", [(2, None), (5, None)])
+def test_features_match_oracle(k, variant):
+    w = small(k, variant)
+    f = decoder(k, variant, "fp16").features(dq(w.queries)).cpu().numpy()
+    ref = oracle.features(w.assets, w.queries)
+    assert np.abs(f - ref).max() <= 1e-5 * max(1.0, np.abs(ref).max())
+
+
+# --------------------------------------------------------------- decode
+
+@pytest.mark.parametrize("k,variant", SMALL)
+def test_decode_fp32_mode(k, variant):
+    w = small(k, variant)
+    ref, _ = oracle_out(k, variant)
+    got = decoder(k, variant, "fp32").decode(dq(w.queries)).cpu().numpy()
+    assert np.abs(got - ref).max() <= FP32_TOL
+
+
+@pytest.mark.parametrize("precision", ["fp16", "bf16"])
+@pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent"])
+@pytest.mark.parametrize("k,variant", SMALL)
+def test_decode_tensor_core_modes(k, variant, mode, precision):
+    w = small(k, variant)
+    ref, _ = oracle_out(k, variant)
+    got = decoder(k, variant, precision).decode(dq(w.queries), mode=mode).cpu().numpy()
+    check_tc(got, ref, f"config {k}/{variant} {mode} {precision}")
+
+
+def test_hidden_128_and_9_channels_on_all_paths():
+    w = small(5)
+    ref, _ = oracle_out(5)
+    for prec, modes in (("fp32", ["bucketed"]), ("fp16", ["bucketed", "bucketed_mma", "divergent"])):
+        dec = decoder(5, None, prec)
+        for m in modes:
+            got = dec.decode(dq(w.queries), mode=m).cpu().numpy()
+            if prec == "fp32":
+                assert np.abs(got - ref).max() <= FP32_TOL
+            else:
+                check_tc(got, ref, m)
+
+
+@pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent"])
+def test_order_invariance_is_bitwise(mode):
+    w = small(3, "clustered4")
+    dec = decoder(3, "clustered4", "fp16")
+    out = dec.decode(dq(w.queries), mode=mode).cpu().numpy()
+    p = np.random.default_rng(1).permutation(len(w.queries))
+    out2 = dec.decode(dq(w.queries[p]), mode=mode).cpu().numpy()
+    if mode == "divergent":
+        # each warp's rows see the same decoder loop whatever their neighbours,
+        # but fp16 rounding of a row is independent of the other rows too
+        assert np.array_equal(out2, out[p])
+    else:
+        assert np.array_equal(out2, out[p])
+
+
+def test_bad_queries_nan_and_counted():
+    w = small(2)
+    q = w.queries[:5000].copy()
+    q["set_id"][::97] = 999
+    q["u"][5::101] = np.nan
+    q["v"][7::103] = np.inf
+    nbad = len(set(range(0, 5000, 97)) | set(range(5, 5000, 101)) | set(range(7, 5000, 103)))
+    ref, bad = oracle.decode(w.assets, q)
+    assert bad == nbad
+    for prec, mode in (("fp32", "bucketed"), ("fp16", "bucketed"), ("fp16", "bucketed_mma"),
+                       ("fp16", "divergent")):
+        dec = ntc().Decoder(w.assets, prec)
+        got = dec.decode(dq(q), mode=mode).cpu().numpy()
+        assert np.array_equal(np.isnan(got), np.isnan(ref)), (prec, mode)
+        assert dec.error_count() == nbad, (prec, mode)
+        dec.reset_error_count()
+        assert dec.error_count() == 0
+        dec.close()
+
+
+def test_decode_host_equals_device_decode():
+    w = small(3, "identity")
+    dec = decoder(3, "identity", "fp16")
+    dev = dec.decode(dq(w.queries)).cpu().numpy()
+    hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
+    host = dec.decode_host(hq).numpy()
+    assert np.array_equal(host, dev)
+
+
+def test_empty_and_invalid_calls():
+    m = ntc()
+    dec = decoder(1, None, "fp16")
+    empty = torch.empty((0, 4), dtype=torch.int32, device="cuda")
+    out = dec.decode(empty)
+    assert out.shape == (0, 8)
+    with pytest.raises(m.NtcError):
+        m.ntc_decode(dec.ctx, 0, 10, 0, 0, m.NTC_MODE_BUCKETED)
+    with pytest.raises(m.NtcError):
+        fp32 = decoder(1, None, "fp32")
+        fp32.decode(dq(small(1).queries[:64]), mode="divergent")
+
+
+# ------------------------------------------------- full sizes, sampled check
+
+FULL = [(1, None), (2, None), (3, "identity"), (4, "128"), (5, None)]
+
+
+@pytest.mark.parametrize("k,variant", FULL)
+def test_full_size_sampled(k, variant):
+    w = W.config(k, "full", variant)
+    n = len(w.queries)
+    rng = np.random.default_rng(k)
+    sample = np.unique(np.concatenate([rng.integers(0, n, 20000), np.arange(min(n, 4096)),
+                                       np.arange(max(0, n - 300), n)]))
+    ref, _ = oracle.decode(w.assets, w.queries[sample])
+    qd = dq(w.queries)
+    dec = ntc().Decoder(w.assets, "fp16")
+    out = dec.decode(qd, mode="bucketed")
+    got = out[torch.from_numpy(sample).cuda()].cpu().numpy()
+    check_tc(got, ref, f"config {k} full bucketed")
+    div = dec.decode(qd, mode="divergent")[torch.from_numpy(sample).cuda()].cpu().numpy()
+    check_tc(div, ref, f"config {k} full divergent")
+    perm, counts, tiles = dec.bucket(qd)
+    p, c, _, t = oracle.bucket(w.queries["set_id"], w.assets.set_to_decoder, w.assets.num_decoders)
+    assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
+    assert np.array_equal(counts.cpu().numpy().astype(np.uint32), c)
+    assert np.array_equal(tiles.cpu().numpy().astype(np.uint32), t)
+    idx, wt, tt = dec.taps(dq(w.queries[sample]))
+    ri, rw, rt = oracle.taps(w.assets, w.queries[sample])
+    assert np.array_equal(idx.cpu().numpy().view(np.uint64), ri)
+    assert np.array_equal(wt.cpu().numpy().view(np.uint32), rw.view(np.uint32))
+    dec.close()
+    del out, qd
+    torch.cuda.empty_cache()
