@@ -192,6 +192,38 @@ NTC_API ntc_status ntc_stage_times(ntc_ctx *ctx, float times[2]);
 /* Kernels this context has launched since creation (host-side counter). */
 NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
 
+/* ------------------------------------------------------ allocation-free entry
+ *
+ * The paper has no counterpart to this call; it exists for callers that may
+ * not allocate device memory when they sort their queries -- for example a
+ * renderer whose engine owns all GPU memory and forbids cudaMalloc and
+ * cudaMallocAsync inside its frame loop, where an allocation can stall the
+ * frame or fail half-way through it.
+ *
+ * ntc_bucket_static is the bucketing stage of ntc_debug_bucket without a
+ * context and without any allocation: d_perm[n] receives the query indices in
+ * (decoder, original index) order (out-of-range set ids count as decoder
+ * num_decoders) and d_sorted[n] the query records in that order.  h_set_to_decoder
+ * is a HOST array of num_sets entries (each < num_decoders); d_queries,
+ * d_perm and d_sorted are caller-owned device buffers (the query buffers
+ * 16-byte aligned).  Its scratch is one file-scope device array of 1,360,896
+ * bytes that every GPU loading the library holds until the process exits, so:
+ *   - num_sets <= 65536, num_decoders <= 4095 and
+ *     (num_decoders + 1) * ceil(n / 4096) <= 262144 (larger calls return
+ *     NTC_ERR_UNSUPPORTED and enqueue nothing);
+ *   - every call on a device shares that array and it keeps the previous
+ *     call's contents; the call clears what must start at zero itself, but two
+ *     calls whose work overlaps on the GPU (different streams, threads or
+ *     processes sharing the context) race and corrupt each other's result;
+ *   - the first call on each device looks the array's device address up
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ * Asynchronous on cuda_stream; n = 0 is a no-op.  It calls no cudaMalloc,
+ * cudaFree or allocating library routine. */
+NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder, uint32_t num_sets,
+                                     uint32_t num_decoders, const ntc_query *d_queries, size_t n,
+                                     uint32_t *d_perm, ntc_query *d_sorted, void *cuda_stream);
+
 /* Human-readable message of the last failed call on this host thread. */
 NTC_API const char *ntc_last_error(void);
 NTC_API const char *ntc_status_string(ntc_status s);

@@ -50,6 +50,10 @@ static ntc_status fail(ntc_status s, const char *fmt, ...) {
   return s;
 }
 
+namespace ntc {
+void set_last_error(const char *msg) { snprintf(g_err, sizeof g_err, "%s", msg); }
+}  // namespace ntc
+
 static ntc_status cuda_fail(cudaError_t e, const char *what) {
   if (e == cudaErrorMemoryAllocation)
     return fail(NTC_ERR_OUT_OF_MEMORY, "%s: %s", what, cudaGetErrorString(e));

@@ -27,7 +27,7 @@ MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucket
 EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps",
            "ntc_debug_features", "ntc_debug_bucket", "ntc_max_tiles", "ntc_get_error_count",
            "ntc_reset_error_count", "ntc_launch_count", "ntc_set_stage_timing", "ntc_stage_times",
-           "ntc_last_error", "ntc_status_string")
+           "ntc_bucket_static", "ntc_last_error", "ntc_status_string")
 
 
 class ntc_desc(ctypes.Structure):
@@ -77,6 +77,7 @@ def _load():
         "ntc_launch_count": ([P], ctypes.c_uint64),
         "ntc_set_stage_timing": ([P, I], I),
         "ntc_stage_times": ([P, P], I),
+        "ntc_bucket_static": ([P, ctypes.c_uint32, ctypes.c_uint32, P, S, P, P, P], I),
         "ntc_last_error": ([], ctypes.c_char_p),
         "ntc_status_string": ([I], ctypes.c_char_p),
     }
@@ -153,6 +154,12 @@ def ntc_stage_times(ctx):
     t = (ctypes.c_float * 2)()
     _check(_lib.ntc_stage_times(ctx, t))
     return float(t[0]), float(t[1])
+
+
+def ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm, d_sorted, stream):
+    """Allocation-free bucketing (no context): see include/ntc.h."""
+    _check(_lib.ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm,
+                                  d_sorted, stream))
 
 
 def ntc_last_error() -> str:

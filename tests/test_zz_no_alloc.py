@@ -1,0 +1,50 @@
+"""The allocation-free bucketing entry point (ntc_bucket_static).
+
+It serves callers that may not allocate device memory when they sort queries
+(an engine that owns all GPU memory and forbids cudaMalloc inside its frame
+loop).  Its result must equal the context-based bucketing (ntc_debug_bucket) bit
+for bit, on consecutive calls that share its static scratch.  This file sorts
+last so a run that stops at the first failure has run every other test first.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_27888_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _static_bucket(ntc, a, qd):
+    n = qd.shape[0]
+    perm = torch.full((n,), -1, dtype=torch.int32, device="cuda")
+    srt = torch.zeros((n, 4), dtype=torch.int32, device="cuda")
+    m = np.ascontiguousarray(a.set_to_decoder, dtype=np.uint32)
+    ntc.ntc_bucket_static(m.ctypes.data, a.num_sets, a.num_decoders, qd.data_ptr(), n, perm.data_ptr(),
+                          srt.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    return perm, srt
+
+
+def test_static_bucketing_matches_context_bucketing_on_consecutive_calls():
+    from paper_2608_27888_gb300 import ntc
+    cases = [W.config(3, "small", "clustered4"), W.config(2, "small"), W.config(3, "small", "clustered4")]
+    for w in cases:  # three calls in a row, different sizes and decoder counts
+        qd = ntc.queries_to_device(w.queries)
+        perm, srt = _static_bucket(ntc, w.assets, qd)
+        dec = ntc.Decoder(w.assets, "fp16")
+        ref_perm, _, _ = dec.bucket(qd)
+        dec.close()
+        torch.cuda.synchronize()
+        assert torch.equal(perm, ref_perm)
+        assert torch.equal(srt, qd[ref_perm.long()])
+
+
+def test_static_bucketing_rejects_sizes_beyond_its_scratch():
+    from paper_2608_27888_gb300 import ntc
+    w = W.config(1, "small")
+    qd = ntc.queries_to_device(w.queries)
+    m = np.zeros(1, dtype=np.uint32)
+    n_too_many = 262144 // 4096 * 4096 * 2  # (4095 + 1) * ceil(n / 4096) > 262144
+    with pytest.raises(ntc.NtcError, match="static scratch"):
+        ntc.ntc_bucket_static(m.ctypes.data, 1, 4095, qd.data_ptr(), n_too_many, qd.data_ptr(),
+                              qd.data_ptr(), 0)
