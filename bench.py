@@ -40,6 +40,10 @@ WORKLOAD = ("config2: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16)
 BYTES_PER_QUERY = 16 + 8 * 16 + 8 * 4  # query record + 8 taps of 16 B + 8 fp32 outputs
 FLOPS_PER_QUERY = 2 * (16 * 64 + 64 * 64 + 64 * 8)
 L2_FLUSH_BYTES = 256 << 20
+KERNEL_NAMES = {("bucketed", False): "k_decode_tc (tcgen05/TMEM gather-decode)",
+                ("bucketed", True): "k_decode_fp32 (FFMA gather-decode)",
+                ("bucketed_mma", False): "k_decode_mma (mma.sync gather-decode)",
+                ("divergent", False): "k_decode_divergent (mma.sync, unsorted)"}
 
 
 def parse():
@@ -126,7 +130,7 @@ def peaks():
 
 def kernel_source_hash():
     h = hashlib.sha1()
-    for f in ("decode_tc.cu", "decode_mma.cu", "ntc_internal.cuh"):
+    for f in ("decode_tc.cu", "ntc_internal.cuh"):
         with open(os.path.join(ROOT, "paper_2608_27888_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
@@ -279,8 +283,7 @@ def main():
     kernel_tag = f"{args.mode}-{args.precision}"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": recorded_traffic(kernel_tag),
-                "kernel": "gather-decode (" + ("tcgen05" if args.mode == "bucketed" and args.precision != "fp32"
-                                               else args.mode) + ")",
+                "kernel": KERNEL_NAMES[(args.mode, args.precision == "fp32")],
                 "kernel_ms": decode_ms, "bucketing_ms": bucket_ms,
                 "peak_kind": f"{peak_kind} HBM copy bandwidth",
                 "algorithmic_bytes_per_launch": alg_bytes}

@@ -262,9 +262,9 @@ cudaError_t launch_pack_weights(const float *w32, uint32_t D, uint32_t H, uint32
     k_pack<__nv_bfloat16><<<D, 256, 0, st>>>(w32, H, C, mma, mma_stride, f32, f32_stride);
   else
     k_pack<__half><<<D, 256, 0, st>>>(w32, H, C, mma, mma_stride, f32, f32_stride);
-  (void)tc;
-  (void)tc_stride;
-  return cudaGetLastError();
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_pack_tc(w32, D, H, C, bf16, tc, tc_stride, st);
 }
 
 }  // namespace ntc

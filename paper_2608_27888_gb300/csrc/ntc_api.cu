@@ -25,6 +25,7 @@ struct ntc_ctx {
   uint8_t *d_tc = nullptr;
   size_t mma_stride = 0, f32_stride = 0, tc_stride = 0;
   unsigned long long *d_err = nullptr;
+  unsigned int *d_status = nullptr;  // nonzero: a decode kernel gave up a bounded wait
   // bucketing scratch (grows on demand, stream-ordered)
   size_t cap_n = 0, cap_counts = 0;
   uint32_t *d_counts = nullptr, *d_perm = nullptr, *d_meta = nullptr;
@@ -117,6 +118,7 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_f32);
   cudaFree(c->d_tc);
   cudaFree(c->d_err);
+  cudaFree(c->d_status);
   cudaFree(c->d_counts);
   cudaFree(c->d_perm);
   cudaFree(c->d_sorted);
@@ -265,6 +267,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   step(cudaMalloc((void **)&c->d_f32, c->f32_stride * 4 * c->D));
   step(cudaMalloc((void **)&c->d_tc, c->tc_stride * c->D));
   step(cudaMalloc((void **)&c->d_err, sizeof(unsigned long long)));
+  step(cudaMalloc((void **)&c->d_status, sizeof(unsigned int)));
   step(cudaMalloc((void **)&d_w32, P * 4 * c->D));
   if (e == cudaSuccess) {
     step(cudaMemcpy(c->d_lat, d->latents, d->num_texels * 16, cudaMemcpyHostToDevice));
@@ -272,6 +275,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
     step(cudaMemcpy(c->d_map, d->set_to_decoder, (size_t)S * 4, cudaMemcpyHostToDevice));
     step(cudaMemcpy(d_w32, d->weights, P * 4 * c->D, cudaMemcpyHostToDevice));
     step(cudaMemset(c->d_err, 0, sizeof(unsigned long long)));
+    step(cudaMemset(c->d_status, 0, sizeof(unsigned int)));
     step(cudaMemset(c->d_tc, 0, c->tc_stride * c->D));
     step(launch_pack_weights(d_w32, c->D, c->H, c->C, c->prec == NTC_PREC_TC_BF16, c->d_mma,
                              c->mma_stride, c->d_f32, c->f32_stride, c->d_tc, c->tc_stride, 0));
@@ -342,8 +346,10 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
   if (fp32)
     e = launch_decode_fp32(A, W, B, n, out, c->d_err, c->num_sms, st, &launches);
-  else
+  else if (mode == NTC_MODE_BUCKETED_MMA)
     e = launch_decode_mma(A, W, B, n, out, c->d_err, bf16, c->num_sms, st, &launches);
+  else
+    e = launch_decode_tc(A, W, B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
   c->launches += launches;
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if (c->timing) {
@@ -442,8 +448,11 @@ ntc_status ntc_get_error_count(ntc_ctx *c, uint64_t *count) {
   DeviceGuard g(c->device);
   CK(cudaDeviceSynchronize(), "synchronize");
   unsigned long long v = 0;
+  unsigned int st = 0;
   CK(cudaMemcpy(&v, c->d_err, sizeof v, cudaMemcpyDeviceToHost), "error counter read");
+  CK(cudaMemcpy(&st, c->d_status, sizeof st, cudaMemcpyDeviceToHost), "status read");
   *count = v;
+  if (st) return fail(NTC_ERR_CUDA, "a decode kernel gave up waiting for the tensor core; results are invalid");
   return NTC_OK;
 }
 
@@ -452,6 +461,7 @@ ntc_status ntc_reset_error_count(ntc_ctx *c) {
   DeviceGuard g(c->device);
   CK(cudaDeviceSynchronize(), "synchronize");
   CK(cudaMemset(c->d_err, 0, sizeof(unsigned long long)), "error counter reset");
+  CK(cudaMemset(c->d_status, 0, sizeof(unsigned int)), "status reset");
   return NTC_OK;
 }
 

@@ -233,8 +233,10 @@ cudaError_t launch_decode_divergent(const Assets &A, const WeightImages &W, cons
                                     size_t n, float *out, unsigned long long *err, bool bf16,
                                     int num_sms, cudaStream_t st, int *launches);
 cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
-                             float *out, unsigned long long *err, bool bf16, int num_sms,
-                             cudaStream_t st, int *launches);
+                             float *out, unsigned long long *err, unsigned int *status, bool bf16,
+                             int num_sms, cudaStream_t st, int *launches);
+cudaError_t launch_pack_tc(const float *w32, uint32_t D, uint32_t H, uint32_t C, bool bf16,
+                           uint8_t *tc, size_t tc_stride, cudaStream_t st);
 cudaError_t launch_debug_taps(const Assets &A, const ntc_query *q, size_t n, unsigned long long *idx,
                               float *w, float *t, cudaStream_t st, int *launches);
 cudaError_t launch_debug_features(const Assets &A, const ntc_query *q, size_t n, float *f,
