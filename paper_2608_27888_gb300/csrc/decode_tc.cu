@@ -135,6 +135,36 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "r"(taddr));
 }
 
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};\n" ::"r"(taddr), "r"(r[0]),
+               "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
+}
+
+// D[tmem] (+)= A[tmem] x B[smem]: A read from tensor memory (row = lane, two
+// 16-bit K elements per 32-bit column).
+__device__ __forceinline__ void umma_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc,
+                                        uint32_t accum) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(accum)
+      : "memory");
+}
+
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 }
@@ -161,25 +191,28 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
 }
 
 // TMEM accumulator row (H fp32 columns) -> ReLU -> fp16/bf16 hidden tile row.
-template <int H, bool BF16>
+// CH columns are read per tcgen05.wait::ld (64: two loads in flight; 32: one).
+template <int H, bool BF16, int CH = (H <= 64 ? 64 : 32)>
 __device__ __forceinline__ void epilogue_hidden(uint32_t tmem_row, uint32_t sH, uint32_t row) {
   constexpr uint32_t KH = H + 16;
-#pragma unroll
-  for (int c0 = 0; c0 < H; c0 += 64) {
+#pragma unroll 1
+  for (int c0 = 0; c0 < H; c0 += CH) {
     uint32_t a[32], b[32];
     tmem_ld32(tmem_row + c0, a);
-    tmem_ld32(tmem_row + c0 + 32, b);
+    if (CH == 64) tmem_ld32(tmem_row + c0 + 32, b);
     tmem_wait_ld();
 #pragma unroll
     for (int i = 0; i < 4; ++i)
       sts128(sH + core_off(row, c0 + 8 * i, KH), pack_relu<BF16>(a[8 * i], a[8 * i + 1]),
              pack_relu<BF16>(a[8 * i + 2], a[8 * i + 3]), pack_relu<BF16>(a[8 * i + 4], a[8 * i + 5]),
              pack_relu<BF16>(a[8 * i + 6], a[8 * i + 7]));
+    if (CH == 64) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      sts128(sH + core_off(row, c0 + 32 + 8 * i, KH), pack_relu<BF16>(b[8 * i], b[8 * i + 1]),
-             pack_relu<BF16>(b[8 * i + 2], b[8 * i + 3]), pack_relu<BF16>(b[8 * i + 4], b[8 * i + 5]),
-             pack_relu<BF16>(b[8 * i + 6], b[8 * i + 7]));
+      for (int i = 0; i < 4; ++i)
+        sts128(sH + core_off(row, c0 + 32 + 8 * i, KH), pack_relu<BF16>(b[8 * i], b[8 * i + 1]),
+               pack_relu<BF16>(b[8 * i + 2], b[8 * i + 3]), pack_relu<BF16>(b[8 * i + 4], b[8 * i + 5]),
+               pack_relu<BF16>(b[8 * i + 6], b[8 * i + 7]));
+    }
   }
 }
 
@@ -195,179 +228,474 @@ struct TcLayout {
   static constexpr uint32_t WG = WIMG + A + HT;  // shared bytes per warpgroup
 };
 
-template <int H, int NWG, bool BF16>
-__global__ void __launch_bounds__(NWG * 128, 1)
-    k_decode_tc(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
-                unsigned int *status) {
-  using L = TcLayout<H>;
-  extern __shared__ __align__(128) uint8_t smem[];
-  const int wg = threadIdx.x >> 7, tid = threadIdx.x & 127, warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  uint8_t *my = smem + (size_t)wg * L::WG;
-  const uint32_t sW1 = saddr(my), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2, sA = sW3 + L::W3,
-                 sH = sA + L::A;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)NWG * L::WG);
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + NWG);
-  volatile uint32_t *abort_flag = tmem_slot + 1;  // [NWG]
-  constexpr uint32_t kCols = NWG * H;             // 256
-  const uint32_t bar = saddr(bars + wg);
+// Latent taps of one query, loaded ahead of use: 8 taps (2 levels x 4), or 16
+// when a mip blend is possible (mip lo, then mip lo+1); the blend factor is
+// folded into the weights.
+template <bool TRI>
+struct Taps {
+  static constexpr int N = TRI ? 16 : 8;
+  uint4 raw[N];
+  float w[N];
+};
 
+template <bool TRI>
+__device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                           bool good, Taps<TRI> &tp) {
+#pragma unroll
+  for (int i = 0; i < Taps<TRI>::N; ++i) {
+    tp.w[i] = 0.0f;
+    tp.raw[i] = make_uint4(0, 0, 0, 0);
+  }
+  if (!good) return;
+  float t;
+  const int lo = select_mip(q.lod, A.num_mips, t);
+  const GridDesc *g = grids + (size_t)q.set_id * kLevels * A.num_mips;
+  const float s = TRI ? __fsub_rn(1.0f, t) : 1.0f;
+#pragma unroll
+  for (int k = 0; k < kLevels; ++k) {
+    unsigned long long idx[4];
+    float w[4];
+    grid_taps(g[k * A.num_mips + lo], q.u, q.v, A.address_mode, idx, w);
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      tp.w[k * 4 + p] = TRI ? w[p] * s : w[p];
+      tp.raw[k * 4 + p] = __ldg(A.lat + idx[p]);
+    }
+  }
+  if (TRI && t > 0.0f) {
+#pragma unroll
+    for (int k = 0; k < kLevels; ++k) {
+      unsigned long long idx[4];
+      float w[4];
+      grid_taps(g[k * A.num_mips + lo + 1], q.u, q.v, A.address_mode, idx, w);
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        tp.w[8 + k * 4 + p] = w[p] * t;
+        tp.raw[8 + k * 4 + p] = __ldg(A.lat + idx[p]);
+      }
+    }
+  }
+}
+
+// acc[c/2] += w * tap[c] over the 8 channels of one tap, as packed fp32 pairs.
+__device__ __forceinline__ void accum_tap_x2(unsigned long long (&acc)[4], uint4 raw, float w) {
+  unsigned long long ww;
+  asm("mov.b64 %0, {%1, %1};" : "=l"(ww) : "f"(w));
+  const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const float2 x = __half22float2(h[p]);
+    unsigned long long xx;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(xx) : "f"(x.x), "f"(x.y));
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc[p]) : "l"(ww), "l"(xx));
+  }
+}
+
+template <bool TRI, bool BF16>
+__device__ __forceinline__ void taps_to_row(const Taps<TRI> &tp, uint32_t (&packed)[8]) {
+  unsigned long long acc[kLevels][4];
+#pragma unroll
+  for (int k = 0; k < kLevels; ++k)
+#pragma unroll
+    for (int p = 0; p < 4; ++p) acc[k][p] = 0ull;
+#pragma unroll
+  for (int k = 0; k < kLevels; ++k)
+#pragma unroll
+    for (int p = 0; p < 4; ++p) accum_tap_x2(acc[k], tp.raw[k * 4 + p], tp.w[k * 4 + p]);
+  if (TRI && __any_sync(0xFFFFFFFFu, tp.w[8] != 0.0f || tp.w[9] != 0.0f || tp.w[10] != 0.0f ||
+                                         tp.w[11] != 0.0f)) {
+#pragma unroll
+    for (int k = 0; k < kLevels; ++k)
+#pragma unroll
+      for (int p = 0; p < 4; ++p) accum_tap_x2(acc[k], tp.raw[8 + k * 4 + p], tp.w[8 + k * 4 + p]);
+  }
+#pragma unroll
+  for (int k = 0; k < kLevels; ++k)
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      float lo, hi;
+      asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(acc[k][p]));
+      packed[k * 4 + p] = pack<BF16>(lo, hi);
+    }
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+// Tile t of the bucketed order from (possibly shared-memory) copies of the
+// segment starts and tile starts: decoder, first sorted position and length.
+__device__ __forceinline__ void tile_lookup(const uint32_t *seg, const uint32_t *tst, uint32_t D,
+                                            uint32_t t, uint32_t &dec, uint32_t &start, uint32_t &len) {
+  uint32_t lo = 0, hi = D + 1;
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (tst[mid] <= t) lo = mid; else hi = mid;
+  }
+  dec = lo;
+  start = seg[lo] + (t - tst[lo]) * kTile;
+  len = min((uint32_t)kTile, seg[lo + 1] - start);
+}
+
+// Per-thread view of one tile row.
+struct Row {
+  uint32_t dec, start, len;  // the tile
+  uint32_t oi;               // original query index of this row
+  bool valid, good;
+};
+
+__device__ __forceinline__ Row load_row(const Buckets &B, const uint32_t *seg, const uint32_t *tst,
+                                        uint32_t D, uint32_t t, uint32_t T, int tid, ntc_query &q) {
+  Row r;
+  r.valid = r.good = false;
+  r.oi = 0;
+  r.dec = 0xFFFFFFFFu;
+  r.start = r.len = 0;
+  if (t >= T) return r;
+  tile_lookup(seg, tst, D, t, r.dec, r.start, r.len);
+  r.valid = (uint32_t)tid < r.len;
+  if (r.valid) {
+    q = load_query(B.sorted + r.start + tid);
+    r.oi = __ldg(B.perm + r.start + tid);
+  }
+  return r;
+}
+
+constexpr uint32_t kSmemTileTable = 1024;  // staged when D + 2 <= this
+constexpr uint32_t kSmemGrids = 1024;      // staged when S * 2 * M <= this
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+
+// Shared-memory plan of the warp-specialised kernel: only the decoders' weights
+// (the B operands) and bookkeeping live in shared memory; every A operand and
+// accumulator lives in tensor memory, so most of the SM's L1/shared array stays
+// L1, which holds the in-flight latent gathers.
+template <int H, int NC, int S>
+struct TmSmem {
+  using L = TcLayout<H>;
+  static constexpr size_t weights = 0;                                  // per consumer
+  static constexpr size_t flags = weights + (size_t)NC * L::WIMG;       // per stage: 128 row flags
+  static constexpr size_t bars = flags + (size_t)S * 128;
+  static constexpr int nbars = 2 * S + 2 * NC;                          // full, empty, mma, weights
+  static constexpr size_t misc = bars + (size_t)nbars * 8;
+  static constexpr size_t tiles = misc + 64;
+  static constexpr size_t total = tiles + 2 * kSmemTileTable * 4;
+};
+
+// Tensor-memory plan (columns): consumer c owns [c*SC, c*SC + H) for the fp32
+// accumulator and [c*SC + H, c*SC + H + KH/2) for its hidden A operand (two
+// 16-bit K elements per column); ring stage s owns 16 columns at RING + 16 s for
+// the layer-1 A operand [128 x 32].
+template <int H, int NC, int S>
+struct TmCols {
+  static constexpr uint32_t KH = H + 16;
+  static constexpr uint32_t SC = ((H + KH / 2) + 31) / 32 * 32;  // consumer stride, 32-aligned
+  static constexpr uint32_t RING = NC * SC;
+  static constexpr uint32_t used = RING + 16 * S;
+  static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
+  static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
+};
+
+// Warp-specialised gather-decode with tensor-memory operands.
+//   Producer warpgroups 0..NP-1 gather: each thread computes the taps of one
+//   query row, blends them in fp32 and stores the fp16/bf16 feature row (plus the
+//   bias column) into the TMEM A region of one ring stage (tcgen05.st; warp q of
+//   a warpgroup owns TMEM lanes 32q..32q+31, exactly its rows).  Producer p takes
+//   the CTA's local tiles k = p, p + NP, ...; the query record of its next tile is
+//   loaded while the current one is gathered.
+//   Consumer warpgroups NP..NP+NC-1 each take local tiles k = c, c + NC, ...:
+//   layer 1 reads A from the stage's TMEM region and B (weights) from shared
+//   memory, the ReLU/convert epilogue goes TMEM -> registers -> TMEM, layers 2
+//   and 3 read their A from TMEM too, and the sigmoid epilogue scatters rows to
+//   out[perm[i]].  Stage hand-off uses full/empty mbarriers: four producer-warp
+//   arrivals fill a stage, the completion of the layer-1 MMA empties it.
+// CTA b owns the global tiles b, b + grid, b + 2 grid, ...
+template <int H, bool BF16, bool TRI, int CP, int NP, int NC, int S>
+__global__ void __launch_bounds__((NP + NC) * 128, 1)
+    k_decode_tm(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
+                unsigned int *status, int vec_out) {
+  using L = TcLayout<H>;
+  using M = TmSmem<H, NC, S>;
+  using TC = TmCols<H, NC, S>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int role = threadIdx.x >> 7, row = threadIdx.x & 127, warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t lanes = (uint32_t)((warp & 3) * 32) << 16;  // this warp's TMEM lane quadrant
+  const uint32_t sbase = saddr(smem);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + M::bars);
+  auto full_bar = [&](uint32_t s) { return saddr(bars + s); };
+  auto empty_bar = [&](uint32_t s) { return saddr(bars + S + s); };
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + M::misc);
+  volatile uint32_t *abort_flag = tmem_slot + 1;
+  volatile uint32_t *stop_flag = tmem_slot + 2;  // [NC], each read only after its warpgroup's barrier
+  const uint32_t D = A.num_decoders, C = W.out_dim;
+
+  const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
+  if (D + 2 <= kSmemTileTable) {
+    uint32_t *s_seg = reinterpret_cast<uint32_t *>(smem + M::tiles);
+    uint32_t *s_tst = s_seg + kSmemTileTable;
+    for (uint32_t i = threadIdx.x; i < D + 2; i += blockDim.x) {
+      s_seg[i] = __ldg(seg + i);
+      s_tst[i] = __ldg(tst + i);
+    }
+    seg = s_seg;
+    tst = s_tst;
+  }
   if (threadIdx.x == 0) {
-    for (int w = 0; w < NWG; ++w) mbar_init(saddr(bars + w), 1);
+    for (int i = 0; i < S; ++i) {
+      mbar_init(full_bar(i), 4);   // one arrival per producer warp
+      mbar_init(empty_bar(i), 1);  // the consumer's layer-1 commit
+    }
+    for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), 1);
+    *abort_flag = 0;
+    for (int i = 0; i < NC; ++i) stop_flag[i] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
-  if (tid == 0) abort_flag[wg] = 0;
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
                      saddr(tmem_slot)),
-                 "r"(kCols)
+                 "r"(TC::alloc)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
   }
-  // constant columns: A[r][16] = 1 (bias), A[r][17..31] = 0; H[r][H] = 1, H[r][H+1..] = 0
-  const uint32_t one = BF16 ? 0x3F80u : 0x3C00u;
-  sts128(sA + core_off(tid, 16, kTcKA), one, 0, 0, 0);
-  sts128(sA + core_off(tid, 24, kTcKA), 0, 0, 0, 0);
-  sts128(sH + core_off(tid, H, L::KH), one, 0, 0, 0);
-  sts128(sH + core_off(tid, H + 8, L::KH), 0, 0, 0, 0);
-  fence_async_smem();
   fence_before();
   __syncthreads();
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t tmem_wg = tmem_base + (uint32_t)(wg * H);
-  const uint32_t tmem_row = tmem_wg + ((uint32_t)((warp & 3) * 32) << 16);
-
-  const uint32_t D = A.num_decoders, C = W.out_dim;
+  const uint32_t one = BF16 ? 0x3F80u : 0x3C00u;  // 1.0 in the low half, 0 in the high half
   const uint32_t T = __ldg(B.meta);
-  const uint32_t G = gridDim.x * NWG;
-  uint32_t phase = 0, cur = 0xFFFFFFFFu;
-  constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
+  const uint32_t grid = gridDim.x;
+  const uint32_t K = blockIdx.x < T ? (T - blockIdx.x + grid - 1) / grid : 0;  // local tiles
 
-  for (uint32_t t = blockIdx.x * NWG + wg; t < T; t += G) {
-    uint32_t dec, start, len;
-    tile_info(B.meta, D, t, dec, start, len);
-    const bool valid = (uint32_t)tid < len;
+  if (role < NP) {
+    // ------------------------------------------------------------ producer
+    uint32_t k = role;
+    uint32_t dec = D, start = 0, len = 0;
     ntc_query q;
-    uint32_t oi = 0;
-    bool bad = true;
-    if (valid) {
-      q = load_query(B.sorted + start + tid);
-      oi = __ldg(B.perm + start + tid);
-      bad = dec == D || query_bad(A, q);
+    if (k < K) {
+      tile_lookup(seg, tst, D, blockIdx.x + k * grid, dec, start, len);
+      if ((uint32_t)row < len) q = load_query(B.sorted + start + row);
     }
-    const uint32_t badm = __ballot_sync(0xFFFFFFFFu, valid && bad);
-    if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
-    if (valid && bad)
-      for (uint32_t c = 0; c < C; ++c) out[(size_t)oi * C + c] = __int_as_float(0x7fc00000);
-    if (dec == D) continue;  // the whole tile is bad queries (uniform)
-
-    if (dec != cur) {  // this warpgroup's previous MMAs are complete: reload weights
-      const uint4 *src = reinterpret_cast<const uint4 *>(W.tc + (size_t)dec * W.tc_stride);
-      uint4 *dst = reinterpret_cast<uint4 *>(my);
-      for (uint32_t i = tid; i < L::WIMG / 16; i += 128) dst[i] = __ldg(src + i);
-      cur = dec;
-    }
-    float f[kInDim];
+    for (; k < K; k += NP) {
+      if (*abort_flag) break;
+      // the next tile's query record goes in flight first
+      uint32_t ndec = D, nstart = 0, nlen = 0;
+      ntc_query nq;
+      if (k + NP < K) {
+        tile_lookup(seg, tst, D, blockIdx.x + (k + NP) * grid, ndec, nstart, nlen);
+        if ((uint32_t)row < nlen) nq = load_query(B.sorted + nstart + row);
+      }
+      const bool valid = (uint32_t)row < len;
+      const bool good = valid && dec < D && !query_bad(A, q);
+      Taps<TRI> taps;
+      issue_taps<TRI>(A, A.grids, q, good, taps);
+      // bad rows (set id out of range, non-finite UV, or the bad bucket) decode to NaN
+      const bool bad = valid && !good;
+      const uint32_t badm = __ballot_sync(0xFFFFFFFFu, bad);
+      if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
+      if (bad) {
+        const uint32_t oi = __ldg(B.perm + start + row);
+        for (uint32_t cc = 0; cc < C; ++cc) out[(size_t)oi * C + cc] = __int_as_float(0x7fc00000);
+      }
+      uint32_t a[16];
+      {
+        uint32_t pk[8];
+        taps_to_row<TRI, BF16>(taps, pk);
 #pragma unroll
-    for (int c = 0; c < kInDim; ++c) f[c] = 0.0f;
-    if (valid && !bad) query_features(A, q, f);
-    sts128(sA + core_off(tid, 0, kTcKA), pack<BF16>(f[0], f[1]), pack<BF16>(f[2], f[3]),
-           pack<BF16>(f[4], f[5]), pack<BF16>(f[6], f[7]));
-    sts128(sA + core_off(tid, 8, kTcKA), pack<BF16>(f[8], f[9]), pack<BF16>(f[10], f[11]),
-           pack<BF16>(f[12], f[13]), pack<BF16>(f[14], f[15]));
-    fence_async_smem();
-    wg_bar(wg);
-    // layer 1: [128 x 32] x [32 x H]
-    if (tid == 0) {
+        for (int i = 0; i < 8; ++i) a[i] = pk[i];
+      }
+      a[8] = one;
+#pragma unroll
+      for (int i = 9; i < 16; ++i) a[i] = 0u;
+      const uint32_t s = k % S, n = k / S;
+      if (!mbar_wait(empty_bar(s), (n & 1) ^ 1)) {  // the stage's previous tile has left layer 1
+        atomicOr(status, 1u);
+        *abort_flag = 1;
+      }
       fence_after();
+      tmem_st16(tmem_base + TC::RING + 16 * s + lanes, a);
+      tmem_wait_st();
+      smem[M::flags + s * 128 + row] = good ? 1 : 0;
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(full_bar(s));
+      dec = ndec;
+      start = nstart;
+      len = nlen;
+      q = nq;
+    }
+  } else {
+    // ------------------------------------------------------------ consumer
+    const int c = role - NP;
+    const int wgid = role;  // named barrier id role + 1
+    const bool poller = (row >> 5) == 0;
+    const uint32_t tD = tmem_base + c * TC::SC;  // accumulator
+    const uint32_t tH = tD + H;                  // hidden A operand
+    const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
+    const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
+    uint32_t ph = 0, wph = 0, cur = 0xFFFFFFFFu;
+    constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
+    const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
+    auto wait_bar = [&](uint32_t b, uint32_t parity) {
+      if (poller && !mbar_wait(b, parity)) {
+        atomicOr(status, 1u);
+        *abort_flag = 1;
+      }
+    };
+    // the hidden A operand's bias column (k = H) and zero padding never change
+    {
+      uint32_t z[8] = {one, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+      tmem_st8(tH + H / 2 + lanes, z);
+      tmem_wait_st();
+    }
+    // TMEM accumulator -> ReLU -> fp16/bf16 pairs -> hidden A operand
+    auto hidden = [&]() {
+#pragma unroll 1
+      for (int c0 = 0; c0 < H; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(tD + lanes + c0, v);
+        tmem_wait_ld();
+        uint32_t p[16];
 #pragma unroll
-      for (uint32_t k = 0; k < kTcKA / 16; ++k)
-        umma(tmem_wg, smem_desc(sA + k * 256, kTcKA), smem_desc(sW1 + k * 256, kTcKA), id_hidden, k);
-      umma_commit(bar);
-    }
-    if (!mbar_wait(bar, phase)) {
-      atomicOr(status, 1u);
-      abort_flag[wg] = 1;
-    }
-    phase ^= 1;
-    fence_after();
-    epilogue_hidden<H, BF16>(tmem_row, sH, tid);
-    fence_async_smem();
-    fence_before();
-    wg_bar(wg);
-    // layer 2: [128 x (H+16)] x [(H+16) x H]
-    if (tid == 0) {
-      fence_after();
+        for (int i = 0; i < 16; ++i) p[i] = pack_relu<BF16>(v[2 * i], v[2 * i + 1]);
+        tmem_st16(tH + lanes + c0 / 2, p);
+      }
+      tmem_wait_st();
+    };
+    for (uint32_t k = c; k < K; k += NC) {
+      const uint32_t t = blockIdx.x + k * grid, s = k % S, n = k / S;
+      uint32_t dec, start, len;
+      tile_lookup(seg, tst, D, t, dec, start, len);
+      const uint32_t oi = (uint32_t)row < len ? __ldg(B.perm + start + row) : 0u;
+      bool wpend = false;
+      if (dec < D && dec != cur) {  // this consumer's previous tile is complete
+        if (row == 0) bulk_g2s(sW1, W.tc + (size_t)dec * W.tc_stride, L::WIMG, wbar);
+        wpend = true;
+        cur = dec;
+      }
+      wait_bar(full_bar(s), n & 1);
+      if (wpend) {
+        wait_bar(wbar, wph);
+        wph ^= 1;
+      }
+      wg_bar(wgid);
+      const bool good = smem[M::flags + s * 128 + row] != 0;
+      if (row == 0) {
+        fence_after();
+        if (dec < D) {
+          const uint32_t tA = tmem_base + TC::RING + 16 * s;
 #pragma unroll
-      for (uint32_t k = 0; k < L::KH / 16; ++k)
-        umma(tmem_wg, smem_desc(sH + k * 256, L::KH), smem_desc(sW2 + k * 256, L::KH), id_hidden, k);
-      umma_commit(bar);
-    }
-    if (!mbar_wait(bar, phase)) {
-      atomicOr(status, 1u);
-      abort_flag[wg] = 1;
-    }
-    phase ^= 1;
-    fence_after();
-    epilogue_hidden<H, BF16>(tmem_row, sH, tid);
-    fence_async_smem();
-    fence_before();
-    wg_bar(wg);
-    // layer 3: [128 x (H+16)] x [(H+16) x 16]
-    if (tid == 0) {
-      fence_after();
+          for (uint32_t kq = 0; kq < kTcKA / 16; ++kq) umma_ta(tD, tA + 8 * kq, dW1 + 16 * kq, id_hidden, kq);
+          umma_commit(mbar);
+          umma_commit(empty_bar(s));
+        } else {
+          mbar_arrive(empty_bar(s));  // a tile of bad queries: nothing to multiply
+        }
+      }
+      if (dec < D) {
+#pragma unroll 1
+        for (int layer = 0; layer < 2; ++layer) {
+          wait_bar(mbar, ph);
+          ph ^= 1;
+          wg_bar(wgid);
+          fence_after();
+          hidden();
+          fence_before();
+          wg_bar(wgid);
+          if (row == 0) {
+            fence_after();
+            const uint64_t dW = layer == 0 ? dW2 : dW3;
+            const uint32_t id = layer == 0 ? id_hidden : id_out;
 #pragma unroll
-      for (uint32_t k = 0; k < L::KH / 16; ++k)
-        umma(tmem_wg, smem_desc(sH + k * 256, L::KH), smem_desc(sW3 + k * 256, L::KH), id_out, k);
-      umma_commit(bar);
-    }
-    if (!mbar_wait(bar, phase)) {
-      atomicOr(status, 1u);
-      abort_flag[wg] = 1;
-    }
-    phase ^= 1;
-    fence_after();
-    uint32_t o[16];
-    tmem_ld16(tmem_row, o);
-    tmem_wait_ld();
-    if (valid && !bad) {
-      float *dst = out + (size_t)oi * C;
+            for (uint32_t kq = 0; kq < L::KH / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW + 16 * kq, id, kq);
+            umma_commit(mbar);
+          }
+        }
+        wait_bar(mbar, ph);
+        ph ^= 1;
+        wg_bar(wgid);
+        fence_after();
+        uint32_t o[16];
+        tmem_ld16(tD + lanes, o);
+        tmem_wait_ld();
+        if (good) {
+          // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
+          float y[CP];
 #pragma unroll
-      for (int c = 0; c < 16; ++c)
-        if (c < (int)C) dst[c] = 1.0f / (1.0f + __expf(-__uint_as_float(o[c])));
+          for (int cc = 0; cc < CP; ++cc) {
+            float th;
+            asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
+            y[cc] = fmaf(0.5f, th, 0.5f);
+          }
+          float *dst = out + (size_t)oi * C;
+          if (CP == 8 && vec_out && C == 8) {
+            reinterpret_cast<float4 *>(dst)[0] = make_float4(y[0], y[1], y[2], y[3]);
+            reinterpret_cast<float4 *>(dst)[1] = make_float4(y[4], y[5], y[6], y[7]);
+          } else {
+#pragma unroll
+            for (int cc = 0; cc < CP; ++cc)
+              if (cc < (int)C) dst[cc] = y[cc];
+          }
+        }
+        fence_before();
+      }
+      // every warp of this warpgroup takes the same decision to stop
+      if (row == 0) stop_flag[c] = *abort_flag;
+      wg_bar(wgid);
+      if (stop_flag[c]) break;
     }
-    fence_before();
-    wg_bar(wg);
-    if (abort_flag[wg]) break;
   }
   fence_before();
   __syncthreads();
   if (warp == 0) {
     fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(kCols)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(TC::alloc)
                  : "memory");
   }
 }
 
-template <int H, int NWG, bool BF16>
-cudaError_t launch_tc_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
-                        float *out, unsigned long long *err, unsigned int *status, int num_sms,
-                        cudaStream_t st) {
-  using L = TcLayout<H>;
-  const size_t smem = (size_t)NWG * L::WG + NWG * 8 + 8 + 4 * NWG;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_decode_tc<H, NWG, BF16>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+template <int H, bool BF16, bool TRI, int NP, int NC, int S>
+cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, float *out,
+                        unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
+  using M = TmSmem<H, NC, S>;
+  const size_t smem = M::total;
+  const bool c8 = W.out_dim <= 8;
+  static bool attr[2] = {false, false};
+  if (!attr[c8]) {
+    // as little shared memory as the kernel needs: the rest of the array is L1
+    const int carve = (int)((smem * 100 + 232448 - 1) / 232448);
+    cudaError_t e;
+    if (c8) {
+      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, S>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, S>,
+                                 cudaFuncAttributePreferredSharedMemoryCarveout, carve);
+    } else {
+      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, S>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, S>,
+                                 cudaFuncAttributePreferredSharedMemoryCarveout, carve);
+    }
     if (e != cudaSuccess) return e;
-    attr = true;
+    attr[c8] = true;
   }
   const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms;
-  const size_t need = (max_tiles + NWG - 1) / NWG;
-  if (grid > need) grid = need;
-  k_decode_tc<H, NWG, BF16><<<(unsigned)grid, NWG * 128, smem, st>>>(A, W, B, out, err, status);
+  if (grid > max_tiles) grid = max_tiles;
+  const int vec_out = ((uintptr_t)out & 15) == 0;
+  const unsigned threads = (NP + NC) * 128;
+  if (c8)
+    k_decode_tm<H, BF16, TRI, 8, NP, NC, S><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+  else
+    k_decode_tm<H, BF16, TRI, 16, NP, NC, S><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
   return cudaGetLastError();
 }
 
@@ -416,11 +744,17 @@ cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Bucke
                              float *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches) {
   *launches += 1;
-  if (W.hidden == 64)
-    return bf16 ? launch_tc_t<64, 4, true>(A, W, B, n, out, err, status, num_sms, st)
-                : launch_tc_t<64, 4, false>(A, W, B, n, out, err, status, num_sms, st);
-  return bf16 ? launch_tc_t<128, 2, true>(A, W, B, n, out, err, status, num_sms, st)
-              : launch_tc_t<128, 2, false>(A, W, B, n, out, err, status, num_sms, st);
+  const bool tri = A.num_mips > 1;
+#define NTC_WS(H, TRI, NP, NC, S)                                                                \
+  return bf16 ? launch_tm_t<H, true, TRI, NP, NC, S>(A, W, B, n, out, err, status, num_sms, st) \
+              : launch_tm_t<H, false, TRI, NP, NC, S>(A, W, B, n, out, err, status, num_sms, st)
+  if (W.hidden == 64) {
+    if (tri) NTC_WS(64, true, 2, 2, 8);
+    NTC_WS(64, false, 4, 3, 8);
+  }
+  if (tri) NTC_WS(128, true, 2, 2, 4);
+  NTC_WS(128, false, 2, 2, 4);
+#undef NTC_WS
 }
 
 }  // namespace ntc
