@@ -75,6 +75,26 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   return true;
 }
 
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Like mbar_wait but polls without suspending (lower wake-up latency).
+__device__ __forceinline__ bool mbar_spin(uint32_t bar, uint32_t parity) {
+  if (mbar_test(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (!mbar_test(bar, parity))
+    if (global_ns() - t0 > kWaitLimitNs) return false;
+  return true;
+}
+
 __device__ __forceinline__ void fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
 }
@@ -385,7 +405,8 @@ struct TmSmem {
   static constexpr int nbars = 2 * S + 2 * NC;                          // full, empty, mma, weights
   static constexpr size_t misc = bars + (size_t)nbars * 8;
   static constexpr size_t tiles = misc + 64;
-  static constexpr size_t total = tiles + 2 * kSmemTileTable * 4;
+  static constexpr size_t grids = tiles + 2 * kSmemTileTable * 4;
+  static constexpr size_t total = grids + kSmemGrids * sizeof(GridDesc);
 };
 
 // Tensor-memory plan (columns): consumer c owns [c*SC, c*SC + H) for the fp32
@@ -447,6 +468,13 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     seg = s_seg;
     tst = s_tst;
   }
+  const GridDesc *grids = A.grids;
+  const uint32_t ngrids = A.num_sets * kLevels * A.num_mips;
+  if (ngrids <= kSmemGrids) {
+    GridDesc *s_grids = reinterpret_cast<GridDesc *>(smem + M::grids);
+    for (uint32_t i = threadIdx.x; i < ngrids; i += blockDim.x) s_grids[i] = A.grids[i];
+    grids = s_grids;
+  }
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
       mbar_init(full_bar(i), 4);   // one arrival per producer warp
@@ -494,7 +522,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       const bool valid = (uint32_t)row < len;
       const bool good = valid && dec < D && !query_bad(A, q);
       Taps<TRI> taps;
-      issue_taps<TRI>(A, A.grids, q, good, taps);
+      issue_taps<TRI>(A, grids, q, good, taps);
       // bad rows (set id out of range, non-finite UV, or the bad bucket) decode to NaN
       const bool bad = valid && !good;
       const uint32_t badm = __ballot_sync(0xFFFFFFFFu, bad);
@@ -543,7 +571,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
     const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
     auto wait_bar = [&](uint32_t b, uint32_t parity) {
-      if (poller && !mbar_wait(b, parity)) {
+      if (poller && !mbar_spin(b, parity)) {
         atomicOr(status, 1u);
         *abort_flag = 1;
       }
@@ -568,13 +596,16 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       }
       tmem_wait_st();
     };
-    for (uint32_t k = c; k < K; k += NC) {
+    // Start tile k: its output rows, its decoder's weights, wait for its A
+    // stage and issue layer 1.  Requires this consumer's previous tile to have
+    // finished all MMAs.
+    auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good) {
       const uint32_t t = blockIdx.x + k * grid, s = k % S, n = k / S;
-      uint32_t dec, start, len;
+      uint32_t start, len;
       tile_lookup(seg, tst, D, t, dec, start, len);
-      const uint32_t oi = (uint32_t)row < len ? __ldg(B.perm + start + row) : 0u;
+      oi = (uint32_t)row < len ? __ldg(B.perm + start + row) : 0u;
       bool wpend = false;
-      if (dec < D && dec != cur) {  // this consumer's previous tile is complete
+      if (dec < D && dec != cur) {
         if (row == 0) bulk_g2s(sW1, W.tc + (size_t)dec * W.tc_stride, L::WIMG, wbar);
         wpend = true;
         cur = dec;
@@ -585,7 +616,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         wph ^= 1;
       }
       wg_bar(wgid);
-      const bool good = smem[M::flags + s * 128 + row] != 0;
+      good = smem[M::flags + s * 128 + row] != 0;
       if (row == 0) {
         fence_after();
         if (dec < D) {
@@ -598,6 +629,12 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
           mbar_arrive(empty_bar(s));  // a tile of bad queries: nothing to multiply
         }
       }
+    };
+    uint32_t k = c, dec = D, oi = 0;
+    bool good = false;
+    if (k < K) begin(k, dec, oi, good);
+    while (k < K) {
+      uint32_t o[16];
       if (dec < D) {
 #pragma unroll 1
         for (int layer = 0; layer < 2; ++layer) {
@@ -621,30 +658,38 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         ph ^= 1;
         wg_bar(wgid);
         fence_after();
-        uint32_t o[16];
         tmem_ld16(tD + lanes, o);
         tmem_wait_ld();
-        if (good) {
-          // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
-          float y[CP];
-#pragma unroll
-          for (int cc = 0; cc < CP; ++cc) {
-            float th;
-            asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
-            y[cc] = fmaf(0.5f, th, 0.5f);
-          }
-          float *dst = out + (size_t)oi * C;
-          if (CP == 8 && vec_out && C == 8) {
-            reinterpret_cast<float4 *>(dst)[0] = make_float4(y[0], y[1], y[2], y[3]);
-            reinterpret_cast<float4 *>(dst)[1] = make_float4(y[4], y[5], y[6], y[7]);
-          } else {
-#pragma unroll
-            for (int cc = 0; cc < CP; ++cc)
-              if (cc < (int)C) dst[cc] = y[cc];
-          }
-        }
         fence_before();
       }
+      // the next tile's layer 1 runs while this tile's outputs are written
+      const uint32_t kn = k + NC;
+      uint32_t ndec = D, noi = 0;
+      bool ngood = false;
+      if (kn < K) begin(kn, ndec, noi, ngood);
+      if (dec < D && good) {
+        // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
+        float y[CP];
+#pragma unroll
+        for (int cc = 0; cc < CP; ++cc) {
+          float th;
+          asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
+          y[cc] = fmaf(0.5f, th, 0.5f);
+        }
+        float *dst = out + (size_t)oi * C;
+        if (CP == 8 && vec_out && C == 8) {
+          reinterpret_cast<float4 *>(dst)[0] = make_float4(y[0], y[1], y[2], y[3]);
+          reinterpret_cast<float4 *>(dst)[1] = make_float4(y[4], y[5], y[6], y[7]);
+        } else {
+#pragma unroll
+          for (int cc = 0; cc < CP; ++cc)
+            if (cc < (int)C) dst[cc] = y[cc];
+        }
+      }
+      k = kn;
+      dec = ndec;
+      oi = noi;
+      good = ngood;
       // every warp of this warpgroup takes the same decision to stop
       if (row == 0) stop_flag[c] = *abort_flag;
       wg_bar(wgid);
