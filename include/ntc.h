@@ -209,7 +209,7 @@ NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
  * 16-byte aligned).  Its scratch is one file-scope device array of 1,360,896
  * bytes that every GPU loading the library holds until the process exits, so:
  *   - num_sets <= 65536, num_decoders <= 4095 and
- *     (num_decoders + 1) * ceil(n / 4096) <= 262144 (larger calls return
+ *     (num_decoders + 1) * ceil(n / 2048) <= 262144 (larger calls return
  *     NTC_ERR_UNSUPPORTED and enqueue nothing);
  *   - every call on a device shares that array and it keeps the previous
  *     call's contents; the call clears what must start at zero itself, but two

@@ -9,8 +9,9 @@
 //   k_scan    one CTA per decoder scans that decoder's per-chunk counts; the last
 //             CTA to finish (atomic ticket) scans the decoder totals into the
 //             segment starts and the tile starts
-//   k_scatter recomputes each warp's counts, turns them into running bases and
-//             writes perm[] and the sorted query records
+//   k_scatter recomputes each warp's counts, sorts its chunk stably by decoder
+//             in shared memory, then copies each decoder's run out to its
+//             segment with coalesced stores (perm[] and the sorted records)
 // A query whose set id is out of range goes to the extra bucket D.
 #include "ntc_internal.cuh"
 
@@ -142,64 +143,106 @@ __global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks
   (void)n;
 }
 
+// In-place exclusive scan of len values (in shared memory) by the 256 threads of
+// a block, each over a contiguous run of ceil(len / 256) values.
+__device__ void block_scan_256(uint32_t *a, uint32_t len) {
+  __shared__ uint32_t wsum[kWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t per = (len + kBucketThreads - 1) / kBucketThreads;
+  const uint32_t b = threadIdx.x * per, e = min(len, b + per);
+  uint32_t s = 0;
+  for (uint32_t i = b; i < e; ++i) s += a[i];
+  uint32_t x = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  uint32_t wp = 0;
+  for (int w = 0; w < warp; ++w) wp += wsum[w];
+  uint32_t run = wp + x - s;
+  for (uint32_t i = b; i < e; ++i) {
+    const uint32_t c = a[i];
+    a[i] = run;
+    run += c;
+  }
+  __syncthreads();
+}
+
 __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_query *q, size_t n,
                                                             const uint32_t *counts, uint32_t chunks,
                                                             const uint32_t *meta, uint32_t *perm,
                                                             ntc_query *sorted) {
-  extern __shared__ uint32_t cnt[];  // [kWarps][D+1]
+  // shared memory: chunk-local index [chunk] (u16) and decoder [chunk] (u16) of
+  // every sorted slot, then per-warp counters [kWarps][D+1] and the chunk's
+  // per-decoder local offsets and global bases [D+1] each
+  extern __shared__ uint32_t sm32[];
+  uint16_t *sidx = reinterpret_cast<uint16_t *>(sm32);
+  uint16_t *sdec = sidx + kBucketChunk;
+  uint32_t *cnt = reinterpret_cast<uint32_t *>(sdec + kBucketChunk);
   const uint32_t D1 = A.num_decoders + 1;
+  uint32_t *loff = cnt + kWarps * D1;  // chunk-local start of each decoder's run
+  uint32_t *gbase = loff + D1;         // global position of that run's first element
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
   __syncthreads();
-  const size_t base = (size_t)blockIdx.x * kBucketChunk + (size_t)warp * (kBucketItems * 32);
-  uint4 rec[kBucketItems];
+  const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
+  const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
   uint32_t dec[kBucketItems];
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
-    size_t i = base + (size_t)it * 32 + lane;
-    if (i < n) {
-      rec[it] = __ldg(reinterpret_cast<const uint4 *>(q + i));
-      dec[it] = decoder_of(A, rec[it].x);
-    } else {
-      dec[it] = 0xFFFFFFFFu;
-    }
+    const size_t i = cbase + wbase + (size_t)it * 32 + lane;
+    dec[it] = i < n ? decoder_of(A, __ldg(&q[i].set_id)) : 0xFFFFFFFFu;
   }
   uint32_t *my = cnt + warp * D1;
-#pragma unroll
-  for (int it = 0; it < kBucketItems; ++it) {
-    const uint32_t d = dec[it];
-    const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
-    if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
-    __syncwarp();
-  }
-  __syncthreads();
-  // running base of (warp, decoder) = segment start + this chunk's offset in
-  // the decoder's segment + the counts of the earlier warps of this chunk
-  const uint32_t *seg = meta + 1;
-  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
-    uint32_t run = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      uint32_t c = cnt[w * D1 + d];
-      cnt[w * D1 + d] = run;
-      run += c;
-    }
-  }
-  __syncthreads();
+  // rank of each query among the equal decoders of this warp's run, in order
+  uint32_t rank[kBucketItems];
   const uint32_t lt = (1u << lane) - 1u;
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
     const uint32_t d = dec[it];
     const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
-    if (d != 0xFFFFFFFFu) {
-      uint32_t pos = my[d] + __popc(m & lt);
-      size_t i = base + (size_t)it * 32 + lane;
-      perm[pos] = (uint32_t)i;
-      reinterpret_cast<uint4 *>(sorted)[pos] = rec[it];
-    }
+    rank[it] = d != 0xFFFFFFFFu ? my[d] + __popc(m & lt) : 0u;
     __syncwarp();
     if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
     __syncwarp();
+  }
+  __syncthreads();
+  // per decoder: warp prefix (in place), chunk total and global base
+  const uint32_t *seg = meta + 1;
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
+    uint32_t run = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const uint32_t c = cnt[w * D1 + d];
+      cnt[w * D1 + d] = run;
+      run += c;
+    }
+    loff[d] = run;
+    gbase[d] = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
+  }
+  __syncthreads();
+  block_scan_256(loff, D1);  // exclusive scan of the chunk totals over decoders
+  // stable local sort of (local index, decoder) pairs
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) {
+    const uint32_t d = dec[it];
+    if (d == 0xFFFFFFFFu) continue;
+    const uint32_t lp = loff[d] + cnt[warp * D1 + d] + rank[it];
+    sidx[lp] = (uint16_t)(wbase + it * 32 + lane);
+    sdec[lp] = (uint16_t)d;
+  }
+  __syncthreads();
+  // coalesced copy-out: consecutive slots of one decoder go to consecutive
+  // positions of that decoder's segment; the record is re-read (L1/L2 hit)
+  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+  for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
+    const uint32_t d = sdec[i], j = sidx[i];
+    const uint32_t pos = gbase[d] + (i - loff[d]);
+    perm[pos] = (uint32_t)(cbase + j);
+    reinterpret_cast<uint4 *>(sorted)[pos] = __ldg(reinterpret_cast<const uint4 *>(q + cbase + j));
   }
 }
 
@@ -232,6 +275,7 @@ cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const S
   const uint32_t chunks = (uint32_t)((n + kBucketChunk - 1) / kBucketChunk);
   const uint32_t D = A.num_decoders;
   const size_t smem = (size_t)kWarps * (D + 1) * sizeof(uint32_t);
+  const size_t smem_scatter = (size_t)kBucketChunk * (2 + 2) + smem + 2 * (D + 1) * sizeof(uint32_t);
   static bool attr_done = false;
   if (!attr_done) {
     cudaFuncSetAttribute(k_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
@@ -243,7 +287,7 @@ cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const S
   uint32_t *ticket = totals + (D + 1);
   k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks);
   k_scan<<<D + 1, 1024, 0, st>>>(s.counts, chunks, D, (uint32_t)n, totals, s.meta, ticket);
-  k_scatter<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks, s.meta, s.perm, s.sorted);
+  k_scatter<<<chunks, kBucketThreads, smem_scatter, st>>>(A, q, n, s.counts, chunks, s.meta, s.perm, s.sorted);
   *launches += 3;
   return cudaGetLastError();
 }

@@ -24,7 +24,7 @@ namespace {
 
 constexpr size_t kMapWords = 65536;    // set->decoder map copy
 constexpr size_t kMetaWords = 12544;   // meta (2D+5) + totals (D+1) + ticket (1), D <= 4095
-constexpr size_t kCountWords = 262144; // (D+1) * ceil(n / 4096) per-chunk counts
+constexpr size_t kCountWords = 262144; // (D+1) * ceil(n / 2048) per-chunk counts
 constexpr size_t kStaticWords = kMapWords + kMetaWords + kCountWords;  // 1,360,896 bytes
 
 // The scratch.  In host code this name is only a host-side stand-in: kernels
@@ -58,7 +58,7 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
     return failed(NTC_ERR_INVALID_ARG, "query buffers must be 16-byte aligned");
   if (bucket_scratch_counts(num_decoders, n) > kCountWords)
     return failed(NTC_ERR_UNSUPPORTED,
-                  "(num_decoders + 1) * ceil(n / 4096) exceeds the static scratch (262144 counts)");
+                  "(num_decoders + 1) * ceil(n / 2048) exceeds the static scratch (262144 counts)");
   for (uint32_t s = 0; s < num_sets; ++s)
     if (h_set_to_decoder[s] >= num_decoders)
       return failed(NTC_ERR_INVALID_ARG, "set_to_decoder entry is not a decoder");

@@ -216,7 +216,7 @@ struct Scratch {
 };
 
 constexpr int kBucketThreads = 256;
-constexpr int kBucketItems = 16;  // queries per thread
+constexpr int kBucketItems = 8;  // queries per thread
 constexpr int kBucketChunk = kBucketThreads * kBucketItems;
 
 cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,

@@ -44,7 +44,7 @@ def test_static_bucketing_rejects_sizes_beyond_its_scratch():
     w = W.config(1, "small")
     qd = ntc.queries_to_device(w.queries)
     m = np.zeros(1, dtype=np.uint32)
-    n_too_many = 262144 // 4096 * 4096 * 2  # (4095 + 1) * ceil(n / 4096) > 262144
+    n_too_many = 262144 // 4096 * 4096 * 2  # (4095 + 1) * ceil(n / 2048) > 262144
     with pytest.raises(ntc.NtcError, match="static scratch"):
         ntc.ntc_bucket_static(m.ctypes.data, 1, 4095, qd.data_ptr(), n_too_many, qd.data_ptr(),
                               qd.data_ptr(), 0)
