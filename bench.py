@@ -159,16 +159,28 @@ def dist_env():
 
 
 def workload(small: bool, rank: int):
+    """The benchmark batch of one rank: the same assets on every rank, a
+    rank-specific query stream (queries are sharded, assets replicated)."""
     from paper_2608_27888_gb300 import workloads as W
-    if small:
-        w = W.config(2, "small")
-    else:
-        seed = W.BASE_SEED + 2
-        S, T, n = 16, 1024, 4_194_304
-        a = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
-        q = W.queries_uniform(seed + 1000 * rank, n, S)
-        w = W.Workload("config2-full", a, q, {})
-    return w
+    seed = W.BASE_SEED + 2
+    S, T, n = (16, 128, 40_077) if small else (16, 1024, 4_194_304)
+    a = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
+    q = W.queries_uniform(seed + 1000 * rank, n, S)
+    return W.Workload("config2-small" if small else "config2-full", a, q, {})
+
+
+def aggregate(n_per_rank: int, ms_local: float, dist=None):
+    """Whole-job throughput: all ranks' queries over the slowest rank's step time."""
+    ws = 1
+    ms = ms_local
+    if dist is not None and dist.is_initialized():
+        import torch
+        ws = dist.get_world_size()
+        t = torch.tensor([ms_local], dtype=torch.float64,
+                         device="cuda" if dist.get_backend() == "nccl" else "cpu")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return n_per_rank * ws / (ms / 1e3), ms
 
 
 def mean_distinct(q, assets):
@@ -266,12 +278,7 @@ def main():
     sampler.start()
     ms, stages, launches = timed_steps(args.mode, args.steps, args.warmup, stages=True)
     clocks = sampler.stop()
-    ms_step = statistics.mean(ms)
-    if dist is not None:
-        t = torch.tensor([ms_step], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_step = float(t.item())
-    value = n * ws / (ms_step / 1e3)
+    value, ms_step = aggregate(n, statistics.mean(ms), dist)
     bucket_ms = statistics.mean(s[0] for s in stages)
     decode_ms = statistics.mean(s[1] for s in stages)
 
