@@ -396,9 +396,10 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 // (the B operands) and bookkeeping live in shared memory; every A operand and
 // accumulator lives in tensor memory, so most of the SM's L1/shared array stays
 // L1, which holds the in-flight latent gathers.
-template <int H, int NC, int S>
+template <int H, int NC, int SC>
 struct TmSmem {
   using L = TcLayout<H>;
+  static constexpr int S = NC * SC;                                     // stages in all rings
   static constexpr size_t weights = 0;                                  // per consumer
   static constexpr size_t flags = weights + (size_t)NC * L::WIMG;       // per stage: 128 row flags
   static constexpr size_t bars = flags + (size_t)S * 128;
@@ -409,41 +410,52 @@ struct TmSmem {
   static constexpr size_t total = grids + kSmemGrids * sizeof(GridDesc);
 };
 
-// Tensor-memory plan (columns): consumer c owns [c*SC, c*SC + H) for the fp32
-// accumulator and [c*SC + H, c*SC + H + KH/2) for its hidden A operand (two
-// 16-bit K elements per column); ring stage s owns 16 columns at RING + 16 s for
-// the layer-1 A operand [128 x 32].
-template <int H, int NC, int S>
+// Tensor-memory plan (columns).  Consumer c owns CS columns from c*CS: the fp32
+// accumulator at +0 (H columns), its hidden A operand at +H (KH/2 columns, two
+// 16-bit K elements per column) and the layer-1 A operands [128 x 32] of its SC
+// ring stages at +AOFF + 16 st (16 columns each).  Accumulators stay 32-column
+// aligned and every A operand 16-column aligned.
+template <int H, int NC, int SC>
 struct TmCols {
   static constexpr uint32_t KH = H + 16;
-  static constexpr uint32_t SC = ((H + KH / 2) + 31) / 32 * 32;  // consumer stride, 32-aligned
-  static constexpr uint32_t RING = NC * SC;
-  static constexpr uint32_t used = RING + 16 * S;
+  static constexpr uint32_t AOFF = (H + KH / 2 + 15) / 16 * 16;
+  static constexpr uint32_t CS = (AOFF + 16 * SC + 31) / 32 * 32;
+  static constexpr uint32_t used = NC * CS;
   static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
   static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
+  // layer-1 A operand of stage s (= consumer * SC + st)
+  static __device__ __forceinline__ uint32_t a1(uint32_t s) { return (s / SC) * CS + AOFF + 16 * (s % SC); }
 };
 
 // Warp-specialised gather-decode with tensor-memory operands.
-//   Producer warpgroups 0..NP-1 gather: each thread computes the taps of one
-//   query row, blends them in fp32 and stores the fp16/bf16 feature row (plus the
-//   bias column) into the TMEM A region of one ring stage (tcgen05.st; warp q of
-//   a warpgroup owns TMEM lanes 32q..32q+31, exactly its rows).  Producer p takes
-//   the CTA's local tiles k = p, p + NP, ...; the query record of its next tile is
-//   loaded while the current one is gathered.
-//   Consumer warpgroups NP..NP+NC-1 each take local tiles k = c, c + NC, ...:
-//   layer 1 reads A from the stage's TMEM region and B (weights) from shared
-//   memory, the ReLU/convert epilogue goes TMEM -> registers -> TMEM, layers 2
-//   and 3 read their A from TMEM too, and the sigmoid epilogue scatters rows to
-//   out[perm[i]].  Stage hand-off uses full/empty mbarriers: four producer-warp
-//   arrivals fill a stage, the completion of the layer-1 MMA empties it.
+//   Consumer warpgroups (the last NC) each decode the CTA's local tiles
+//   k = c, c + NC, ... (j = k / NC counts a consumer's tiles).  Each consumer has
+//   a private ring of SC stages in tensor memory, filled by its own R = NP / NC
+//   producer warpgroups: tile j of consumer c is gathered by producer c + NC *
+//   (j mod R) into stage j mod SC.  SC is a multiple of R, so every stage has one
+//   producer and one consumer and successive uses of a stage are ordered by
+//   program order on both sides -- an mbarrier parity wait can then never be two
+//   phases ahead of its barrier.
+//   Producer: each thread computes the taps of one query row, blends them in
+//   fp32 and stores the fp16/bf16 feature row (plus the bias column) into the
+//   stage's TMEM A region (tcgen05.st; warp q of a warpgroup owns TMEM lanes
+//   32q..32q+31, exactly its rows); four warp arrivals fill the stage.  The next
+//   tile's query record is loaded while the current one is gathered.
+//   Consumer: layer 1 reads A from the stage and B (weights) from shared memory;
+//   its completion empties the stage; the ReLU/convert epilogue goes TMEM ->
+//   registers -> TMEM; layers 2 and 3 read their A from TMEM too; the sigmoid
+//   epilogue scatters rows to out[perm[i]] while the next tile's layer 1 runs.
 // CTA b owns the global tiles b, b + grid, b + 2 grid, ...
-template <int H, bool BF16, bool TRI, int CP, int NP, int NC, int S>
+template <int H, bool BF16, bool TRI, int CP, int NP, int NC, int SC>
 __global__ void __launch_bounds__((NP + NC) * 128, 1)
     k_decode_tm(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
                 unsigned int *status, int vec_out) {
+  static_assert(NP % NC == 0 && SC % (NP / NC) == 0, "each ring stage needs one producer");
+  constexpr int R = NP / NC;  // producers per consumer
+  constexpr int S = NC * SC;
   using L = TcLayout<H>;
-  using M = TmSmem<H, NC, S>;
-  using TC = TmCols<H, NC, S>;
+  using M = TmSmem<H, NC, SC>;
+  using TC = TmCols<H, NC, SC>;
   extern __shared__ __align__(128) uint8_t smem[];
   const int role = threadIdx.x >> 7, row = threadIdx.x & 127, warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -503,20 +515,22 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
 
   if (role < NP) {
     // ------------------------------------------------------------ producer
-    uint32_t k = role;
+    const uint32_t pc = role % NC, pq = role / NC;  // serves consumer pc, tiles j = pq mod R
+    auto tile_of = [&](uint32_t j) { return pc + NC * j; };
+    uint32_t j = pq;
     uint32_t dec = D, start = 0, len = 0;
     ntc_query q;
-    if (k < K) {
-      tile_lookup(seg, tst, D, blockIdx.x + k * grid, dec, start, len);
+    if (tile_of(j) < K) {
+      tile_lookup(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
       if ((uint32_t)row < len) q = load_query(B.sorted + start + row);
     }
-    for (; k < K; k += NP) {
+    for (; tile_of(j) < K; j += R) {
       if (*abort_flag) break;
       // the next tile's query record goes in flight first
       uint32_t ndec = D, nstart = 0, nlen = 0;
       ntc_query nq;
-      if (k + NP < K) {
-        tile_lookup(seg, tst, D, blockIdx.x + (k + NP) * grid, ndec, nstart, nlen);
+      if (tile_of(j + R) < K) {
+        tile_lookup(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
         if ((uint32_t)row < nlen) nq = load_query(B.sorted + nstart + row);
       }
       const bool valid = (uint32_t)row < len;
@@ -541,13 +555,13 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       a[8] = one;
 #pragma unroll
       for (int i = 9; i < 16; ++i) a[i] = 0u;
-      const uint32_t s = k % S, n = k / S;
+      const uint32_t s = pc * SC + j % SC, n = j / SC;
       if (!mbar_wait(empty_bar(s), (n & 1) ^ 1)) {  // the stage's previous tile has left layer 1
         atomicOr(status, 1u);
         *abort_flag = 1;
       }
       fence_after();
-      tmem_st16(tmem_base + TC::RING + 16 * s + lanes, a);
+      tmem_st16(tmem_base + TC::a1(s) + lanes, a);
       tmem_wait_st();
       smem[M::flags + s * 128 + row] = good ? 1 : 0;
       fence_before();
@@ -563,7 +577,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const int c = role - NP;
     const int wgid = role;  // named barrier id role + 1
     const bool poller = (row >> 5) == 0;
-    const uint32_t tD = tmem_base + c * TC::SC;  // accumulator
+    const uint32_t tD = tmem_base + c * TC::CS;  // accumulator
     const uint32_t tH = tD + H;                  // hidden A operand
     const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
     const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
@@ -600,7 +614,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     // stage and issue layer 1.  Requires this consumer's previous tile to have
     // finished all MMAs.
     auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good) {
-      const uint32_t t = blockIdx.x + k * grid, s = k % S, n = k / S;
+      const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
       uint32_t start, len;
       tile_lookup(seg, tst, D, t, dec, start, len);
       oi = (uint32_t)row < len ? __ldg(B.perm + start + row) : 0u;
@@ -620,7 +634,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       if (row == 0) {
         fence_after();
         if (dec < D) {
-          const uint32_t tA = tmem_base + TC::RING + 16 * s;
+          const uint32_t tA = tmem_base + TC::a1(s);
 #pragma unroll
           for (uint32_t kq = 0; kq < kTcKA / 16; ++kq) umma_ta(tD, tA + 8 * kq, dW1 + 16 * kq, id_hidden, kq);
           umma_commit(mbar);
@@ -705,10 +719,10 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   }
 }
 
-template <int H, bool BF16, bool TRI, int NP, int NC, int S>
+template <int H, bool BF16, bool TRI, int NP, int NC, int SC>
 cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, float *out,
                         unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
-  using M = TmSmem<H, NC, S>;
+  using M = TmSmem<H, NC, SC>;
   const size_t smem = M::total;
   const bool c8 = W.out_dim <= 8;
   static bool attr[2] = {false, false};
@@ -717,16 +731,16 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
     const int carve = (int)((smem * 100 + 232448 - 1) / 232448);
     cudaError_t e;
     if (c8) {
-      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, S>,
+      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, SC>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, S>,
+        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, SC>,
                                  cudaFuncAttributePreferredSharedMemoryCarveout, carve);
     } else {
-      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, S>,
+      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, SC>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, S>,
+        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, SC>,
                                  cudaFuncAttributePreferredSharedMemoryCarveout, carve);
     }
     if (e != cudaSuccess) return e;
@@ -738,9 +752,9 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   const int vec_out = ((uintptr_t)out & 15) == 0;
   const unsigned threads = (NP + NC) * 128;
   if (c8)
-    k_decode_tm<H, BF16, TRI, 8, NP, NC, S><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+    k_decode_tm<H, BF16, TRI, 8, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
   else
-    k_decode_tm<H, BF16, TRI, 16, NP, NC, S><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+    k_decode_tm<H, BF16, TRI, 16, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
   return cudaGetLastError();
 }
 
@@ -790,15 +804,15 @@ cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Bucke
                              int num_sms, cudaStream_t st, int *launches) {
   *launches += 1;
   const bool tri = A.num_mips > 1;
-#define NTC_WS(H, TRI, NP, NC, S)                                                                \
-  return bf16 ? launch_tm_t<H, true, TRI, NP, NC, S>(A, W, B, n, out, err, status, num_sms, st) \
-              : launch_tm_t<H, false, TRI, NP, NC, S>(A, W, B, n, out, err, status, num_sms, st)
+#define NTC_WS(H, TRI, NP, NC, SC)                                                                \
+  return bf16 ? launch_tm_t<H, true, TRI, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st) \
+              : launch_tm_t<H, false, TRI, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st)
   if (W.hidden == 64) {
-    if (tri) NTC_WS(64, true, 2, 2, 8);
-    NTC_WS(64, false, 4, 3, 8);
+    if (tri) NTC_WS(64, true, 2, 2, 2);
+    NTC_WS(64, false, 4, 4, 1);
   }
-  if (tri) NTC_WS(128, true, 2, 2, 4);
-  NTC_WS(128, false, 2, 2, 4);
+  if (tri) NTC_WS(128, true, 2, 2, 2);
+  NTC_WS(128, false, 2, 2, 2);
 #undef NTC_WS
 }
 
