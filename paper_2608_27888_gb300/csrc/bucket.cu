@@ -24,24 +24,60 @@ __device__ __forceinline__ uint32_t decoder_of(const Assets &A, uint32_t set_id)
   return set_id < A.num_sets ? __ldg(A.map + set_id) : A.num_decoders;
 }
 
+__device__ __forceinline__ uint32_t saddr_b(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// Stream `bytes` (a multiple of 16) from global memory into shared memory with
+// one bulk copy (TMA) and wait for it; false if the copy has not landed after
+// 200 ms.  Called by every thread of the block; thread 0 issues the copy.
+__device__ bool bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+  const uint32_t b = saddr_b(bar);
+  if (threadIdx.x == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(b) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(b), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
+                     saddr_b(dst)),
+                 "l"(src), "r"(bytes), "r"(b)
+                 : "memory");
+  }
+  uint64_t t0 = 0;
+  for (uint32_t spin = 0;; ++spin) {
+    uint32_t ok;
+    asm volatile(
+        "{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\nselp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(b)
+        : "memory");
+    if (ok) return true;
+    uint64_t now;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(now));
+    if (spin == 0) t0 = now;
+    else if (now - t0 > 200ull * 1000ull * 1000ull) return false;
+  }
+}
+
 __global__ void __launch_bounds__(kBucketThreads) k_hist(Assets A, const ntc_query *q, size_t n,
-                                                         uint32_t *counts, uint32_t chunks) {
-  extern __shared__ uint32_t cnt[];  // [kWarps][D+1]
+                                                         uint32_t *counts, uint32_t chunks,
+                                                         unsigned int *status) {
+  // shared memory: the chunk's records [kBucketChunk], then [kWarps][D+1] counters
+  extern __shared__ uint4 srec[];
+  __shared__ uint64_t bar;
+  uint32_t *cnt = reinterpret_cast<uint32_t *>(srec + kBucketChunk);
   const uint32_t D1 = A.num_decoders + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
+  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
-  __syncthreads();
-  const size_t base = (size_t)blockIdx.x * kBucketChunk + (size_t)warp * (kBucketItems * 32);
-  uint32_t dec[kBucketItems];
-#pragma unroll
-  for (int it = 0; it < kBucketItems; ++it) {
-    size_t i = base + (size_t)it * 32 + lane;
-    dec[it] = i < n ? decoder_of(A, __ldg(&q[i].set_id)) : 0xFFFFFFFFu;
-  }
+  if (!bulk_load(srec, q + cbase, valid * 16u, &bar)) atomicOr(status, 2u);
+  const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);
   uint32_t *my = cnt + warp * D1;
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
-    const uint32_t d = dec[it];
+    const uint32_t j = wbase + it * 32 + lane;
+    const uint32_t d = j < valid ? decoder_of(A, srec[j].x) : 0xFFFFFFFFu;
     const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
     if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
     __syncwarp();
@@ -174,27 +210,30 @@ __device__ void block_scan_256(uint32_t *a, uint32_t len) {
 __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_query *q, size_t n,
                                                             const uint32_t *counts, uint32_t chunks,
                                                             const uint32_t *meta, uint32_t *perm,
-                                                            ntc_query *sorted) {
-  // shared memory: chunk-local index [chunk] (u16) and decoder [chunk] (u16) of
-  // every sorted slot, then per-warp counters [kWarps][D+1] and the chunk's
-  // per-decoder local offsets and global bases [D+1] each
-  extern __shared__ uint32_t sm32[];
-  uint16_t *sidx = reinterpret_cast<uint16_t *>(sm32);
+                                                            ntc_query *sorted, unsigned int *status) {
+  // shared memory: the chunk's records [chunk] (16 B), the chunk-local index
+  // [chunk] (u16) and decoder [chunk] (u16) of every sorted slot, then per-warp
+  // counters [kWarps][D+1] and the chunk's per-decoder local offsets and global
+  // bases [D+1] each
+  extern __shared__ uint4 srec[];
+  __shared__ uint64_t bar;
+  uint16_t *sidx = reinterpret_cast<uint16_t *>(srec + kBucketChunk);
   uint16_t *sdec = sidx + kBucketChunk;
   uint32_t *cnt = reinterpret_cast<uint32_t *>(sdec + kBucketChunk);
   const uint32_t D1 = A.num_decoders + 1;
   uint32_t *loff = cnt + kWarps * D1;  // chunk-local start of each decoder's run
   uint32_t *gbase = loff + D1;         // global position of that run's first element
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
-  __syncthreads();
   const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
+  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+  for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
+  if (!bulk_load(srec, q + cbase, valid * 16u, &bar)) atomicOr(status, 2u);
   const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
   uint32_t dec[kBucketItems];
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
-    const size_t i = cbase + wbase + (size_t)it * 32 + lane;
-    dec[it] = i < n ? decoder_of(A, __ldg(&q[i].set_id)) : 0xFFFFFFFFu;
+    const uint32_t j = wbase + it * 32 + lane;
+    dec[it] = j < valid ? decoder_of(A, srec[j].x) : 0xFFFFFFFFu;
   }
   uint32_t *my = cnt + warp * D1;
   // rank of each query among the equal decoders of this warp's run, in order
@@ -236,13 +275,12 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
   }
   __syncthreads();
   // coalesced copy-out: consecutive slots of one decoder go to consecutive
-  // positions of that decoder's segment; the record is re-read (L1/L2 hit)
-  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+  // positions of that decoder's segment
   for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
     const uint32_t d = sdec[i], j = sidx[i];
     const uint32_t pos = gbase[d] + (i - loff[d]);
     perm[pos] = (uint32_t)(cbase + j);
-    reinterpret_cast<uint4 *>(sorted)[pos] = __ldg(reinterpret_cast<const uint4 *>(q + cbase + j));
+    reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
   }
 }
 
@@ -271,11 +309,12 @@ size_t bucket_scratch_counts(uint32_t D, size_t n) {
 }
 
 cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
-                          cudaStream_t st, int *launches) {
+                          cudaStream_t st, int *launches, unsigned int *status) {
   const uint32_t chunks = (uint32_t)((n + kBucketChunk - 1) / kBucketChunk);
   const uint32_t D = A.num_decoders;
-  const size_t smem = (size_t)kWarps * (D + 1) * sizeof(uint32_t);
-  const size_t smem_scatter = (size_t)kBucketChunk * (2 + 2) + smem + 2 * (D + 1) * sizeof(uint32_t);
+  const size_t cnt_bytes = (size_t)kWarps * (D + 1) * sizeof(uint32_t);
+  const size_t smem = (size_t)kBucketChunk * 16 + cnt_bytes;
+  const size_t smem_scatter = (size_t)kBucketChunk * (16 + 2 + 2) + cnt_bytes + 2 * (D + 1) * sizeof(uint32_t);
   static bool attr_done = false;
   if (!attr_done) {
     cudaFuncSetAttribute(k_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
@@ -285,9 +324,10 @@ cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const S
   // totals[D+1] and the ticket live after meta
   uint32_t *totals = s.meta + meta_words(D);
   uint32_t *ticket = totals + (D + 1);
-  k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks);
+  k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks, status);
   k_scan<<<D + 1, 1024, 0, st>>>(s.counts, chunks, D, (uint32_t)n, totals, s.meta, ticket);
-  k_scatter<<<chunks, kBucketThreads, smem_scatter, st>>>(A, q, n, s.counts, chunks, s.meta, s.perm, s.sorted);
+  k_scatter<<<chunks, kBucketThreads, smem_scatter, st>>>(A, q, n, s.counts, chunks, s.meta, s.perm, s.sorted,
+                                                          status);
   *launches += 3;
   return cudaGetLastError();
 }

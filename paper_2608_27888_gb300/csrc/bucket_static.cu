@@ -96,7 +96,8 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
   s.sorted = d_sorted;
   s.meta = meta;
   int launches = 0;
-  e = launch_bucket(A, d_queries, n, s, st, &launches);
+  // the last meta word (cleared above) takes the kernels' bounded-wait status
+  e = launch_bucket(A, d_queries, n, s, st, &launches, meta + kMetaWords - 1);
   if (e != cudaSuccess) return failed(NTC_ERR_CUDA, cudaGetErrorString(e));
   return NTC_OK;
 }

@@ -334,7 +334,7 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     }
     return NTC_OK;
   }
-  e = launch_bucket(A, q, n, scratch_of(c), st, &launches);
+  e = launch_bucket(A, q, n, scratch_of(c), st, &launches, c->d_status);
   if (e != cudaSuccess) {
     c->launches += launches;
     return cuda_fail(e, "bucketing launch");
@@ -434,7 +434,7 @@ ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *
   }
   s = ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
-  cudaError_t e = launch_bucket(assets_of(c), q, n, scratch_of(c), st, &launches);
+  cudaError_t e = launch_bucket(assets_of(c), q, n, scratch_of(c), st, &launches, c->d_status);
   if (e == cudaSuccess) e = cudaMemcpyAsync(perm, c->d_perm, n * 4, cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && (counts || tiles || num_tiles))
     e = launch_tiles_export(c->d_meta, c->D, tiles, num_tiles, counts, ntc_max_tiles(c, n), st, &launches);

@@ -220,7 +220,7 @@ constexpr int kBucketItems = 8;  // queries per thread
 constexpr int kBucketChunk = kBucketThreads * kBucketItems;
 
 cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
-                          cudaStream_t st, int *launches);
+                          cudaStream_t st, int *launches, unsigned int *status);
 cudaError_t launch_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,
                                 uint32_t *counts, size_t max_tiles, cudaStream_t st, int *launches);
 cudaError_t launch_decode_fp32(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
