@@ -258,40 +258,75 @@ struct Taps {
   float w[N];
 };
 
-template <bool TRI>
+// One axis of the tap addressing, fp32 round-to-nearest with no contraction
+// (the same operations, in the same order, as the reference addressing).
+// WRAP: c is finite and the texel pair wraps at the edge; clamp: both texels
+// are clamped into [0, n-1].
+template <bool WRAP>
+__device__ __forceinline__ void axis_pair(float c, uint32_t n, uint32_t &i0, uint32_t &i1, float &frac) {
+  const float x = WRAP ? __fsub_rn(__fmul_rn(__fsub_rn(c, floorf(c)), (float)n), 0.5f)
+                       : __fsub_rn(__fmul_rn(c, (float)n), 0.5f);
+  const float x0f = floorf(x);
+  frac = __fsub_rn(x, x0f);
+  if (WRAP) {
+    const int x0 = (int)x0f;  // in [-1, n-1]
+    i0 = x0 < 0 ? n - 1 : (uint32_t)x0;
+    const uint32_t a1 = (uint32_t)(x0 + 1);
+    i1 = a1 == n ? 0u : a1;
+  } else {
+    const int x0 = (int)fminf(fmaxf(x0f, -1.0f), (float)n);
+    i0 = (uint32_t)min(max(x0, 0), (int)n - 1);
+    i1 = (uint32_t)min(x0 + 1, (int)n - 1);
+  }
+}
+
+// Issue the four tap loads of one grid (order 00, 10, 01, 11) and compute
+// their bilinear weights, scaled by sc.  In-grid offsets are 32-bit (a grid
+// holds fewer than 2^32 texels).
+template <bool WRAP>
+__device__ __forceinline__ void grid_fetch(const uint4 *lat, const GridDesc &g, float u, float v, float sc,
+                                           uint4 *raw, float *w) {
+  uint32_t i0, i1, j0, j1;
+  float fx, fy;
+  axis_pair<WRAP>(u, g.W, i0, i1, fx);
+  axis_pair<WRAP>(v, g.H, j0, j1, fy);
+  const uint4 *p = lat + g.base;
+  const uint32_t r0 = j0 * g.W, r1 = j1 * g.W;
+  raw[0] = __ldg(p + (r0 + i0));
+  raw[1] = __ldg(p + (r0 + i1));
+  raw[2] = __ldg(p + (r1 + i0));
+  raw[3] = __ldg(p + (r1 + i1));
+  const float ax = __fsub_rn(1.0f, fx), ay = __fsub_rn(1.0f, fy);
+  w[0] = __fmul_rn(ax, ay) * sc;
+  w[1] = __fmul_rn(fx, ay) * sc;
+  w[2] = __fmul_rn(ax, fy) * sc;
+  w[3] = __fmul_rn(fx, fy) * sc;
+}
+
+// All tap loads of one query, issued before any is consumed.  A row that is
+// not good (padding, bad set id or UV, bad bucket) fetches texel (0, 0) of
+// set 0 instead: no branch and no out-of-range address; its flag marks it.
+template <bool TRI, bool WRAP>
 __device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grids, const ntc_query &q,
                                            bool good, Taps<TRI> &tp) {
-#pragma unroll
-  for (int i = 0; i < Taps<TRI>::N; ++i) {
-    tp.w[i] = 0.0f;
-    tp.raw[i] = make_uint4(0, 0, 0, 0);
-  }
-  if (!good) return;
+  const uint32_t sid = good ? q.set_id : 0u;
+  const float u = good ? q.u : 0.0f, v = good ? q.v : 0.0f;
   float t;
-  const int lo = select_mip(q.lod, A.num_mips, t);
-  const GridDesc *g = grids + (size_t)q.set_id * kLevels * A.num_mips;
+  const int lo = select_mip(good ? q.lod : 0.0f, A.num_mips, t);
+  const GridDesc *g = grids + (size_t)sid * kLevels * A.num_mips;
   const float s = TRI ? __fsub_rn(1.0f, t) : 1.0f;
 #pragma unroll
-  for (int k = 0; k < kLevels; ++k) {
-    unsigned long long idx[4];
-    float w[4];
-    grid_taps(g[k * A.num_mips + lo], q.u, q.v, A.address_mode, idx, w);
+  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.lat, g[k * A.num_mips + lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
+  if (TRI) {
+    if (t > 0.0f) {
 #pragma unroll
-    for (int p = 0; p < 4; ++p) {
-      tp.w[k * 4 + p] = TRI ? w[p] * s : w[p];
-      tp.raw[k * 4 + p] = __ldg(A.lat + idx[p]);
-    }
-  }
-  if (TRI && t > 0.0f) {
+      for (int k = 0; k < kLevels; ++k)
+        grid_fetch<WRAP>(A.lat, g[k * A.num_mips + lo + 1], u, v, t, tp.raw + 8 + 4 * k, tp.w + 8 + 4 * k);
+    } else {
 #pragma unroll
-    for (int k = 0; k < kLevels; ++k) {
-      unsigned long long idx[4];
-      float w[4];
-      grid_taps(g[k * A.num_mips + lo + 1], q.u, q.v, A.address_mode, idx, w);
-#pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        tp.w[8 + k * 4 + p] = w[p] * t;
-        tp.raw[8 + k * 4 + p] = __ldg(A.lat + idx[p]);
+      for (int i = 8; i < Taps<TRI>::N; ++i) {
+        tp.w[i] = 0.0f;
+        tp.raw[i] = make_uint4(0, 0, 0, 0);
       }
     }
   }
@@ -361,6 +396,19 @@ __device__ __forceinline__ void tile_lookup(const uint32_t *seg, const uint32_t 
   len = min((uint32_t)kTile, seg[lo + 1] - start);
 }
 
+// The tiles of one role in increasing order: the decoder index only moves
+// forward, so a lookup is a few compares instead of a binary search.
+struct TileWalk {
+  uint32_t d = 0;
+  __device__ __forceinline__ void at(const uint32_t *seg, const uint32_t *tst, uint32_t D, uint32_t t,
+                                     uint32_t &dec, uint32_t &start, uint32_t &len) {
+    while (d < D && tst[d + 1] <= t) ++d;
+    dec = d;
+    start = seg[d] + (t - tst[d]) * kTile;
+    len = min((uint32_t)kTile, seg[d + 1] - start);
+  }
+};
+
 // Per-thread view of one tile row.
 struct Row {
   uint32_t dec, start, len;  // the tile
@@ -402,7 +450,8 @@ struct TmSmem {
   static constexpr int S = NC * SC;                                     // stages in all rings
   static constexpr size_t weights = 0;                                  // per consumer
   static constexpr size_t flags = weights + (size_t)NC * L::WIMG;       // per stage: 128 row flags
-  static constexpr size_t bars = flags + (size_t)S * 128;
+  static constexpr size_t oidx = flags + (size_t)S * 128;               // per stage: 128 output rows
+  static constexpr size_t bars = oidx + (size_t)S * 128 * 4;
   static constexpr int nbars = 2 * S + 2 * NC;                          // full, empty, mma, weights
   static constexpr size_t misc = bars + (size_t)nbars * 8;
   static constexpr size_t tiles = misc + 64;
@@ -410,21 +459,25 @@ struct TmSmem {
   static constexpr size_t total = grids + kSmemGrids * sizeof(GridDesc);
 };
 
-// Tensor-memory plan (columns).  Consumer c owns CS columns from c*CS: the fp32
-// accumulator at +0 (H columns), its hidden A operand at +H (KH/2 columns, two
-// 16-bit K elements per column) and the layer-1 A operands [128 x 32] of its SC
-// ring stages at +AOFF + 16 st (16 columns each).  Accumulators stay 32-column
-// aligned and every A operand 16-column aligned.
+// Tensor-memory plan (columns).  The NC fp32 accumulators (H columns each)
+// come first, so every accumulator starts on a multiple of H; then each
+// consumer's hidden A operand (H/2 columns: two 16-bit K elements per column);
+// then the layer-1 feature operands [128 x 16] of the NC * SC ring stages (8
+// columns each); last, one shared 8-column block holding a 1 in K column 0 and
+// zeros elsewhere: the A operand of every layer's bias K step (the decoder image
+// keeps each layer's bias as the first row of an extra 16-row K block).
 template <int H, int NC, int SC>
 struct TmCols {
-  static constexpr uint32_t KH = H + 16;
-  static constexpr uint32_t AOFF = (H + KH / 2 + 15) / 16 * 16;
-  static constexpr uint32_t CS = (AOFF + 16 * SC + 31) / 32 * 32;
-  static constexpr uint32_t used = NC * CS;
+  static constexpr uint32_t HID = NC * H;
+  static constexpr uint32_t STG = HID + NC * (H / 2);
+  static constexpr uint32_t ONES = STG + NC * SC * 8;
+  static constexpr uint32_t used = ONES + 8;
   static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
   static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
+  static __device__ __forceinline__ uint32_t acc(uint32_t c) { return c * H; }
+  static __device__ __forceinline__ uint32_t hid(uint32_t c) { return HID + c * (H / 2); }
   // layer-1 A operand of stage s (= consumer * SC + st)
-  static __device__ __forceinline__ uint32_t a1(uint32_t s) { return (s / SC) * CS + AOFF + 16 * (s % SC); }
+  static __device__ __forceinline__ uint32_t a1(uint32_t s) { return STG + 8 * s; }
 };
 
 // Warp-specialised gather-decode with tensor-memory operands.
@@ -446,7 +499,7 @@ struct TmCols {
 //   registers -> TMEM; layers 2 and 3 read their A from TMEM too; the sigmoid
 //   epilogue scatters rows to out[perm[i]] while the next tile's layer 1 runs.
 // CTA b owns the global tiles b, b + grid, b + 2 grid, ...
-template <int H, bool BF16, bool TRI, int CP, int NP, int NC, int SC>
+template <int H, bool BF16, bool TRI, bool WRAP, int CP, int NP, int NC, int SC>
 __global__ void __launch_bounds__((NP + NC) * 128, 1)
     k_decode_tm(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
                 unsigned int *status, int vec_out) {
@@ -469,6 +522,10 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   volatile uint32_t *stop_flag = tmem_slot + 2;  // [NC], each read only after its warpgroup's barrier
   const uint32_t D = A.num_decoders, C = W.out_dim;
 
+  // no stage has rows yet: a consumer that stops on a wait timeout reads
+  // all-bad flags, never an uninitialised output index
+  for (uint32_t i = threadIdx.x; i < (uint32_t)S * 128 / 4; i += blockDim.x)
+    reinterpret_cast<uint32_t *>(smem + M::flags)[i] = 0u;
   const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
   if (D + 2 <= kSmemTileTable) {
     uint32_t *s_seg = reinterpret_cast<uint32_t *>(smem + M::tiles);
@@ -509,6 +566,14 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const uint32_t one = BF16 ? 0x3F80u : 0x3C00u;  // 1.0 in the low half, 0 in the high half
+  if (warp < 4) {  // the shared bias operand: K column 0 is 1, the rest 0
+    const uint32_t z[8] = {one, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+    tmem_st8(tmem_base + TC::ONES + lanes, z);
+    tmem_wait_st();
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
   const uint32_t T = __ldg(B.meta);
   const uint32_t grid = gridDim.x;
   const uint32_t K = blockIdx.x < T ? (T - blockIdx.x + grid - 1) / grid : 0;  // local tiles
@@ -518,70 +583,70 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t pc = role % NC, pq = role / NC;  // serves consumer pc, tiles j = pq mod R
     auto tile_of = [&](uint32_t j) { return pc + NC * j; };
     uint32_t j = pq;
-    uint32_t dec = D, start = 0, len = 0;
+    uint32_t dec = D, start = 0, len = 0, oi = 0;
     ntc_query q;
+    TileWalk walk;
     if (tile_of(j) < K) {
-      tile_lookup(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
-      if ((uint32_t)row < len) q = load_query(B.sorted + start + row);
+      walk.at(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
+      if ((uint32_t)row < len) {
+        q = load_query(B.sorted + start + row);
+        oi = __ldg(B.perm + start + row);
+      }
     }
     for (; tile_of(j) < K; j += R) {
       if (*abort_flag) break;
-      // the next tile's query record goes in flight first
-      uint32_t ndec = D, nstart = 0, nlen = 0;
+      // the next tile's query record and output row go in flight first
+      uint32_t ndec = D, nstart = 0, nlen = 0, noi = 0;
       ntc_query nq;
       if (tile_of(j + R) < K) {
-        tile_lookup(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
-        if ((uint32_t)row < nlen) nq = load_query(B.sorted + nstart + row);
+        walk.at(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
+        if ((uint32_t)row < nlen) {
+          nq = load_query(B.sorted + nstart + row);
+          noi = __ldg(B.perm + nstart + row);
+        }
       }
       const bool valid = (uint32_t)row < len;
       const bool good = valid && dec < D && !query_bad(A, q);
       Taps<TRI> taps;
-      issue_taps<TRI>(A, grids, q, good, taps);
+      issue_taps<TRI, WRAP>(A, grids, q, good, taps);
       // bad rows (set id out of range, non-finite UV, or the bad bucket) decode to NaN
       const bool bad = valid && !good;
       const uint32_t badm = __ballot_sync(0xFFFFFFFFu, bad);
       if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
-      if (bad) {
-        const uint32_t oi = __ldg(B.perm + start + row);
+      if (bad)
         for (uint32_t cc = 0; cc < C; ++cc) out[(size_t)oi * C + cc] = __int_as_float(0x7fc00000);
-      }
-      uint32_t a[16];
-      {
-        uint32_t pk[8];
-        taps_to_row<TRI, BF16>(taps, pk);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) a[i] = pk[i];
-      }
-      a[8] = one;
-#pragma unroll
-      for (int i = 9; i < 16; ++i) a[i] = 0u;
+      uint32_t a[8];
+      taps_to_row<TRI, BF16>(taps, a);
       const uint32_t s = pc * SC + j % SC, n = j / SC;
       if (!mbar_wait(empty_bar(s), (n & 1) ^ 1)) {  // the stage's previous tile has left layer 1
         atomicOr(status, 1u);
         *abort_flag = 1;
       }
       fence_after();
-      tmem_st16(tmem_base + TC::a1(s) + lanes, a);
+      tmem_st8(tmem_base + TC::a1(s) + lanes, a);
       tmem_wait_st();
       smem[M::flags + s * 128 + row] = good ? 1 : 0;
+      reinterpret_cast<uint32_t *>(smem + M::oidx)[s * 128 + row] = oi;
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(full_bar(s));
       dec = ndec;
-      start = nstart;
       len = nlen;
       q = nq;
+      oi = noi;
     }
   } else {
     // ------------------------------------------------------------ consumer
     const int c = role - NP;
     const int wgid = role;  // named barrier id role + 1
-    const bool poller = (row >> 5) == 0;
-    const uint32_t tD = tmem_base + c * TC::CS;  // accumulator
-    const uint32_t tH = tD + H;                  // hidden A operand
+    const bool poller = (row >> 5) == (c & 3);  // pollers spread over the sub-partitions
+    const uint32_t tD = tmem_base + TC::acc(c);  // accumulator
+    const uint32_t tH = tmem_base + TC::hid(c);  // hidden A operand
+    const uint32_t tOnes = tmem_base + TC::ONES; // the bias K step's A operand
     const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
     const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
     uint32_t ph = 0, wph = 0, cur = 0xFFFFFFFFu;
+    TileWalk cwalk;
     constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
     const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
     auto wait_bar = [&](uint32_t b, uint32_t parity) {
@@ -590,12 +655,6 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         *abort_flag = 1;
       }
     };
-    // the hidden A operand's bias column (k = H) and zero padding never change
-    {
-      uint32_t z[8] = {one, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-      tmem_st8(tH + H / 2 + lanes, z);
-      tmem_wait_st();
-    }
     // TMEM accumulator -> ReLU -> fp16/bf16 pairs -> hidden A operand
     auto hidden = [&]() {
 #pragma unroll 1
@@ -610,14 +669,13 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       }
       tmem_wait_st();
     };
-    // Start tile k: its output rows, its decoder's weights, wait for its A
-    // stage and issue layer 1.  Requires this consumer's previous tile to have
-    // finished all MMAs.
+    // Start tile k: its decoder's weights, wait for its A stage (with the
+    // rows' flags and output indices) and issue layer 1.  Requires this
+    // consumer's previous tile to have finished all MMAs.
     auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good) {
       const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
       uint32_t start, len;
-      tile_lookup(seg, tst, D, t, dec, start, len);
-      oi = (uint32_t)row < len ? __ldg(B.perm + start + row) : 0u;
+      cwalk.at(seg, tst, D, t, dec, start, len);
       bool wpend = false;
       if (dec < D && dec != cur) {
         if (row == 0) bulk_g2s(sW1, W.tc + (size_t)dec * W.tc_stride, L::WIMG, wbar);
@@ -631,12 +689,13 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       }
       wg_bar(wgid);
       good = smem[M::flags + s * 128 + row] != 0;
+      oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[s * 128 + row];
       if (row == 0) {
         fence_after();
         if (dec < D) {
           const uint32_t tA = tmem_base + TC::a1(s);
-#pragma unroll
-          for (uint32_t kq = 0; kq < kTcKA / 16; ++kq) umma_ta(tD, tA + 8 * kq, dW1 + 16 * kq, id_hidden, kq);
+          umma_ta(tD, tA, dW1, id_hidden, 0);
+          umma_ta(tD, tOnes, dW1 + 16, id_hidden, 1);  // + bias
           umma_commit(mbar);
           umma_commit(empty_bar(s));
         } else {
@@ -664,7 +723,8 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
             const uint64_t dW = layer == 0 ? dW2 : dW3;
             const uint32_t id = layer == 0 ? id_hidden : id_out;
 #pragma unroll
-            for (uint32_t kq = 0; kq < L::KH / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW + 16 * kq, id, kq);
+            for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW + 16 * kq, id, kq);
+            umma_ta(tD, tOnes, dW + 16 * (H / 16), id, 1);  // + bias
             umma_commit(mbar);
           }
         }
@@ -719,7 +779,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   }
 }
 
-template <int H, bool BF16, bool TRI, int NP, int NC, int SC>
+template <int H, bool BF16, bool TRI, bool WRAP, int NP, int NC, int SC>
 cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, float *out,
                         unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
   using M = TmSmem<H, NC, SC>;
@@ -731,16 +791,16 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
     const int carve = (int)((smem * 100 + 232448 - 1) / 232448);
     cudaError_t e;
     if (c8) {
-      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, SC>,
+      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 8, NP, NC, SC>,
+        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC>,
                                  cudaFuncAttributePreferredSharedMemoryCarveout, carve);
     } else {
-      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, SC>,
+      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, 16, NP, NC, SC>,
+        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC>,
                                  cudaFuncAttributePreferredSharedMemoryCarveout, carve);
     }
     if (e != cudaSuccess) return e;
@@ -752,9 +812,9 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   const int vec_out = ((uintptr_t)out & 15) == 0;
   const unsigned threads = (NP + NC) * 128;
   if (c8)
-    k_decode_tm<H, BF16, TRI, 8, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+    k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
   else
-    k_decode_tm<H, BF16, TRI, 16, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+    k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
   return cudaGetLastError();
 }
 
@@ -803,10 +863,15 @@ cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Bucke
                              float *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches) {
   *launches += 1;
-  const bool tri = A.num_mips > 1;
-#define NTC_WS(H, TRI, NP, NC, SC)                                                                \
-  return bf16 ? launch_tm_t<H, true, TRI, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st) \
-              : launch_tm_t<H, false, TRI, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st)
+  const bool tri = A.num_mips > 1, wrap = A.address_mode == 0;
+#define NTC_WS2(H, TRI, WRAP, NP, NC, SC)                                                                  \
+  return bf16 ? launch_tm_t<H, true, TRI, WRAP, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st) \
+              : launch_tm_t<H, false, TRI, WRAP, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st)
+#define NTC_WS(H, TRI, NP, NC, SC)              \
+  do {                                          \
+    if (wrap) NTC_WS2(H, TRI, true, NP, NC, SC); \
+    NTC_WS2(H, TRI, false, NP, NC, SC);          \
+  } while (0)
   if (W.hidden == 64) {
     if (tri) NTC_WS(64, true, 2, 2, 2);
     NTC_WS(64, false, 4, 4, 1);
@@ -814,6 +879,7 @@ cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Bucke
   if (tri) NTC_WS(128, true, 2, 2, 2);
   NTC_WS(128, false, 2, 2, 2);
 #undef NTC_WS
+#undef NTC_WS2
 }
 
 }  // namespace ntc
