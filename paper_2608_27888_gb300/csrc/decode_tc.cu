@@ -280,27 +280,42 @@ __device__ __forceinline__ void axis_pair(float c, uint32_t n, uint32_t &i0, uin
   }
 }
 
-// Issue the four tap loads of one grid (order 00, 10, 01, 11) and compute
-// their bilinear weights, scaled by sc.  In-grid offsets are 32-bit (a grid
-// holds fewer than 2^32 texels).
+// Both texels of one bilinear row from the row-pair copy: one 32-byte load.
+struct alignas(32) TexelPair {
+  uint4 a, b;
+};
+__device__ __forceinline__ void ld_pair(const TexelPair *p, uint4 &a, uint4 &b) {
+  asm volatile("ld.global.nc.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+               : "l"(p));
+}
+
+// Issue the tap loads of one grid (taps 00, 10 from row j0; 01, 11 from row
+// j1) and compute their bilinear weights, scaled by sc.  In-grid offsets are
+// 32-bit (a grid holds fewer than 2^32 texels).  Clamp mode at an edge has
+// x0 = x1, while the pair at x0 holds x0 and its right neighbour: the whole
+// row weight then goes to the first texel.
 template <bool WRAP>
-__device__ __forceinline__ void grid_fetch(const uint4 *lat, const GridDesc &g, float u, float v, float sc,
+__device__ __forceinline__ void grid_fetch(const uint4 *pair, const GridDesc &g, float u, float v, float sc,
                                            uint4 *raw, float *w) {
   uint32_t i0, i1, j0, j1;
   float fx, fy;
   axis_pair<WRAP>(u, g.W, i0, i1, fx);
   axis_pair<WRAP>(v, g.H, j0, j1, fy);
-  const uint4 *p = lat + g.base;
-  const uint32_t r0 = j0 * g.W, r1 = j1 * g.W;
-  raw[0] = __ldg(p + (r0 + i0));
-  raw[1] = __ldg(p + (r0 + i1));
-  raw[2] = __ldg(p + (r1 + i0));
-  raw[3] = __ldg(p + (r1 + i1));
+  const TexelPair *p = reinterpret_cast<const TexelPair *>(pair) + g.base;
+  ld_pair(p + (j0 * g.W + i0), raw[0], raw[1]);
+  ld_pair(p + (j1 * g.W + i0), raw[2], raw[3]);
   const float ax = __fsub_rn(1.0f, fx), ay = __fsub_rn(1.0f, fy);
-  w[0] = __fmul_rn(ax, ay) * sc;
-  w[1] = __fmul_rn(fx, ay) * sc;
-  w[2] = __fmul_rn(ax, fy) * sc;
-  w[3] = __fmul_rn(fx, fy) * sc;
+  float w00 = __fmul_rn(ax, ay), w10 = __fmul_rn(fx, ay), w01 = __fmul_rn(ax, fy), w11 = __fmul_rn(fx, fy);
+  if (!WRAP && i1 == i0) {
+    w00 = __fadd_rn(w00, w10);
+    w01 = __fadd_rn(w01, w11);
+    w10 = w11 = 0.0f;
+  }
+  w[0] = w00 * sc;
+  w[1] = w10 * sc;
+  w[2] = w01 * sc;
+  w[3] = w11 * sc;
 }
 
 // All tap loads of one query, issued before any is consumed.  A row that is
@@ -316,12 +331,12 @@ __device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grid
   const GridDesc *g = grids + (size_t)sid * kLevels * A.num_mips;
   const float s = TRI ? __fsub_rn(1.0f, t) : 1.0f;
 #pragma unroll
-  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.lat, g[k * A.num_mips + lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
+  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.pair, g[k * A.num_mips + lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
   if (TRI) {
     if (t > 0.0f) {
 #pragma unroll
       for (int k = 0; k < kLevels; ++k)
-        grid_fetch<WRAP>(A.lat, g[k * A.num_mips + lo + 1], u, v, t, tp.raw + 8 + 4 * k, tp.w + 8 + 4 * k);
+        grid_fetch<WRAP>(A.pair, g[k * A.num_mips + lo + 1], u, v, t, tp.raw + 8 + 4 * k, tp.w + 8 + 4 * k);
     } else {
 #pragma unroll
       for (int i = 8; i < Taps<TRI>::N; ++i) {
@@ -537,11 +552,11 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     seg = s_seg;
     tst = s_tst;
   }
-  const GridDesc *grids = A.grids;
+  const GridDesc *grids = A.pgrids;  // grid bases in the row-pair copy
   const uint32_t ngrids = A.num_sets * kLevels * A.num_mips;
   if (ngrids <= kSmemGrids) {
     GridDesc *s_grids = reinterpret_cast<GridDesc *>(smem + M::grids);
-    for (uint32_t i = threadIdx.x; i < ngrids; i += blockDim.x) s_grids[i] = A.grids[i];
+    for (uint32_t i = threadIdx.x; i < ngrids; i += blockDim.x) s_grids[i] = A.pgrids[i];
     grids = s_grids;
   }
   if (threadIdx.x == 0) {

@@ -19,6 +19,8 @@ struct ntc_ctx {
   uint64_t num_texels = 0;
   uint4 *d_lat = nullptr;
   GridDesc *d_grids = nullptr;
+  uint4 *d_pair = nullptr;      // row-pair copy of the latents, 32 B per texel
+  GridDesc *d_pgrids = nullptr;  // grid bases in d_pair
   uint32_t *d_map = nullptr;
   uint8_t *d_mma = nullptr;
   float *d_f32 = nullptr;
@@ -87,6 +89,8 @@ Assets assets_of(const ntc_ctx *c) {
   Assets A;
   A.lat = c->d_lat;
   A.grids = c->d_grids;
+  A.pair = c->d_pair;
+  A.pgrids = c->d_pgrids;
   A.map = c->d_map;
   A.num_sets = c->S;
   A.num_decoders = c->D;
@@ -113,6 +117,8 @@ void release(ntc_ctx *c) {
     if (e) cudaEventDestroy(e);
   cudaFree(c->d_lat);
   cudaFree(c->d_grids);
+  cudaFree(c->d_pair);
+  cudaFree(c->d_pgrids);
   cudaFree(c->d_map);
   cudaFree(c->d_mma);
   cudaFree(c->d_f32);
@@ -255,6 +261,21 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   c->mma_stride = round16(mma_image_bytes(c->H));
   c->f32_stride = (f32_image_floats(c->H, c->C) + 3) & ~(size_t)3;
   c->tc_stride = round16(tc_image_bytes(c->H));
+  // the row-pair copy: grids back to back, built in chunks of kPairChunk texels
+  std::vector<GridDesc> pgrids(grids.size());
+  std::vector<uint32_t> chunk_grid, chunk_start;
+  uint64_t num_pairs = 0;
+  for (size_t g = 0; g < grids.size(); ++g) {
+    pgrids[g] = grids[g];
+    pgrids[g].base = num_pairs;
+    const uint64_t nt = (uint64_t)grids[g].W * grids[g].H;
+    num_pairs += nt;
+    for (uint64_t t = 0; t < nt; t += kPairChunk) {
+      chunk_grid.push_back((uint32_t)g);
+      chunk_start.push_back((uint32_t)t);
+    }
+  }
+  uint32_t *d_chunks = nullptr;
   float *d_w32 = nullptr;
   cudaError_t e = cudaSuccess;
   auto step = [&](cudaError_t r) {
@@ -269,11 +290,20 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   step(cudaMalloc((void **)&c->d_err, sizeof(unsigned long long)));
   step(cudaMalloc((void **)&c->d_status, sizeof(unsigned int)));
   step(cudaMalloc((void **)&d_w32, P * 4 * c->D));
+  step(cudaMalloc((void **)&c->d_pair, num_pairs * 32));
+  step(cudaMalloc((void **)&c->d_pgrids, pgrids.size() * sizeof(GridDesc)));
+  step(cudaMalloc((void **)&d_chunks, chunk_grid.size() * 2 * sizeof(uint32_t)));
   if (e == cudaSuccess) {
     step(cudaMemcpy(c->d_lat, d->latents, d->num_texels * 16, cudaMemcpyHostToDevice));
     step(cudaMemcpy(c->d_grids, grids.data(), grids.size() * sizeof(GridDesc), cudaMemcpyHostToDevice));
     step(cudaMemcpy(c->d_map, d->set_to_decoder, (size_t)S * 4, cudaMemcpyHostToDevice));
     step(cudaMemcpy(d_w32, d->weights, P * 4 * c->D, cudaMemcpyHostToDevice));
+    step(cudaMemcpy(c->d_pgrids, pgrids.data(), pgrids.size() * sizeof(GridDesc), cudaMemcpyHostToDevice));
+    step(cudaMemcpy(d_chunks, chunk_grid.data(), chunk_grid.size() * sizeof(uint32_t), cudaMemcpyHostToDevice));
+    step(cudaMemcpy(d_chunks + chunk_grid.size(), chunk_start.data(), chunk_start.size() * sizeof(uint32_t),
+                    cudaMemcpyHostToDevice));
+    step(launch_build_pairs(assets_of(c), d_chunks, d_chunks + chunk_grid.size(), (uint32_t)chunk_grid.size(),
+                            c->d_pair, 0));
     step(cudaMemset(c->d_err, 0, sizeof(unsigned long long)));
     step(cudaMemset(c->d_status, 0, sizeof(unsigned int)));
     step(cudaMemset(c->d_tc, 0, c->tc_stride * c->D));
@@ -282,6 +312,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
     step(cudaDeviceSynchronize());
   }
   cudaFree(d_w32);
+  cudaFree(d_chunks);
   if (e != cudaSuccess) {
     release(c);
     delete c;

@@ -27,6 +27,12 @@ struct alignas(16) GridDesc {
 struct Assets {
   const uint4 *lat;         // latents, one uint4 (8 x fp16) per texel
   const GridDesc *grids;    // [num_sets][kLevels][num_mips]
+  // Row-pair copy of the latents: texel (x, y) of a grid holds its own 8
+  // channels and those of its right neighbour (x + 1 wrapped or clamped by the
+  // address mode), 32 bytes, so one aligned load fetches both texels of a
+  // bilinear row.  pgrids give each grid's base in `pair` (units of 32 bytes).
+  const uint4 *pair;
+  const GridDesc *pgrids;
   const uint32_t *map;      // [num_sets] set -> decoder
   uint32_t num_sets, num_decoders, num_mips, address_mode;
 };
@@ -241,6 +247,9 @@ cudaError_t launch_debug_taps(const Assets &A, const ntc_query *q, size_t n, uns
                               float *w, float *t, cudaStream_t st, int *launches);
 cudaError_t launch_debug_features(const Assets &A, const ntc_query *q, size_t n, float *f,
                                   cudaStream_t st, int *launches);
+cudaError_t launch_build_pairs(const Assets &A, const uint32_t *chunk_grid, const uint32_t *chunk_start,
+                               uint32_t num_chunks, uint4 *pair, cudaStream_t st);
+constexpr uint32_t kPairChunk = 65536;  // texels per work item of launch_build_pairs
 cudaError_t launch_pack_weights(const float *w32, uint32_t D, uint32_t H, uint32_t C, bool bf16,
                                 uint8_t *mma, size_t mma_stride, float *f32, size_t f32_stride,
                                 uint8_t *tc, size_t tc_stride, cudaStream_t st);

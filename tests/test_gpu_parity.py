@@ -133,6 +133,29 @@ def test_taps_tiny_grids_bit_exact(mode, dims):
     dec.close()
 
 
+@pytest.mark.parametrize("mips", [1, 3])
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("dims", [(1, 1), (2, 2), (3, 5), (7, 3), (16, 8)])
+def test_decode_tc_tiny_grids_edges(mode, dims, mips):
+    """The tensor-core path reads each bilinear row as a texel pair: wrap and
+    clamp edges, 1-texel grids and mip blends must still match the oracle."""
+    W0, H0 = dims
+    dims2 = [[(W0, H0), (max(1, W0 // 2), max(1, H0 // 2))]]
+    shape = tiny_assets(dims2, num_mips=mips, hidden=64, out_dim=8)
+    rng = np.random.default_rng(W0 * 31 + H0 * 7 + mips)
+    a = tiny_assets(dims2, num_mips=mips, address_mode=mode, hidden=64, out_dim=8,
+                    latents=rng.normal(0.0, 1.0, shape.latents.size),
+                    weights=rng.uniform(-0.4, 0.4, shape.weights.shape))
+    grid = np.arange(-40, 41) / 16.0
+    rows = [(0, float(u), float(v), float(l)) for u in grid for v in grid[::2] for l in (0.0, 0.75, 2.0)]
+    q = queries(rows)
+    ref, _ = oracle.decode(a, q)
+    for prec in ("fp16", "bf16"):
+        dec = ntc().Decoder(a, prec)
+        check_tc(dec.decode(dq(q)).cpu().numpy(), ref, f"{dims} mode {mode} mips {mips} {prec}")
+        dec.close()
+
+
 @pytest.mark.parametrize("k,variant", [(2, None), (5, None)])
 def test_features_match_oracle(k, variant):
     w = small(k, variant)
