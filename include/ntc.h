@@ -141,8 +141,13 @@ NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n
                       void *cuda_stream, ntc_mode mode);
 
 /* ntc_decode on HOST buffers: copies the queries to context-owned device
- * memory, decodes, copies the outputs back into h_out and synchronises the
- * stream before returning.  Pinned host memory makes the copies faster. */
+ * memory, decodes, copies the outputs back into h_out and synchronises before
+ * returning.  The batch is split into up to 8 chunks (at least 2^18 queries
+ * each) whose upload, decode and download overlap: uploads and downloads run
+ * on two context-owned streams ordered after the work already queued on
+ * `cuda_stream`, decodes on `cuda_stream`.  Each chunk is bucketed on its own;
+ * outputs are the same as one ntc_decode over all n.  Pinned host memory is
+ * needed for the copies to overlap. */
 NTC_API ntc_status ntc_decode_host(ntc_ctx *ctx, const ntc_query *h_queries, size_t n, float *h_out,
                            void *cuda_stream, ntc_mode mode);
 

@@ -11,6 +11,11 @@
 
 using namespace ntc;
 
+// ntc_decode_host splits a batch into at most kHostChunks pipelined chunks of
+// at least kHostChunkMin queries.
+constexpr int kHostChunks = 8, kHostChunksMax = kHostChunks;
+constexpr size_t kHostChunkMin = 1u << 18;
+
 struct ntc_ctx {
   int device = 0;
   int num_sms = 0;
@@ -32,10 +37,12 @@ struct ntc_ctx {
   size_t cap_n = 0, cap_counts = 0;
   uint32_t *d_counts = nullptr, *d_perm = nullptr, *d_meta = nullptr;
   ntc_query *d_sorted = nullptr;
-  // staging for ntc_decode_host
+  // staging for ntc_decode_host, and its copy streams and chunk events
   size_t cap_host = 0;
   ntc_query *d_hq = nullptr;
   float *d_hout = nullptr;
+  cudaStream_t s_up = nullptr, s_down = nullptr;
+  cudaEvent_t ev_begin = nullptr, ev_up[kHostChunksMax] = {}, ev_done[kHostChunksMax] = {};
   uint64_t launches = 0;
   // optional stage timing
   bool timing = false;
@@ -115,6 +122,13 @@ WeightImages weights_of(const ntc_ctx *c) {
 void release(ntc_ctx *c) {
   for (auto &e : c->ev)
     if (e) cudaEventDestroy(e);
+  for (int i = 0; i < kHostChunksMax; ++i) {
+    if (c->ev_up[i]) cudaEventDestroy(c->ev_up[i]);
+    if (c->ev_done[i]) cudaEventDestroy(c->ev_done[i]);
+  }
+  if (c->ev_begin) cudaEventDestroy(c->ev_begin);
+  if (c->s_up) cudaStreamDestroy(c->s_up);
+  if (c->s_down) cudaStreamDestroy(c->s_down);
   cudaFree(c->d_lat);
   cudaFree(c->d_grids);
   cudaFree(c->d_pair);
@@ -400,6 +414,8 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hou
   cudaStream_t st = (cudaStream_t)stream;
   if (n > c->cap_host) {
     CK(cudaStreamSynchronize(st), "staging resize");
+    if (c->s_up) CK(cudaStreamSynchronize(c->s_up), "staging resize");
+    if (c->s_down) CK(cudaStreamSynchronize(c->s_down), "staging resize");
     cudaFree(c->d_hq);
     cudaFree(c->d_hout);
     c->d_hq = nullptr;
@@ -409,10 +425,46 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hou
     CK(cudaMalloc((void **)&c->d_hout, n * c->C * sizeof(float)), "staging allocation");
     c->cap_host = n;
   }
-  CK(cudaMemcpyAsync(c->d_hq, hq, n * sizeof(ntc_query), cudaMemcpyHostToDevice, st), "query upload");
-  s = ntc_decode(c, c->d_hq, n, c->d_hout, stream, mode);
-  if (s != NTC_OK) return s;
-  CK(cudaMemcpyAsync(hout, c->d_hout, n * c->C * sizeof(float), cudaMemcpyDeviceToHost, st), "output download");
+  if (!c->s_up) {
+    CK(cudaStreamCreateWithFlags(&c->s_up, cudaStreamNonBlocking), "copy stream");
+    CK(cudaStreamCreateWithFlags(&c->s_down, cudaStreamNonBlocking), "copy stream");
+    CK(cudaEventCreateWithFlags(&c->ev_begin, cudaEventDisableTiming), "chunk event");
+    for (int i = 0; i < kHostChunksMax; ++i) {
+      CK(cudaEventCreateWithFlags(&c->ev_up[i], cudaEventDisableTiming), "chunk event");
+      CK(cudaEventCreateWithFlags(&c->ev_done[i], cudaEventDisableTiming), "chunk event");
+    }
+  }
+  // Chunks pipeline the upload (s_up), the decode (the caller's stream) and the
+  // download (s_down): chunk i+1 uploads and chunk i-1 downloads while chunk i
+  // decodes.  Each chunk is bucketed on its own; every query's output is the
+  // same as in one call over all n.
+  size_t chunk = (n + kHostChunks - 1) / kHostChunks;
+  if (chunk < kHostChunkMin) chunk = kHostChunkMin;
+  chunk = (chunk + kBucketChunk - 1) / kBucketChunk * kBucketChunk;
+  const size_t nchunks = (n + chunk - 1) / chunk;
+  const size_t C = c->C;
+  CK(cudaEventRecord(c->ev_begin, st), "chunk event");
+  CK(cudaStreamWaitEvent(c->s_up, c->ev_begin, 0), "stream order");
+  CK(cudaStreamWaitEvent(c->s_down, c->ev_begin, 0), "stream order");
+  for (size_t i = 0; i < nchunks; ++i) {
+    const size_t off = i * chunk, m = n - off < chunk ? n - off : chunk;
+    CK(cudaMemcpyAsync(c->d_hq + off, hq + off, m * sizeof(ntc_query), cudaMemcpyHostToDevice, c->s_up),
+       "query upload");
+    CK(cudaEventRecord(c->ev_up[i], c->s_up), "chunk event");
+    CK(cudaStreamWaitEvent(st, c->ev_up[i], 0), "stream order");
+    s = ntc_decode(c, c->d_hq + off, m, c->d_hout + off * C, stream, mode);
+    if (s != NTC_OK) {
+      cudaStreamSynchronize(c->s_up);
+      cudaStreamSynchronize(c->s_down);
+      return s;
+    }
+    CK(cudaEventRecord(c->ev_done[i], st), "chunk event");
+    CK(cudaStreamWaitEvent(c->s_down, c->ev_done[i], 0), "stream order");
+    CK(cudaMemcpyAsync(hout + off * C, c->d_hout + off * C, m * C * sizeof(float), cudaMemcpyDeviceToHost,
+                       c->s_down),
+       "output download");
+  }
+  CK(cudaStreamSynchronize(c->s_down), "decode");
   CK(cudaStreamSynchronize(st), "decode");
   return NTC_OK;
 }
