@@ -1,32 +1,34 @@
-// tcgen05 / TMEM gather-decode (sm_103a).
+// tcgen05 / TMEM gather-decode (sm_103a), warp-specialised.
 //
-// One persistent CTA per SM holds NWG warpgroups; each warpgroup decodes its own
-// single-decoder 128-query tiles (tiles are dealt out round-robin over all
-// warpgroups of the grid, so at any moment the whole GPU works on neighbouring
-// tiles -- the same decoder and, for a set-major bucket order, the same
-// latents, which keeps them in L2).  Per tile:
-//   1. each thread gathers its query's latent taps, blends them in fp32 and
-//      writes one fp16/bf16 row of the A tile [128 x 32] (16 features, a 1 in
-//      column 16 that multiplies the bias row of the weights, zeros) into
-//      shared memory;
-//   2. one thread issues the layer-1 tcgen05.mma (M=128, N=H, K=32) into the
-//      warpgroup's TMEM columns and commits to an mbarrier;
-//   3. the four warps read their 32 TMEM lanes (tcgen05.ld), apply ReLU while
-//      converting to fp16/bf16, and write the hidden tile [128 x (H+16)] (with
-//      its own ones column) to shared memory; layer 2 (N=H) and layer 3 (N=16)
-//      follow the same way; the last epilogue applies the sigmoid and scatters
-//      the rows to out[perm[i]].
-// Shared-memory operands use the no-swizzle K-major canonical layout: 8-row x
-// 16-byte core matrices, K-adjacent core matrices 128 B apart (LBO), 8-row
-// groups K*16 B apart (SBO).  The decoder's weights (bias folded in as an extra
-// K column) are copied from a pre-packed image whenever a warpgroup's tile
-// changes decoder.  Every mbarrier wait is bounded by time; on expiry the
+// One persistent CTA per SM runs NP producer and NC consumer warpgroups.
+// Tiles (128 queries of one decoder, from the bucketing) are dealt out
+// round-robin over the CTAs, so at any moment the whole GPU works on
+// neighbouring tiles -- one decoder and, in set-major bucket order, one set's
+// latents, which keeps them in L2.  Inside a CTA, consumer c takes the CTA's
+// tiles c, c + NC, ... and is fed by its own producers through a private ring
+// of SC tensor-memory stages.
+//   Producer (one thread per tile row): loads the query record and its output
+//     row index, computes the bilinear taps of both latent grids (Sec. 3.1, the
+//     same fp32 operations as the reference addressing), fetches each bilinear
+//     row as one 32-byte load from the row-pair copy of the latents, blends in
+//     fp32 and stores the fp16/bf16 feature row [16] into its stage with
+//     tcgen05.st (warp q writes TMEM lanes 32q..32q+31, exactly its rows).
+//   Consumer (one elected thread issues every MMA): layer 1 reads A from the
+//     stage and B (the decoder's weights, copied by a TMA bulk copy whenever
+//     the decoder changes) from shared memory; its completion frees the stage;
+//     the ReLU/convert epilogue goes TMEM -> registers -> TMEM; layers 2 and 3
+//     read their A operand from TMEM too; each layer's bias is one more K step
+//     whose A is a shared block with a 1 in K column 0.  The sigmoid epilogue
+//     scatters rows to out[perm[i]] while the next tile's layer 1 runs.
+// Shared-memory B operands use the no-swizzle K-major canonical layout: 8-row
+// x 16-byte core matrices, K-adjacent core matrices 128 B apart (LBO), 8-row
+// groups K*16 B apart (SBO).  Every wait is bounded by time; on expiry the
 // kernel records an error and stops cleanly (TMEM is always released).
 #include "ntc_internal.cuh"
 
 namespace ntc {
 
-constexpr int kTcKA = 32;  // K of the A tile: 16 features + bias column + pad
+constexpr int kTcKA = 32;  // K of layer 1's weight image: 16 features + the bias K step
 constexpr uint64_t kWaitLimitNs = 200ull * 1000ull * 1000ull;
 
 size_t tc_image_bytes(uint32_t H) {
@@ -101,9 +103,6 @@ __device__ __forceinline__ void fence_before() {
 __device__ __forceinline__ void fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
 }
-__device__ __forceinline__ void fence_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-}
 __device__ __forceinline__ void wg_bar(int wg) {
   asm volatile("bar.sync %0, 128;\n" ::"r"(wg + 1) : "memory");
 }
@@ -117,15 +116,6 @@ template <bool BF16>
 __host__ __device__ constexpr uint32_t instr_desc(uint32_t N) {
   return (1u << 4) | ((BF16 ? 1u : 0u) << 7) | ((BF16 ? 1u : 0u) << 10) | ((N >> 3) << 17) |
          ((128u >> 4) << 24);
-}
-
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
-                                     uint32_t accum) {
-  asm volatile(
-      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accum)
-      : "memory");
 }
 
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
@@ -205,36 +195,6 @@ __device__ __forceinline__ uint32_t pack(float lo, float hi) {
   return r;
 }
 
-__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
-               : "memory");
-}
-
-// TMEM accumulator row (H fp32 columns) -> ReLU -> fp16/bf16 hidden tile row.
-// CH columns are read per tcgen05.wait::ld (64: two loads in flight; 32: one).
-template <int H, bool BF16, int CH = (H <= 64 ? 64 : 32)>
-__device__ __forceinline__ void epilogue_hidden(uint32_t tmem_row, uint32_t sH, uint32_t row) {
-  constexpr uint32_t KH = H + 16;
-#pragma unroll 1
-  for (int c0 = 0; c0 < H; c0 += CH) {
-    uint32_t a[32], b[32];
-    tmem_ld32(tmem_row + c0, a);
-    if (CH == 64) tmem_ld32(tmem_row + c0 + 32, b);
-    tmem_wait_ld();
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-      sts128(sH + core_off(row, c0 + 8 * i, KH), pack_relu<BF16>(a[8 * i], a[8 * i + 1]),
-             pack_relu<BF16>(a[8 * i + 2], a[8 * i + 3]), pack_relu<BF16>(a[8 * i + 4], a[8 * i + 5]),
-             pack_relu<BF16>(a[8 * i + 6], a[8 * i + 7]));
-    if (CH == 64) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        sts128(sH + core_off(row, c0 + 32 + 8 * i, KH), pack_relu<BF16>(b[8 * i], b[8 * i + 1]),
-               pack_relu<BF16>(b[8 * i + 2], b[8 * i + 3]), pack_relu<BF16>(b[8 * i + 4], b[8 * i + 5]),
-               pack_relu<BF16>(b[8 * i + 6], b[8 * i + 7]));
-    }
-  }
-}
 
 template <int H>
 struct TcLayout {
@@ -243,9 +203,6 @@ struct TcLayout {
   static constexpr uint32_t W2 = H * KH * 2;
   static constexpr uint32_t W3 = 16 * KH * 2;
   static constexpr uint32_t WIMG = W1 + W2 + W3;
-  static constexpr uint32_t A = 128 * kTcKA * 2;
-  static constexpr uint32_t HT = 128 * KH * 2;
-  static constexpr uint32_t WG = WIMG + A + HT;  // shared bytes per warpgroup
 };
 
 // Latent taps of one query, loaded ahead of use: 8 taps (2 levels x 4), or 16
@@ -397,20 +354,6 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
       : "memory");
 }
 
-// Tile t of the bucketed order from (possibly shared-memory) copies of the
-// segment starts and tile starts: decoder, first sorted position and length.
-__device__ __forceinline__ void tile_lookup(const uint32_t *seg, const uint32_t *tst, uint32_t D,
-                                            uint32_t t, uint32_t &dec, uint32_t &start, uint32_t &len) {
-  uint32_t lo = 0, hi = D + 1;
-  while (hi - lo > 1) {
-    const uint32_t mid = (lo + hi) >> 1;
-    if (tst[mid] <= t) lo = mid; else hi = mid;
-  }
-  dec = lo;
-  start = seg[lo] + (t - tst[lo]) * kTile;
-  len = min((uint32_t)kTile, seg[lo + 1] - start);
-}
-
 // The tiles of one role in increasing order: the decoder index only moves
 // forward, so a lookup is a few compares instead of a binary search.
 struct TileWalk {
@@ -423,30 +366,6 @@ struct TileWalk {
     len = min((uint32_t)kTile, seg[d + 1] - start);
   }
 };
-
-// Per-thread view of one tile row.
-struct Row {
-  uint32_t dec, start, len;  // the tile
-  uint32_t oi;               // original query index of this row
-  bool valid, good;
-};
-
-__device__ __forceinline__ Row load_row(const Buckets &B, const uint32_t *seg, const uint32_t *tst,
-                                        uint32_t D, uint32_t t, uint32_t T, int tid, ntc_query &q) {
-  Row r;
-  r.valid = r.good = false;
-  r.oi = 0;
-  r.dec = 0xFFFFFFFFu;
-  r.start = r.len = 0;
-  if (t >= T) return r;
-  tile_lookup(seg, tst, D, t, r.dec, r.start, r.len);
-  r.valid = (uint32_t)tid < r.len;
-  if (r.valid) {
-    q = load_query(B.sorted + r.start + tid);
-    r.oi = __ldg(B.perm + r.start + tid);
-  }
-  return r;
-}
 
 constexpr uint32_t kSmemTileTable = 1024;  // staged when D + 2 <= this
 constexpr uint32_t kSmemGrids = 1024;      // staged when S * 2 * M <= this
@@ -505,10 +424,11 @@ struct TmCols {
 //   program order on both sides -- an mbarrier parity wait can then never be two
 //   phases ahead of its barrier.
 //   Producer: each thread computes the taps of one query row, blends them in
-//   fp32 and stores the fp16/bf16 feature row (plus the bias column) into the
-//   stage's TMEM A region (tcgen05.st; warp q of a warpgroup owns TMEM lanes
-//   32q..32q+31, exactly its rows); four warp arrivals fill the stage.  The next
-//   tile's query record is loaded while the current one is gathered.
+//   fp32 and stores the fp16/bf16 feature row into the stage's TMEM A region
+//   (tcgen05.st; warp q of a warpgroup owns TMEM lanes 32q..32q+31, exactly its
+//   rows), with the row's good flag and output index in shared memory; four
+//   warp arrivals fill the stage.  The next tile's query record and output
+//   index are loaded while the current tile is gathered.
 //   Consumer: layer 1 reads A from the stage and B (weights) from shared memory;
 //   its completion empties the stage; the ReLU/convert epilogue goes TMEM ->
 //   registers -> TMEM; layers 2 and 3 read their A from TMEM too; the sigmoid
