@@ -6,7 +6,8 @@ Workload (one "step" = one ntc_decode over one batch): 16 texture sets of
 non-shared baseline, one decoder per set), 4,194,304 queries with a uniform
 random set id, uniform UV in [0,1)^2 and lod 0 -- fully divergent (about 14
 distinct decoders per 32-query warp).  Inputs are resident in HBM; L2 is
-flushed (a 256 MiB write) before every timed step and the flush is outside the
+flushed (a 256 MiB write, then a 256 MiB read of another buffer, so no dirty
+flush lines are written back inside a step) before every timed step and the flush is outside the
 step's CUDA events.
 
 Prints one JSON line.  ``--impl reference`` times the CPU oracle instead (the
@@ -244,7 +245,14 @@ def main():
     qd = ntc.queries_to_device(w.queries)
     out = torch.empty((n, C), dtype=torch.float32, device="cuda")
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     stream = torch.cuda.current_stream()
+
+    def flush_l2():
+        # a write larger than L2, then a read of another buffer larger than L2:
+        # none of our data and no dirty lines are left in L2 when a step starts
+        flush.zero_()
+        flush_rd.sum()
 
     def barrier():
         if dist is not None:
@@ -261,7 +269,7 @@ def main():
         barrier()
         torch.cuda.synchronize()
         for i in range(steps):
-            flush.zero_()
+            flush_l2()
             ev[i][0].record(stream)
             dec.decode(qd, out, mode=mode)
             ev[i][1].record(stream)
@@ -326,7 +334,7 @@ def main():
         "config": {"workload": WORKLOAD if not args.small else "config2-small", "queries_per_gpu": n,
                    "decoders": w.assets.num_decoders, "mode": args.mode, "precision": args.precision,
                    "mean_distinct_decoders_per_warp": dd,
-                   "l2": "flushed before every timed step (256 MiB write, outside the step events)",
+                   "l2": "flushed before every timed step (256 MiB write, then a 256 MiB read of another buffer; outside the step events)",
                    "parallelism": f"{ws} independent replicas (queries sharded, no collective)"},
         "roofline": roofline, "e2e": e2e, "gpu_launches": launches, "clocks": clocks,
         "flops_per_query": FLOPS_PER_QUERY,
@@ -358,6 +366,7 @@ def sweep(ntc, torch, precision):
         qd = ntc.queries_to_device(wl.queries)
         out = torch.empty((len(wl.queries), a.out_dim), dtype=torch.float32, device="cuda")
         flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+        flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
         row = {"d": d}
         for mode in ("bucketed", "divergent"):
             for _ in range(2):
@@ -365,6 +374,7 @@ def sweep(ntc, torch, precision):
             ts = []
             for _ in range(5):
                 flush.zero_()
+                flush_rd.sum()
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 e0.record()
                 dec.decode(qd, out, mode=mode)
@@ -374,7 +384,7 @@ def sweep(ntc, torch, precision):
             row[mode] = len(wl.queries) / (statistics.mean(ts) / 1e3)
         row["bucketed_over_divergent"] = row["bucketed"] / row["divergent"]
         rows.append(row)
-        del qd, out, flush
+        del qd, out, flush, flush_rd
     dec.close()
     return rows
 

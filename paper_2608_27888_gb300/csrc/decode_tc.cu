@@ -304,46 +304,40 @@ __device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grid
   }
 }
 
-// acc[c/2] += w * tap[c] over the 8 channels of one tap, as packed fp32 pairs.
-__device__ __forceinline__ void accum_tap_x2(unsigned long long (&acc)[4], uint4 raw, float w) {
-  unsigned long long ww;
-  asm("mov.b64 %0, {%1, %1};" : "=l"(ww) : "f"(w));
+// acc[c/2] += w * tap[c] over the 8 channels of one tap, as packed fp32 pairs
+// (fma.rn.f32x2; the first tap multiplies, which rounds the same as an fma
+// into zero).
+template <bool FIRST>
+__device__ __forceinline__ void accum_tap_x2(float2 (&acc)[4], uint4 raw, float w) {
+  const float2 ww = make_float2(w, w);
   const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
 #pragma unroll
   for (int p = 0; p < 4; ++p) {
     const float2 x = __half22float2(h[p]);
-    unsigned long long xx;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(xx) : "f"(x.x), "f"(x.y));
-    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc[p]) : "l"(ww), "l"(xx));
+    acc[p] = FIRST ? __fmul2_rn(ww, x) : __ffma2_rn(ww, x, acc[p]);
   }
 }
 
 template <bool TRI, bool BF16>
 __device__ __forceinline__ void taps_to_row(const Taps<TRI> &tp, uint32_t (&packed)[8]) {
-  unsigned long long acc[kLevels][4];
+  float2 acc[kLevels][4];
 #pragma unroll
-  for (int k = 0; k < kLevels; ++k)
+  for (int k = 0; k < kLevels; ++k) {
+    accum_tap_x2<true>(acc[k], tp.raw[k * 4], tp.w[k * 4]);
 #pragma unroll
-    for (int p = 0; p < 4; ++p) acc[k][p] = 0ull;
-#pragma unroll
-  for (int k = 0; k < kLevels; ++k)
-#pragma unroll
-    for (int p = 0; p < 4; ++p) accum_tap_x2(acc[k], tp.raw[k * 4 + p], tp.w[k * 4 + p]);
+    for (int p = 1; p < 4; ++p) accum_tap_x2<false>(acc[k], tp.raw[k * 4 + p], tp.w[k * 4 + p]);
+  }
   if (TRI && __any_sync(0xFFFFFFFFu, tp.w[8] != 0.0f || tp.w[9] != 0.0f || tp.w[10] != 0.0f ||
                                          tp.w[11] != 0.0f)) {
 #pragma unroll
     for (int k = 0; k < kLevels; ++k)
 #pragma unroll
-      for (int p = 0; p < 4; ++p) accum_tap_x2(acc[k], tp.raw[8 + k * 4 + p], tp.w[8 + k * 4 + p]);
+      for (int p = 0; p < 4; ++p) accum_tap_x2<false>(acc[k], tp.raw[8 + k * 4 + p], tp.w[8 + k * 4 + p]);
   }
 #pragma unroll
   for (int k = 0; k < kLevels; ++k)
 #pragma unroll
-    for (int p = 0; p < 4; ++p) {
-      float lo, hi;
-      asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(acc[k][p]));
-      packed[k * 4 + p] = pack<BF16>(lo, hi);
-    }
+    for (int p = 0; p < 4; ++p) packed[k * 4 + p] = pack<BF16>(acc[k][p].x, acc[k][p].y);
 }
 
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
