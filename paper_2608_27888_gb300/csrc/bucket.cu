@@ -27,22 +27,24 @@ __device__ __forceinline__ uint32_t decoder_of(const Assets &A, uint32_t set_id)
 __device__ __forceinline__ uint32_t saddr_b(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 // Stream `bytes` (a multiple of 16) from global memory into shared memory with
-// one bulk copy (TMA) and wait for it; false if the copy has not landed after
-// 200 ms.  Called by every thread of the block; thread 0 issues the copy.
-__device__ bool bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+// one bulk copy (TMA): bulk_issue (every thread; thread 0 issues), then
+// bulk_wait, which is false if the copy has not landed after 200 ms.
+__device__ void bulk_issue(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
   const uint32_t b = saddr_b(bar);
   if (threadIdx.x == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(b) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(b), "r"(bytes) : "memory");
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
                      saddr_b(dst)),
                  "l"(src), "r"(bytes), "r"(b)
                  : "memory");
   }
+  __syncthreads();
+}
+
+__device__ bool bulk_wait(uint64_t *bar) {
+  const uint32_t b = saddr_b(bar);
   uint64_t t0 = 0;
   for (uint32_t spin = 0;; ++spin) {
     uint32_t ok;
@@ -71,7 +73,9 @@ __global__ void __launch_bounds__(kBucketThreads) k_hist(Assets A, const ntc_que
   const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
   const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
-  if (!bulk_load(srec, q + cbase, valid * 16u, &bar)) atomicOr(status, 2u);
+  bulk_issue(srec, q + cbase, valid * 16u, &bar);
+  pdl_trigger();  // k_scan may launch (it waits for this grid before reading)
+  if (!bulk_wait(&bar)) atomicOr(status, 2u);
   const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);
   uint32_t *my = cnt + warp * D1;
 #pragma unroll
@@ -150,6 +154,7 @@ __global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks
   __shared__ uint32_t ws[32];
   __shared__ bool last;
   const uint32_t d = blockIdx.x;
+  pdl_wait();  // the per-chunk counts of k_hist
   uint32_t tot = block_scan_inplace(counts + (size_t)d * chunks, chunks, ws);
   if (threadIdx.x == 0) {
     totals[d] = tot;
@@ -227,7 +232,10 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
   const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
   const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
-  if (!bulk_load(srec, q + cbase, valid * 16u, &bar)) atomicOr(status, 2u);
+  bulk_issue(srec, q + cbase, valid * 16u, &bar);  // the queries do not depend on k_scan
+  pdl_wait();                                        // the scanned counts and segment starts
+  pdl_trigger();                                     // the decode may launch (it waits for this grid)
+  if (!bulk_wait(&bar)) atomicOr(status, 2u);
   const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
   uint32_t dec[kBucketItems];
 #pragma unroll
@@ -325,10 +333,13 @@ cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const S
   uint32_t *totals = s.meta + meta_words(D);
   uint32_t *ticket = totals + (D + 1);
   k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks, status);
-  k_scan<<<D + 1, 1024, 0, st>>>(s.counts, chunks, D, (uint32_t)n, totals, s.meta, ticket);
-  k_scatter<<<chunks, kBucketThreads, smem_scatter, st>>>(A, q, n, s.counts, chunks, s.meta, s.perm, s.sorted,
-                                                          status);
+  cudaError_t e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, (uint32_t)n, totals,
+                             s.meta, ticket);
+  if (e == cudaSuccess)
+    e = launch_pdl(k_scatter, dim3(chunks), dim3(kBucketThreads), smem_scatter, st, A, q, n,
+                   (const uint32_t *)s.counts, chunks, (const uint32_t *)s.meta, s.perm, s.sorted, status);
   *launches += 3;
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -455,17 +455,6 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   // all-bad flags, never an uninitialised output index
   for (uint32_t i = threadIdx.x; i < (uint32_t)S * 128 / 4; i += blockDim.x)
     reinterpret_cast<uint32_t *>(smem + M::flags)[i] = 0u;
-  const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
-  if (D + 2 <= kSmemTileTable) {
-    uint32_t *s_seg = reinterpret_cast<uint32_t *>(smem + M::tiles);
-    uint32_t *s_tst = s_seg + kSmemTileTable;
-    for (uint32_t i = threadIdx.x; i < D + 2; i += blockDim.x) {
-      s_seg[i] = __ldg(seg + i);
-      s_tst[i] = __ldg(tst + i);
-    }
-    seg = s_seg;
-    tst = s_tst;
-  }
   const GridDesc *grids = A.pgrids;  // grid bases in the row-pair copy
   const uint32_t ngrids = A.num_sets * kLevels * A.num_mips;
   if (ngrids <= kSmemGrids) {
@@ -499,6 +488,19 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t z[8] = {one, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     tmem_st8(tmem_base + TC::ONES + lanes, z);
     tmem_wait_st();
+  }
+  // everything above is independent of the bucketing; the tile table is not
+  pdl_wait();
+  const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
+  if (D + 2 <= kSmemTileTable) {
+    uint32_t *s_seg = reinterpret_cast<uint32_t *>(smem + M::tiles);
+    uint32_t *s_tst = s_seg + kSmemTileTable;
+    for (uint32_t i = threadIdx.x; i < D + 2; i += blockDim.x) {
+      s_seg[i] = __ldg(seg + i);
+      s_tst[i] = __ldg(tst + i);
+    }
+    seg = s_seg;
+    tst = s_tst;
   }
   fence_before();
   __syncthreads();
@@ -740,10 +742,16 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   if (grid > max_tiles) grid = max_tiles;
   const int vec_out = ((uintptr_t)out & 15) == 0;
   const unsigned threads = (NP + NC) * 128;
+  // launched as a programmatic dependent of the bucketing: its prologue overlaps
+  // the end of k_scatter
+  cudaError_t e;
   if (c8)
-    k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+    e = launch_pdl(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC>, dim3((unsigned)grid), dim3(threads), smem, st,
+                   A, W, B, out, err, status, vec_out);
   else
-    k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC><<<(unsigned)grid, threads, smem, st>>>(A, W, B, out, err, status, vec_out);
+    e = launch_pdl(k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC>, dim3((unsigned)grid), dim3(threads), smem, st,
+                   A, W, B, out, err, status, vec_out);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

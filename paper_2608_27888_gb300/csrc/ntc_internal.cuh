@@ -73,6 +73,14 @@ inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D +
 
 // ------------------------------------------------------------- device helpers
 
+// Programmatic dependent launch: a kernel launched with launch_pdl may start
+// while its predecessor on the stream is still running; pdl_wait() blocks
+// until that predecessor has completed and its writes are visible (a no-op for
+// an ordinary launch).  pdl_trigger() lets the successor start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+
 // One axis of the tap addressing, fp32 round-to-nearest with no contraction.
 __device__ __forceinline__ void axis_taps(float c, uint32_t n, uint32_t mode, uint32_t &i0,
                                           uint32_t &i1, float &frac) {
@@ -247,6 +255,23 @@ cudaError_t launch_debug_taps(const Assets &A, const ntc_query *q, size_t n, uns
                               float *w, float *t, cudaStream_t st, int *launches);
 cudaError_t launch_debug_features(const Assets &A, const ntc_query *q, size_t n, float *f,
                                   cudaStream_t st, int *launches);
+// Launch with programmatic stream serialisation (see pdl_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 cudaError_t launch_build_pairs(const Assets &A, const uint32_t *chunk_grid, const uint32_t *chunk_start,
                                uint32_t num_chunks, uint4 *pair, cudaStream_t st);
 constexpr uint32_t kPairChunk = 65536;  // texels per work item of launch_build_pairs
