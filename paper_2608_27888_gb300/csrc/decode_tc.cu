@@ -682,9 +682,10 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
           y[cc] = fmaf(0.5f, th, 0.5f);
         }
         float *dst = out + (size_t)oi * C;
-        if (CP == 8 && vec_out && C == 8) {
-          reinterpret_cast<float4 *>(dst)[0] = make_float4(y[0], y[1], y[2], y[3]);
-          reinterpret_cast<float4 *>(dst)[1] = make_float4(y[4], y[5], y[6], y[7]);
+        if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
+          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]), "f"(y[1]),
+                       "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
+                       : "memory");
         } else {
 #pragma unroll
           for (int cc = 0; cc < CP; ++cc)
@@ -740,7 +741,7 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms;
   if (grid > max_tiles) grid = max_tiles;
-  const int vec_out = ((uintptr_t)out & 15) == 0;
+  const int vec_out = ((uintptr_t)out & 31) == 0;  // 32-byte rows need a 32-byte aligned base
   const unsigned threads = (NP + NC) * 128;
   // launched as a programmatic dependent of the bucketing: its prologue overlaps
   // the end of k_scatter
