@@ -283,17 +283,20 @@ __device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grid
                                            bool good, Taps<TRI> &tp) {
   const uint32_t sid = good ? q.set_id : 0u;
   const float u = good ? q.u : 0.0f, v = good ? q.v : 0.0f;
-  float t;
-  const int lo = select_mip(good ? q.lod : 0.0f, A.num_mips, t);
-  const GridDesc *g = grids + (size_t)sid * kLevels * A.num_mips;
+  // without trilinear blending (the kernel is only dispatched that way when
+  // there is one mip) the mip is always 0
+  float t = 0.0f;
+  const int lo = TRI ? select_mip(good ? q.lod : 0.0f, A.num_mips, t) : 0;
+  const uint32_t M = TRI ? A.num_mips : 1u;
+  const GridDesc *g = grids + (size_t)sid * kLevels * M;
   const float s = TRI ? __fsub_rn(1.0f, t) : 1.0f;
 #pragma unroll
-  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.pair, g[k * A.num_mips + lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
+  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.pair, g[k * M + lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
   if (TRI) {
     if (t > 0.0f) {
 #pragma unroll
       for (int k = 0; k < kLevels; ++k)
-        grid_fetch<WRAP>(A.pair, g[k * A.num_mips + lo + 1], u, v, t, tp.raw + 8 + 4 * k, tp.w + 8 + 4 * k);
+        grid_fetch<WRAP>(A.pair, g[k * M + lo + 1], u, v, t, tp.raw + 8 + 4 * k, tp.w + 8 + 4 * k);
     } else {
 #pragma unroll
       for (int i = 8; i < Taps<TRI>::N; ++i) {
@@ -377,8 +380,9 @@ struct TmSmem {
   using L = TcLayout<H>;
   static constexpr int S = NC * SC;                                     // stages in all rings
   static constexpr size_t weights = 0;                                  // per consumer
-  static constexpr size_t flags = weights + (size_t)NC * L::WIMG;       // per stage: 128 row flags
-  static constexpr size_t oidx = flags + (size_t)S * 128;               // per stage: 128 output rows
+  // per stage: 128 output rows, 0xFFFFFFFF for a row that is not good (never
+  // a valid row: n <= 2^32 - 256)
+  static constexpr size_t oidx = weights + (size_t)NC * L::WIMG;
   static constexpr size_t bars = oidx + (size_t)S * 128 * 4;
   static constexpr int nbars = 2 * S + 2 * NC;                          // full, empty, mma, weights
   static constexpr size_t misc = bars + (size_t)nbars * 8;
@@ -420,7 +424,8 @@ struct TmCols {
 //   Producer: each thread computes the taps of one query row, blends them in
 //   fp32 and stores the fp16/bf16 feature row into the stage's TMEM A region
 //   (tcgen05.st; warp q of a warpgroup owns TMEM lanes 32q..32q+31, exactly its
-//   rows), with the row's good flag and output index in shared memory; four
+//   rows), with the row's output index (or 0xFFFFFFFF if the row is not good)
+//   in shared memory; four
 //   warp arrivals fill the stage.  The next tile's query record and output
 //   index are loaded while the current tile is gathered.
 //   Consumer: layer 1 reads A from the stage and B (weights) from shared memory;
@@ -452,9 +457,9 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   const uint32_t D = A.num_decoders, C = W.out_dim;
 
   // no stage has rows yet: a consumer that stops on a wait timeout reads
-  // all-bad flags, never an uninitialised output index
-  for (uint32_t i = threadIdx.x; i < (uint32_t)S * 128 / 4; i += blockDim.x)
-    reinterpret_cast<uint32_t *>(smem + M::flags)[i] = 0u;
+  // all-bad rows, never an uninitialised output index
+  for (uint32_t i = threadIdx.x; i < (uint32_t)S * 128; i += blockDim.x)
+    reinterpret_cast<uint32_t *>(smem + M::oidx)[i] = 0xFFFFFFFFu;
   const GridDesc *grids = A.pgrids;  // grid bases in the row-pair copy
   const uint32_t ngrids = A.num_sets * kLevels * A.num_mips;
   if (ngrids <= kSmemGrids) {
@@ -556,8 +561,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       fence_after();
       tmem_st8(tmem_base + TC::a1(s) + lanes, a);
       tmem_wait_st();
-      smem[M::flags + s * 128 + row] = good ? 1 : 0;
-      reinterpret_cast<uint32_t *>(smem + M::oidx)[s * 128 + row] = oi;
+      reinterpret_cast<uint32_t *>(smem + M::oidx)[s * 128 + row] = good ? oi : 0xFFFFFFFFu;
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(full_bar(s));
@@ -601,7 +605,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       tmem_wait_st();
     };
     // Start tile k: its decoder's weights, wait for its A stage (with the
-    // rows' flags and output indices) and issue layer 1.  Requires this
+    // rows' output indices) and issue layer 1.  Requires this
     // consumer's previous tile to have finished all MMAs.
     auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good) {
       const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
@@ -619,8 +623,8 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         wph ^= 1;
       }
       wg_bar(wgid);
-      good = smem[M::flags + s * 128 + row] != 0;
       oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[s * 128 + row];
+      good = oi != 0xFFFFFFFFu;
       if (row == 0) {
         fence_after();
         if (dec < D) {
