@@ -24,6 +24,26 @@ __device__ __forceinline__ uint32_t decoder_of(const Assets &A, uint32_t set_id)
   return set_id < A.num_sets ? __ldg(A.map + set_id) : A.num_decoders;
 }
 
+// The set -> decoder map of up to 32 sets lives in one register per lane
+// (lane s holds map[s]); larger maps are read through the cache.
+struct MapLookup {
+  uint32_t reg;
+  bool small;
+  __device__ explicit MapLookup(const Assets &A) {
+    const uint32_t lane = threadIdx.x & 31;
+    small = A.num_sets <= 32;
+    reg = small && lane < A.num_sets ? __ldg(A.map + lane) : A.num_decoders;
+  }
+  // called by all 32 lanes of the warp together
+  __device__ __forceinline__ uint32_t operator()(const Assets &A, uint32_t set_id) const {
+    if (small) {
+      const uint32_t d = __shfl_sync(0xFFFFFFFFu, reg, set_id & 31);
+      return set_id < A.num_sets ? d : A.num_decoders;
+    }
+    return decoder_of(A, set_id);
+  }
+};
+
 __device__ __forceinline__ uint32_t saddr_b(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 // Stream `bytes` (a multiple of 16) from global memory into shared memory with
@@ -70,6 +90,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_hist(Assets A, const ntc_que
   uint32_t *cnt = reinterpret_cast<uint32_t *>(srec + kBucketChunk);
   const uint32_t D1 = A.num_decoders + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const MapLookup lookup(A);
   const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
   const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
@@ -81,7 +102,8 @@ __global__ void __launch_bounds__(kBucketThreads) k_hist(Assets A, const ntc_que
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
     const uint32_t j = wbase + it * 32 + lane;
-    const uint32_t d = j < valid ? decoder_of(A, srec[j].x) : 0xFFFFFFFFu;
+    const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
+    const uint32_t d = j < valid ? dl : 0xFFFFFFFFu;
     const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
     if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
     __syncwarp();
@@ -229,6 +251,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
   uint32_t *loff = cnt + kWarps * D1;  // chunk-local start of each decoder's run
   uint32_t *gbase = loff + D1;         // global position of that run's first element
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const MapLookup lookup(A);
   const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
   const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
@@ -241,7 +264,8 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
     const uint32_t j = wbase + it * 32 + lane;
-    dec[it] = j < valid ? decoder_of(A, srec[j].x) : 0xFFFFFFFFu;
+    const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
+    dec[it] = j < valid ? dl : 0xFFFFFFFFu;
   }
   uint32_t *my = cnt + warp * D1;
   // rank of each query among the equal decoders of this warp's run, in order
