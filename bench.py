@@ -10,6 +10,12 @@ flushed (a 256 MiB write, then a 256 MiB read of another buffer, so no dirty
 flush lines are written back inside a step) before every timed step and the flush is outside the
 step's CUDA events.
 
+Beside the headline the line carries the in-run comparisons: the unsorted
+mma.sync ("divergent") and per-lane FMA ("divergent_fma") kernels on the same
+batch, a sweep over exactly d distinct decoders per warp, and a mirror of the
+paper's Tables 5-6 (shared vs non-shared decoders at 5 and 10 decoders per warp,
+512^2 to 8192^2 queries).
+
 Prints one JSON line.  ``--impl reference`` times the CPU oracle instead (the
 only other code that computes the same result) on a bounded query sample.
 
@@ -44,7 +50,9 @@ L2_FLUSH_BYTES = 256 << 20
 KERNEL_NAMES = {("bucketed", False): "k_decode_tc (tcgen05/TMEM gather-decode)",
                 ("bucketed", True): "k_decode_fp32 (FFMA gather-decode)",
                 ("bucketed_mma", False): "k_decode_mma (mma.sync gather-decode)",
-                ("divergent", False): "k_decode_divergent (mma.sync, unsorted)"}
+                ("divergent", False): "k_decode_divergent (mma.sync, unsorted)",
+                ("divergent_fma", False): "k_decode_divergent_fma (per-lane FFMA, unsorted)",
+                ("divergent_fma", True): "k_decode_divergent_fma (per-lane FFMA, unsorted)"}
 
 
 def parse():
@@ -53,10 +61,11 @@ def parse():
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", default="ntc", choices=["ntc", "reference"])
-    p.add_argument("--mode", default="bucketed", choices=["bucketed", "bucketed_mma", "divergent"])
+    p.add_argument("--mode", default="bucketed", choices=["bucketed", "bucketed_mma", "divergent", "divergent_fma"])
     p.add_argument("--precision", default="fp16", choices=["fp16", "bf16", "fp32"])
     p.add_argument("--no-sweep", action="store_true", help="skip the decoders-per-warp sweep")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    p.add_argument("--no-mirror", action="store_true", help="skip the mirror of the paper's Tables 5-6")
     p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
     return p.parse_args()
 
@@ -323,10 +332,12 @@ def main():
 
     # the in-run comparison: the unsorted divergent kernel on the same batch
     extra = {}
-    if args.mode != "divergent" and args.precision != "fp32":
-        dms, _, _ = timed_steps("divergent", max(5, args.steps // 2), 2)
-        extra["divergent"] = {"value": n * ws / (statistics.mean(dms) / 1e3), "unit": UNIT,
-                              "ms_per_step": statistics.mean(dms)}
+    for other in ("divergent", "divergent_fma"):
+        if args.mode == other or (args.precision == "fp32" and other == "divergent"):
+            continue
+        dms, _, _ = timed_steps(other, max(5, args.steps // 2), 2)
+        extra[other] = {"value": n * ws / (statistics.mean(dms) / 1e3), "unit": UNIT,
+                        "ms_per_step": statistics.mean(dms)}
     dd = mean_distinct(w.queries, w.assets)
 
     result = {
@@ -348,6 +359,8 @@ def main():
 
     if not args.no_sweep and not args.small and rank == 0:
         result["sweep"] = sweep(ntc, torch, args.precision)
+    if not args.no_mirror and not args.small and rank == 0 and args.precision != "fp32":
+        result["paper_mirror"] = paper_mirror(ntc, torch, args.precision)
 
     if rank == 0 and not args.no_cpu and ws == 1:
         result["cpu_baseline"] = cpu_baseline(w)
@@ -355,6 +368,68 @@ def main():
         print(json.dumps(result), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def time_decode(torch, dec, qd, out, mode, flush, flush_rd, reps=5, warm=2):
+    """Mean ms of one ntc_decode on the current stream, L2 flushed before each."""
+    for _ in range(warm):
+        dec.decode(qd, out, mode=mode)
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        flush_rd.sum()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        dec.decode(qd, out, mode=mode)
+        e1.record()
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    return statistics.mean(ts)
+
+
+def paper_mirror(ntc, torch, precision, sizes=(512, 1024, 2048, 4096, 8192), ds=(5, 10)):
+    """The setting of the paper's Tables 5-6 on this GPU: an N x N texel-centre
+    raster where every 32-query warp holds d distinct texture sets (32 sets of
+    1024^2), decoded once with one decoder shared by all sets ("Shared-Decoder")
+    and once with one decoder per set (d distinct decoders per warp).  Times in
+    microseconds: shared = the warp-level mma.sync kernel on the shared map (one
+    decoder per warp, no loop); wmma / fma = the unsorted mma.sync and per-lane
+    FMA kernels on the per-set map ("Non-Shared WMMA / FMA"); bucketed = this
+    library's default path (sort by decoder, tcgen05 decode) on the per-set map.
+    avg_increase_* is the paper's statistic, mean(t_nonshared / t_shared) - 1."""
+    from paper_2608_27888_gb300 import workloads as W
+    S, T = 32, 1024
+    seed = W.BASE_SEED + 100
+    a_sh = W.make_assets(seed, S, T, 1, 1, W.map_shared(S))
+    a_ns = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
+    dsh, dns = ntc.Decoder(a_sh, precision), ntc.Decoder(a_ns, precision)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    rows = []
+    for d in ds:
+        for N in sizes:
+            q = W.queries_controlled(seed + d, N, S, d)
+            qd = ntc.queries_to_device(q)
+            out = torch.empty((len(q), a_ns.out_dim), dtype=torch.float32, device="cuda")
+            reps = 5 if N <= 4096 else 3
+            row = {"d": d, "N": N,
+                   "shared_us": 1e3 * time_decode(torch, dsh, qd, out, "divergent", flush, flush_rd, reps),
+                   "shared_bucketed_us": 1e3 * time_decode(torch, dsh, qd, out, "bucketed", flush, flush_rd, reps),
+                   "wmma_us": 1e3 * time_decode(torch, dns, qd, out, "divergent", flush, flush_rd, reps),
+                   "fma_us": 1e3 * time_decode(torch, dns, qd, out, "divergent_fma", flush, flush_rd, reps),
+                   "bucketed_us": 1e3 * time_decode(torch, dns, qd, out, "bucketed", flush, flush_rd, reps)}
+            rows.append(row)
+            del qd, out
+    dsh.close()
+    dns.close()
+    summary = {}
+    for d in ds:
+        rs = [r for r in rows if r["d"] == d]
+        for k in ("wmma", "fma", "bucketed"):
+            summary[f"d{d}_avg_increase_{k}_over_shared"] = statistics.mean(
+                r[f"{k}_us"] / r["shared_us"] for r in rs) - 1.0
+    return {"rows": rows, "summary": summary,
+            "what": "32 sets of 1024^2, N x N texel-centre raster, d distinct sets per warp; times in us"}
 
 
 def sweep(ntc, torch, precision):
@@ -373,21 +448,12 @@ def sweep(ntc, torch, precision):
         flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
         flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
         row = {"d": d}
-        for mode in ("bucketed", "divergent"):
-            for _ in range(2):
-                dec.decode(qd, out, mode=mode)
-            ts = []
-            for _ in range(5):
-                flush.zero_()
-                flush_rd.sum()
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record()
-                dec.decode(qd, out, mode=mode)
-                e1.record()
-                torch.cuda.synchronize()
-                ts.append(e0.elapsed_time(e1))
-            row[mode] = len(wl.queries) / (statistics.mean(ts) / 1e3)
-        row["bucketed_over_divergent"] = row["bucketed"] / row["divergent"]
+        modes = ("bucketed", "divergent_fma") if precision == "fp32" else ("bucketed", "divergent", "divergent_fma")
+        for mode in modes:
+            ms = time_decode(torch, dec, qd, out, mode, flush, flush_rd, reps=5)
+            row[mode] = len(wl.queries) / (ms / 1e3)
+        for mode in modes[1:]:
+            row[f"bucketed_over_{mode}"] = row["bucketed"] / row[mode]
         rows.append(row)
         del qd, out, flush, flush_rd
     dec.close()

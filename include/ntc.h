@@ -88,11 +88,18 @@ typedef enum {
  *               its distinct decoders (the non-shared setting of Sec. 4.4).
  *               Tensor-core precisions only.
  * BUCKETED_MMA: the bucketed path with the warp-level mma.sync decode kernel.
- *               Tensor-core precisions only. */
+ *               Tensor-core precisions only.
+ * DIVERGENT_FMA: no sorting and no tensor cores: every thread evaluates its
+ *               own query's decoder with fp32 fused multiply-adds, weights read
+ *               per lane (the "Non-Shared FMA" setting of Sec. 4.4, Tables
+ *               5-6).  Every precision: with TC_FP16/TC_BF16 the features,
+ *               weights and hidden activations are rounded to that type and
+ *               accumulated in fp32; FP32 rounds nothing. */
 typedef enum {
   NTC_MODE_BUCKETED = 0,
   NTC_MODE_DIVERGENT = 1,
-  NTC_MODE_BUCKETED_MMA = 2
+  NTC_MODE_BUCKETED_MMA = 2,
+  NTC_MODE_DIVERGENT_FMA = 3
 } ntc_mode;
 
 /* Everything ntc_create needs.  All pointers are HOST memory owned by the

@@ -30,7 +30,8 @@ struct ntc_ctx {
   uint8_t *d_mma = nullptr;
   float *d_f32 = nullptr;
   uint8_t *d_tc = nullptr;
-  size_t mma_stride = 0, f32_stride = 0, tc_stride = 0;
+  uint8_t *d_fma = nullptr;
+  size_t mma_stride = 0, f32_stride = 0, tc_stride = 0, fma_stride = 0;
   unsigned long long *d_err = nullptr;
   unsigned int *d_status = nullptr;  // nonzero: a decode kernel gave up a bounded wait
   // bucketing scratch (grows on demand, stream-ordered)
@@ -114,6 +115,8 @@ WeightImages weights_of(const ntc_ctx *c) {
   W.f32_stride = c->f32_stride;
   W.tc = c->d_tc;
   W.tc_stride = c->tc_stride;
+  W.fma = c->d_fma;
+  W.fma_stride = c->fma_stride;
   W.hidden = c->H;
   W.out_dim = c->C;
   return W;
@@ -137,6 +140,7 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_mma);
   cudaFree(c->d_f32);
   cudaFree(c->d_tc);
+  cudaFree(c->d_fma);
   cudaFree(c->d_err);
   cudaFree(c->d_status);
   cudaFree(c->d_counts);
@@ -275,6 +279,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   c->mma_stride = round16(mma_image_bytes(c->H));
   c->f32_stride = (f32_image_floats(c->H, c->C) + 3) & ~(size_t)3;
   c->tc_stride = round16(tc_image_bytes(c->H));
+  c->fma_stride = round16(fma_image_bytes(c->H, c->C, c->prec == NTC_PREC_FP32 ? 4u : 2u));
   // the row-pair copy: grids back to back, built in chunks of kPairChunk texels
   std::vector<GridDesc> pgrids(grids.size());
   std::vector<uint32_t> chunk_grid, chunk_start;
@@ -301,6 +306,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   step(cudaMalloc((void **)&c->d_mma, c->mma_stride * c->D));
   step(cudaMalloc((void **)&c->d_f32, c->f32_stride * 4 * c->D));
   step(cudaMalloc((void **)&c->d_tc, c->tc_stride * c->D));
+  step(cudaMalloc((void **)&c->d_fma, c->fma_stride * c->D));
   step(cudaMalloc((void **)&c->d_err, sizeof(unsigned long long)));
   step(cudaMalloc((void **)&c->d_status, sizeof(unsigned int)));
   step(cudaMalloc((void **)&d_w32, P * 4 * c->D));
@@ -323,6 +329,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
     step(cudaMemset(c->d_tc, 0, c->tc_stride * c->D));
     step(launch_pack_weights(d_w32, c->D, c->H, c->C, c->prec == NTC_PREC_TC_BF16, c->d_mma,
                              c->mma_stride, c->d_f32, c->f32_stride, c->d_tc, c->tc_stride, 0));
+    step(launch_pack_fma(d_w32, c->D, c->H, c->C, c->prec, c->d_fma, c->fma_stride, 0));
     step(cudaDeviceSynchronize());
   }
   cudaFree(d_w32);
@@ -351,11 +358,12 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   if (s != NTC_OK) return s;
   if (n && !out) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
   if (((uintptr_t)out & 3) != 0) return fail(NTC_ERR_INVALID_ARG, "output buffer is not 4-byte aligned");
-  if (mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT && mode != NTC_MODE_BUCKETED_MMA)
+  if (mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT && mode != NTC_MODE_BUCKETED_MMA &&
+      mode != NTC_MODE_DIVERGENT_FMA)
     return fail(NTC_ERR_INVALID_ARG, "unknown mode");
   const bool fp32 = c->prec == NTC_PREC_FP32;
-  if (fp32 && mode != NTC_MODE_BUCKETED)
-    return fail(NTC_ERR_UNSUPPORTED, "the fp32 precision has only the bucketed mode");
+  if (fp32 && mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT_FMA)
+    return fail(NTC_ERR_UNSUPPORTED, "the fp32 precision has only the bucketed and divergent FMA modes");
   if (n == 0) return NTC_OK;
   DeviceGuard g(c->device);
   if (!g.ok) return fail(NTC_ERR_CUDA, "cannot select the context's device");
@@ -365,12 +373,16 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   const bool bf16 = c->prec == NTC_PREC_TC_BF16;
   int launches = 0;
   cudaError_t e;
-  s = mode == NTC_MODE_DIVERGENT ? NTC_OK : ensure_scratch(c, n, st);
+  const bool unsorted = mode == NTC_MODE_DIVERGENT || mode == NTC_MODE_DIVERGENT_FMA;
+  s = unsorted ? NTC_OK : ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
   if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
-  if (mode == NTC_MODE_DIVERGENT) {
+  if (unsorted) {
     if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
-    e = launch_decode_divergent(A, W, q, n, out, c->d_err, bf16, c->num_sms, st, &launches);
+    if (mode == NTC_MODE_DIVERGENT)
+      e = launch_decode_divergent(A, W, q, n, out, c->d_err, bf16, c->num_sms, st, &launches);
+    else
+      e = launch_decode_divergent_fma(A, W, q, n, out, c->d_err, c->prec, c->num_sms, st, &launches);
     c->launches += launches;
     if (e != cudaSuccess) return cuda_fail(e, "divergent decode launch");
     if (c->timing) {

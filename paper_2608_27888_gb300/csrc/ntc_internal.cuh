@@ -50,8 +50,11 @@ struct WeightImages {
   size_t f32_stride;
   const uint8_t *tc;        // [D][tc_stride] bytes, tcgen05 shared-memory image
   size_t tc_stride;
+  const uint8_t *fma;       // [D][fma_stride] bytes, per-lane FMA image
+  size_t fma_stride;
   uint32_t hidden, out_dim;
 };
+
 
 inline __host__ __device__ size_t mma_image_bytes(uint32_t H) {
   return (size_t)H * (16 + 8) * 2 + (size_t)H * (H + 8) * 2 + (size_t)16 * (H + 8) * 2 +
@@ -61,6 +64,13 @@ inline __host__ __device__ uint32_t out_pad(uint32_t C) { return C <= 8 ? 8u : 1
 inline __host__ __device__ size_t f32_image_floats(uint32_t H, uint32_t C) {
   uint32_t CP = out_pad(C);
   return (size_t)H * 16 + H + (size_t)H * H + H + (size_t)CP * H + CP;
+}
+// Per-lane FMA image, element type T = the precision's operand type (fp32,
+// fp16 or bf16): W1[H][16], W2[H][H], W3^T[H][CP] in T, then fp32 b1[H],
+// b2[H], b3[CP] (rows of W3^T and entries of b3 at c >= C are zero).
+inline __host__ __device__ size_t fma_image_bytes(uint32_t H, uint32_t C, uint32_t elem) {
+  const size_t CP = out_pad(C);
+  return ((size_t)H * 16 + (size_t)H * H + (size_t)H * CP) * elem + (2 * (size_t)H + CP) * 4;
 }
 
 // Bucketing results on the device.
@@ -246,6 +256,11 @@ cudaError_t launch_decode_mma(const Assets &A, const WeightImages &W, const Buck
 cudaError_t launch_decode_divergent(const Assets &A, const WeightImages &W, const ntc_query *q,
                                     size_t n, float *out, unsigned long long *err, bool bf16,
                                     int num_sms, cudaStream_t st, int *launches);
+cudaError_t launch_decode_divergent_fma(const Assets &A, const WeightImages &W, const ntc_query *q,
+                                        size_t n, float *out, unsigned long long *err, ntc_precision prec,
+                                        int num_sms, cudaStream_t st, int *launches);
+cudaError_t launch_pack_fma(const float *w32, uint32_t D, uint32_t H, uint32_t C, ntc_precision prec,
+                            uint8_t *fma, size_t fma_stride, cudaStream_t st);
 cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
                              float *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches);

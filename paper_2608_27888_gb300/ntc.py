@@ -18,12 +18,13 @@ LIB_PATH = os.path.join(_HERE, "_build", "libntc.so")
 
 NTC_OK, NTC_ERR_INVALID_ARG, NTC_ERR_UNSUPPORTED, NTC_ERR_OUT_OF_MEMORY, NTC_ERR_CUDA = range(5)
 NTC_PREC_TC_FP16, NTC_PREC_TC_BF16, NTC_PREC_FP32 = range(3)
-NTC_MODE_BUCKETED, NTC_MODE_DIVERGENT, NTC_MODE_BUCKETED_MMA = range(3)
+NTC_MODE_BUCKETED, NTC_MODE_DIVERGENT, NTC_MODE_BUCKETED_MMA, NTC_MODE_DIVERGENT_FMA = range(4)
 NTC_MAX_DECODERS = 4095
 NTC_TILE_ROWS = 128
 
 PRECISIONS = {"fp16": NTC_PREC_TC_FP16, "bf16": NTC_PREC_TC_BF16, "fp32": NTC_PREC_FP32}
-MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucketed_mma": NTC_MODE_BUCKETED_MMA}
+MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucketed_mma": NTC_MODE_BUCKETED_MMA,
+         "divergent_fma": NTC_MODE_DIVERGENT_FMA}
 EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps",
            "ntc_debug_features", "ntc_debug_bucket", "ntc_max_tiles", "ntc_get_error_count",
            "ntc_reset_error_count", "ntc_launch_count", "ntc_set_stage_timing", "ntc_stage_times",

@@ -166,16 +166,17 @@ def test_features_match_oracle(k, variant):
 
 # --------------------------------------------------------------- decode
 
+@pytest.mark.parametrize("mode", ["bucketed", "divergent_fma"])
 @pytest.mark.parametrize("k,variant", SMALL)
-def test_decode_fp32_mode(k, variant):
+def test_decode_fp32_mode(k, variant, mode):
     w = small(k, variant)
     ref, _ = oracle_out(k, variant)
-    got = decoder(k, variant, "fp32").decode(dq(w.queries)).cpu().numpy()
+    got = decoder(k, variant, "fp32").decode(dq(w.queries), mode=mode).cpu().numpy()
     assert np.abs(got - ref).max() <= FP32_TOL
 
 
 @pytest.mark.parametrize("precision", ["fp16", "bf16"])
-@pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent"])
+@pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent", "divergent_fma"])
 @pytest.mark.parametrize("k,variant", SMALL)
 def test_decode_tensor_core_modes(k, variant, mode, precision):
     w = small(k, variant)
@@ -187,7 +188,9 @@ def test_decode_tensor_core_modes(k, variant, mode, precision):
 def test_hidden_128_and_9_channels_on_all_paths():
     w = small(5)
     ref, _ = oracle_out(5)
-    for prec, modes in (("fp32", ["bucketed"]), ("fp16", ["bucketed", "bucketed_mma", "divergent"])):
+    for prec, modes in (("fp32", ["bucketed", "divergent_fma"]),
+                        ("fp16", ["bucketed", "bucketed_mma", "divergent", "divergent_fma"]),
+                        ("bf16", ["divergent_fma"])):
         dec = decoder(5, None, prec)
         for m in modes:
             got = dec.decode(dq(w.queries), mode=m).cpu().numpy()
@@ -197,19 +200,16 @@ def test_hidden_128_and_9_channels_on_all_paths():
                 check_tc(got, ref, m)
 
 
-@pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent"])
+@pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent", "divergent_fma"])
 def test_order_invariance_is_bitwise(mode):
     w = small(3, "clustered4")
     dec = decoder(3, "clustered4", "fp16")
     out = dec.decode(dq(w.queries), mode=mode).cpu().numpy()
     p = np.random.default_rng(1).permutation(len(w.queries))
     out2 = dec.decode(dq(w.queries[p]), mode=mode).cpu().numpy()
-    if mode == "divergent":
-        # each warp's rows see the same decoder loop whatever their neighbours,
-        # but fp16 rounding of a row is independent of the other rows too
-        assert np.array_equal(out2, out[p])
-    else:
-        assert np.array_equal(out2, out[p])
+    # every row's arithmetic is independent of the other rows of its tile or
+    # warp (the divergent kernels mask, they do not mix rows)
+    assert np.array_equal(out2, out[p])
 
 
 def test_bad_queries_nan_and_counted():
@@ -222,7 +222,7 @@ def test_bad_queries_nan_and_counted():
     ref, bad = oracle.decode(w.assets, q)
     assert bad == nbad
     for prec, mode in (("fp32", "bucketed"), ("fp16", "bucketed"), ("fp16", "bucketed_mma"),
-                       ("fp16", "divergent")):
+                       ("fp16", "divergent"), ("fp16", "divergent_fma"), ("fp32", "divergent_fma")):
         dec = ntc().Decoder(w.assets, prec)
         got = dec.decode(dq(q), mode=mode).cpu().numpy()
         assert np.array_equal(np.isnan(got), np.isnan(ref)), (prec, mode)
@@ -272,8 +272,9 @@ def test_full_size_sampled(k, variant):
     out = dec.decode(qd, mode="bucketed")
     got = out[torch.from_numpy(sample).cuda()].cpu().numpy()
     check_tc(got, ref, f"config {k} full bucketed")
-    div = dec.decode(qd, mode="divergent")[torch.from_numpy(sample).cuda()].cpu().numpy()
-    check_tc(div, ref, f"config {k} full divergent")
+    for mode in ("divergent", "divergent_fma"):
+        div = dec.decode(qd, mode=mode)[torch.from_numpy(sample).cuda()].cpu().numpy()
+        check_tc(div, ref, f"config {k} full {mode}")
     perm, counts, tiles = dec.bucket(qd)
     p, c, _, t = oracle.bucket(w.queries["set_id"], w.assets.set_to_decoder, w.assets.num_decoders)
     assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
