@@ -66,6 +66,8 @@ def parse():
     p.add_argument("--no-sweep", action="store_true", help="skip the decoders-per-warp sweep")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     p.add_argument("--no-mirror", action="store_true", help="skip the mirror of the paper's Tables 5-6")
+    p.add_argument("--configs", action="store_true",
+                   help="also time every full-size workload (1-5 and their maps); adds about two minutes")
     p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
     return p.parse_args()
 
@@ -361,6 +363,8 @@ def main():
         result["sweep"] = sweep(ntc, torch, args.precision)
     if not args.no_mirror and not args.small and rank == 0 and args.precision != "fp32":
         result["paper_mirror"] = paper_mirror(ntc, torch, args.precision)
+    if args.configs and rank == 0:
+        result["configs"] = per_config(ntc, torch, args.precision)
 
     if rank == 0 and not args.no_cpu and ws == 1:
         result["cpu_baseline"] = cpu_baseline(w)
@@ -430,6 +434,51 @@ def paper_mirror(ntc, torch, precision, sizes=(512, 1024, 2048, 4096, 8192), ds=
                 r[f"{k}_us"] / r["shared_us"] for r in rs) - 1.0
     return {"rows": rows, "summary": summary,
             "what": "32 sets of 1024^2, N x N texel-centre raster, d distinct sets per warp; times in us"}
+
+
+def per_config(ntc, torch, precision):
+    """Every full-size workload: queries/s of the whole ntc_decode (bucketed),
+    the bucketing / gather-decode split, the unsorted kernels, and the whole
+    step against the roofline rate of that workload's algorithmic bytes."""
+    from paper_2608_27888_gb300 import workloads as W
+    peak, _ = peaks()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    rows = []
+    for k, variant in ((1, None), (2, None), (3, "identity"), (3, "clustered4"), (3, "shared"),
+                       (4, "128"), (4, "16"), (4, "8"), (4, "1"), (5, None)):
+        w = W.config(k, "full", variant)
+        a, q = w.assets, w.queries
+        n, C = len(q), a.out_dim
+        dec = ntc.Decoder(a, precision)
+        qd = ntc.queries_to_device(q)
+        out = torch.empty((n, C), dtype=torch.float32, device="cuda")
+        ms = time_decode(torch, dec, qd, out, "bucketed", flush, flush_rd, reps=10, warm=3)
+        dec.set_stage_timing(True)
+        st = []
+        for _ in range(5):
+            flush.zero_()
+            flush_rd.sum()
+            dec.decode(qd, out, mode="bucketed")
+            st.append(dec.stage_times())
+        dec.set_stage_timing(False)
+        tri = a.num_mips > 1 and bool((q["lod"] != np.floor(q["lod"])).any())
+        bpq = 16 + (16 if tri else 8) * 16 + 4 * C
+        dd = mean_distinct(q, a)
+        row = {"workload": w.name, "queries": n, "decoders": a.num_decoders, "hidden": a.hidden,
+               "mean_distinct_decoders_per_warp": dd, "divergence_score_eq1": dd - 1.0,
+               "bucketed": n / (ms / 1e3), "ms_per_step": ms,
+               "bucketing_ms": statistics.mean(t[0] for t in st), "decode_ms": statistics.mean(t[1] for t in st),
+               "bytes_per_query": bpq, "roofline_rate": peak * 1e9 / bpq}
+        row["frac_of_roofline"] = row["bucketed"] / row["roofline_rate"]
+        reps = 3 if n > 10_000_000 else 5
+        for m in (("divergent_fma",) if precision == "fp32" else ("divergent", "divergent_fma")):
+            row[m] = n / (time_decode(torch, dec, qd, out, m, flush, flush_rd, reps=reps, warm=1) / 1e3)
+        rows.append(row)
+        dec.close()
+        del qd, out, w, a, q
+        torch.cuda.empty_cache()
+    return rows
 
 
 def sweep(ntc, torch, precision):

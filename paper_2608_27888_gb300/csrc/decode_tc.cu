@@ -205,14 +205,19 @@ struct TcLayout {
   static constexpr uint32_t WIMG = W1 + W2 + W3;
 };
 
-// Latent taps of one query, loaded ahead of use: 8 taps (2 levels x 4), or 16
-// when a mip blend is possible (mip lo, then mip lo+1); the blend factor is
-// folded into the weights.
-template <bool TRI>
+// Latent taps of one query from one mip, loaded ahead of use: 2 levels x 4
+// taps; a mip blend factor is folded into the weights.
 struct Taps {
-  static constexpr int N = TRI ? 16 : 8;
+  static constexpr int N = 8;
   uint4 raw[N];
   float w[N];
+};
+
+// Mip selection of one query row, kept between the two fetch phases of a
+// kernel that may blend mips.
+struct MipPick {
+  int lo = 0;
+  float t = 0.0f;
 };
 
 // One axis of the tap addressing, fp32 round-to-nearest with no contraction
@@ -275,34 +280,40 @@ __device__ __forceinline__ void grid_fetch(const uint4 *pair, const GridDesc &g,
   w[3] = w11 * sc;
 }
 
-// All tap loads of one query, issued before any is consumed.  A row that is
-// not good (padding, bad set id or UV, bad bucket) fetches texel (0, 0) of
-// set 0 instead: no branch and no out-of-range address; its flag marks it.
+// All tap loads of one query from mip lo, issued before any is consumed.  A
+// row that is not good (padding, bad set id or UV, bad bucket) fetches texel
+// (0, 0) of set 0 instead: no branch and no out-of-range address; its flag
+// marks it.  TRI: the kernel may blend mips, so the mip is selected per row
+// and mip lo is weighted by 1 - t; otherwise every grid has one mip.
 template <bool TRI, bool WRAP>
 __device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grids, const ntc_query &q,
-                                           bool good, Taps<TRI> &tp) {
+                                           bool good, Taps &tp, MipPick &mp) {
   const uint32_t sid = good ? q.set_id : 0u;
   const float u = good ? q.u : 0.0f, v = good ? q.v : 0.0f;
-  // without trilinear blending (the kernel is only dispatched that way when
-  // there is one mip) the mip is always 0
-  float t = 0.0f;
-  const int lo = TRI ? select_mip(good ? q.lod : 0.0f, A.num_mips, t) : 0;
+  if (TRI) mp.lo = select_mip(good ? q.lod : 0.0f, A.num_mips, mp.t);
   const uint32_t M = TRI ? A.num_mips : 1u;
   const GridDesc *g = grids + (size_t)sid * kLevels * M;
-  const float s = TRI ? __fsub_rn(1.0f, t) : 1.0f;
+  const float s = TRI ? __fsub_rn(1.0f, mp.t) : 1.0f;
 #pragma unroll
-  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.pair, g[k * M + lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
-  if (TRI) {
-    if (t > 0.0f) {
+  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.pair, g[k * M + mp.lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
+}
+
+// The second phase of a mip blend, one level at a time (fewer registers live
+// than a whole query's taps): the taps of level k at mip lo + 1, weighted by
+// t, for the rows with t > 0 (the others load nothing and get zero weights, so
+// their accumulation is unchanged).
+template <bool WRAP>
+__device__ __forceinline__ void issue_level_hi(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                               bool good, const MipPick &mp, int k, uint4 (&raw)[4],
+                                               float (&w)[4]) {
+  if (good && mp.t > 0.0f) {
+    const uint32_t M = A.num_mips;
+    grid_fetch<WRAP>(A.pair, grids[((size_t)q.set_id * kLevels + k) * M + mp.lo + 1], q.u, q.v, mp.t, raw, w);
+  } else {
 #pragma unroll
-      for (int k = 0; k < kLevels; ++k)
-        grid_fetch<WRAP>(A.pair, g[k * M + lo + 1], u, v, t, tp.raw + 8 + 4 * k, tp.w + 8 + 4 * k);
-    } else {
-#pragma unroll
-      for (int i = 8; i < Taps<TRI>::N; ++i) {
-        tp.w[i] = 0.0f;
-        tp.raw[i] = make_uint4(0, 0, 0, 0);
-      }
+    for (int i = 0; i < 4; ++i) {
+      w[i] = 0.0f;
+      raw[i] = make_uint4(0, 0, 0, 0);
     }
   }
 }
@@ -321,22 +332,20 @@ __device__ __forceinline__ void accum_tap_x2(float2 (&acc)[4], uint4 raw, float 
   }
 }
 
-template <bool TRI, bool BF16>
-__device__ __forceinline__ void taps_to_row(const Taps<TRI> &tp, uint32_t (&packed)[8]) {
-  float2 acc[kLevels][4];
+// Feature accumulation: acc[k][c/2] over the 8 channels of level k, all taps
+// of mip lo first (FIRST: the first tap multiplies), then those of mip lo + 1.
+template <bool FIRST>
+__device__ __forceinline__ void accum_taps(const Taps &tp, float2 (&acc)[kLevels][4]) {
 #pragma unroll
   for (int k = 0; k < kLevels; ++k) {
-    accum_tap_x2<true>(acc[k], tp.raw[k * 4], tp.w[k * 4]);
+    accum_tap_x2<FIRST>(acc[k], tp.raw[k * 4], tp.w[k * 4]);
 #pragma unroll
     for (int p = 1; p < 4; ++p) accum_tap_x2<false>(acc[k], tp.raw[k * 4 + p], tp.w[k * 4 + p]);
   }
-  if (TRI && __any_sync(0xFFFFFFFFu, tp.w[8] != 0.0f || tp.w[9] != 0.0f || tp.w[10] != 0.0f ||
-                                         tp.w[11] != 0.0f)) {
-#pragma unroll
-    for (int k = 0; k < kLevels; ++k)
-#pragma unroll
-      for (int p = 0; p < 4; ++p) accum_tap_x2<false>(acc[k], tp.raw[8 + k * 4 + p], tp.w[8 + k * 4 + p]);
-  }
+}
+
+template <bool BF16>
+__device__ __forceinline__ void pack_row(const float2 (&acc)[kLevels][4], uint32_t (&packed)[8]) {
 #pragma unroll
   for (int k = 0; k < kLevels; ++k)
 #pragma unroll
@@ -531,28 +540,47 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     }
     for (; tile_of(j) < K; j += R) {
       if (*abort_flag) break;
-      // the next tile's query record and output row go in flight first
+      // the next tile's query record and output row go in flight early: before
+      // the taps, or (TRI, where registers are scarcer) once the first mip's
+      // taps are consumed
       uint32_t ndec = D, nstart = 0, nlen = 0, noi = 0;
       ntc_query nq;
-      if (tile_of(j + R) < K) {
-        walk.at(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
-        if ((uint32_t)row < nlen) {
-          nq = load_query(B.sorted + nstart + row);
-          noi = __ldg(B.perm + nstart + row);
+      auto prefetch = [&]() {
+        if (tile_of(j + R) < K) {
+          walk.at(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
+          if ((uint32_t)row < nlen) {
+            nq = load_query(B.sorted + nstart + row);
+            noi = __ldg(B.perm + nstart + row);
+          }
         }
-      }
+      };
+      if (!TRI) prefetch();
       const bool valid = (uint32_t)row < len;
       const bool good = valid && dec < D && !query_bad(A, q);
-      Taps<TRI> taps;
-      issue_taps<TRI, WRAP>(A, grids, q, good, taps);
+      Taps taps;
+      MipPick mp;
+      issue_taps<TRI, WRAP>(A, grids, q, good, taps, mp);
       // bad rows (set id out of range, non-finite UV, or the bad bucket) decode to NaN
       const bool bad = valid && !good;
       const uint32_t badm = __ballot_sync(0xFFFFFFFFu, bad);
       if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
       if (bad)
         for (uint32_t cc = 0; cc < C; ++cc) out[(size_t)oi * C + cc] = __int_as_float(0x7fc00000);
+      float2 acc[kLevels][4];
+      accum_taps<true>(taps, acc);
+      if (TRI) prefetch();
+      if (TRI && __any_sync(0xFFFFFFFFu, good && mp.t > 0.0f)) {  // some row blends two mips
+#pragma unroll
+        for (int k = 0; k < kLevels; ++k) {
+          uint4 raw[4];
+          float w[4];
+          issue_level_hi<WRAP>(A, grids, q, good, mp, k, raw, w);
+#pragma unroll
+          for (int p = 0; p < 4; ++p) accum_tap_x2<false>(acc[k], raw[p], w[p]);
+        }
+      }
       uint32_t a[8];
-      taps_to_row<TRI, BF16>(taps, a);
+      pack_row<BF16>(acc, a);
       const uint32_t s = pc * SC + j % SC, n = j / SC;
       if (!mbar_wait(empty_bar(s), (n & 1) ^ 1)) {  // the stage's previous tile has left layer 1
         atomicOr(status, 1u);
@@ -815,11 +843,11 @@ cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Bucke
     NTC_WS2(H, TRI, false, NP, NC, SC);          \
   } while (0)
   if (W.hidden == 64) {
-    if (tri) NTC_WS(64, true, 2, 2, 2);
+    if (tri) NTC_WS(64, true, 4, 4, 1);
     NTC_WS(64, false, 4, 4, 1);
   }
-  if (tri) NTC_WS(128, true, 2, 2, 2);
-  NTC_WS(128, false, 2, 2, 2);
+  if (tri) NTC_WS(128, true, 4, 2, 2);
+  NTC_WS(128, false, 4, 2, 2);
 #undef NTC_WS
 #undef NTC_WS2
 }
