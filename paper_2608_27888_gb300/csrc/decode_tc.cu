@@ -361,11 +361,20 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
 }
 
 // The tiles of one role in increasing order: the decoder index only moves
-// forward, so a lookup is a few compares instead of a binary search.
+// forward, so a lookup is a few compares instead of a binary search.  With
+// ident_n != 0 (one decoder, nothing sorted) tile t is queries 128t .. of the
+// caller's array.
 struct TileWalk {
   uint32_t d = 0;
+  uint32_t ident_n = 0;
   __device__ __forceinline__ void at(const uint32_t *seg, const uint32_t *tst, uint32_t D, uint32_t t,
                                      uint32_t &dec, uint32_t &start, uint32_t &len) {
+    if (ident_n) {
+      dec = 0;
+      start = t * kTile;
+      len = min((uint32_t)kTile, ident_n - start);
+      return;
+    }
     while (d < D && tst[d + 1] <= t) ++d;
     dec = d;
     start = seg[d] + (t - tst[d]) * kTile;
@@ -506,7 +515,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   // everything above is independent of the bucketing; the tile table is not
   pdl_wait();
   const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
-  if (D + 2 <= kSmemTileTable) {
+  if (!B.identity_n && D + 2 <= kSmemTileTable) {
     uint32_t *s_seg = reinterpret_cast<uint32_t *>(smem + M::tiles);
     uint32_t *s_tst = s_seg + kSmemTileTable;
     for (uint32_t i = threadIdx.x; i < D + 2; i += blockDim.x) {
@@ -519,7 +528,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   fence_before();
   __syncthreads();
   fence_after();
-  const uint32_t T = __ldg(B.meta);
+  const uint32_t T = B.identity_n ? (B.identity_n + kTile - 1) / kTile : __ldg(B.meta);
   const uint32_t grid = gridDim.x;
   const uint32_t K = blockIdx.x < T ? (T - blockIdx.x + grid - 1) / grid : 0;  // local tiles
 
@@ -531,11 +540,12 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     uint32_t dec = D, start = 0, len = 0, oi = 0;
     ntc_query q;
     TileWalk walk;
+    walk.ident_n = B.identity_n;
     if (tile_of(j) < K) {
       walk.at(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
       if ((uint32_t)row < len) {
         q = load_query(B.sorted + start + row);
-        oi = __ldg(B.perm + start + row);
+        oi = B.identity_n ? start + row : __ldg(B.perm + start + row);
       }
     }
     for (; tile_of(j) < K; j += R) {
@@ -550,7 +560,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
           walk.at(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
           if ((uint32_t)row < nlen) {
             nq = load_query(B.sorted + nstart + row);
-            noi = __ldg(B.perm + nstart + row);
+            noi = B.identity_n ? nstart + row : __ldg(B.perm + nstart + row);
           }
         }
       };
@@ -610,6 +620,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
     uint32_t ph = 0, wph = 0, cur = 0xFFFFFFFFu;
     TileWalk cwalk;
+    cwalk.ident_n = B.identity_n;
     constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
     const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
     auto wait_bar = [&](uint32_t b, uint32_t parity) {

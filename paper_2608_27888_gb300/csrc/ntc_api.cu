@@ -374,7 +374,11 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   int launches = 0;
   cudaError_t e;
   const bool unsorted = mode == NTC_MODE_DIVERGENT || mode == NTC_MODE_DIVERGENT_FMA;
-  s = unsorted ? NTC_OK : ensure_scratch(c, n, st);
+  // one decoder shared by every set (the paper's shared decoder): there is no
+  // divergence to remove, so the tensor-core decode takes the queries in their
+  // own order and nothing is sorted
+  const bool shared = mode == NTC_MODE_BUCKETED && !fp32 && c->D == 1;
+  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
   if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
   if (unsorted) {
@@ -391,15 +395,22 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     }
     return NTC_OK;
   }
-  e = launch_bucket(A, q, n, scratch_of(c), st, &launches, c->d_status);
-  if (e != cudaSuccess) {
-    c->launches += launches;
-    return cuda_fail(e, "bucketing launch");
-  }
   Buckets B;
-  B.sorted = c->d_sorted;
-  B.perm = c->d_perm;
-  B.meta = c->d_meta;
+  if (shared) {
+    B.sorted = q;
+    B.perm = nullptr;
+    B.meta = nullptr;
+    B.identity_n = (uint32_t)n;
+  } else {
+    e = launch_bucket(A, q, n, scratch_of(c), st, &launches, c->d_status);
+    if (e != cudaSuccess) {
+      c->launches += launches;
+      return cuda_fail(e, "bucketing launch");
+    }
+    B.sorted = c->d_sorted;
+    B.perm = c->d_perm;
+    B.meta = c->d_meta;
+  }
   if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
   if (fp32)
     e = launch_decode_fp32(A, W, B, n, out, c->d_err, c->num_sms, st, &launches);

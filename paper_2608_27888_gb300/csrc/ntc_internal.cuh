@@ -73,11 +73,14 @@ inline __host__ __device__ size_t fma_image_bytes(uint32_t H, uint32_t C, uint32
   return ((size_t)H * 16 + (size_t)H * H + (size_t)H * CP) * elem + (2 * (size_t)H + CP) * 4;
 }
 
-// Bucketing results on the device.
+// Bucketing results on the device.  identity_n != 0: one decoder and no
+// sorting; `sorted` is the caller's query array itself (identity_n queries),
+// perm and meta are unused.
 struct Buckets {
   const ntc_query *sorted;  // queries in (decoder, index) order
   const uint32_t *perm;     // original index of each sorted query
   const uint32_t *meta;     // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
+  uint32_t identity_n = 0;
 };
 inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2); }
 

@@ -287,3 +287,58 @@ def test_full_size_sampled(k, variant):
     dec.close()
     del out, qd
     torch.cuda.empty_cache()
+
+
+# ------------------------------------------ single-decoder and mixed warps
+
+def _coherent_case(kind, n, rng, assets, base):
+    """Query streams of engineered warps: warps whose sets differ but share one
+    decoder, one bad set id inside an otherwise single-decoder warp, warps
+    alternating between one decoder and uniform sets, ragged tails."""
+    q = base[:n].copy()
+    S = assets.num_sets
+    m = assets.set_to_decoder
+    by_dec = {d: np.flatnonzero(m == d) for d in range(assets.num_decoders)}
+    nw = (n + 31) // 32
+    sets = np.empty(nw * 32, dtype=np.uint32)
+    for w in range(nw):
+        d = rng.integers(0, assets.num_decoders)
+        if kind == "coherent":
+            sets[32 * w:32 * w + 32] = rng.choice(by_dec[d], 32)  # one decoder, several sets
+        elif kind == "alternating":
+            sets[32 * w:32 * w + 32] = rng.choice(by_dec[d], 32) if w % 2 else rng.integers(0, S, 32)
+        elif kind == "bad_inside":
+            sets[32 * w:32 * w + 32] = rng.choice(by_dec[d], 32)
+            if w % 3 == 0:
+                sets[32 * w + rng.integers(0, 32)] = S + 5  # out of range: the warp is mixed
+        else:
+            raise ValueError(kind)
+    q["set_id"] = sets[:n]
+    return q
+
+
+@pytest.mark.parametrize("variant", ["clustered4", "shared"])
+@pytest.mark.parametrize("kind", ["coherent", "alternating", "bad_inside"])
+@pytest.mark.parametrize("n", [1, 31, 32, 33, 127, 129, 2047, 2048, 2081, 20000 + 17])
+def test_single_decoder_and_mixed_warps(kind, n, variant):
+    """With one shared decoder ("shared") the tensor-core path sorts nothing and
+    decodes the queries in their own order; with four it buckets them."""
+    base_w = small(3, variant)
+    a = base_w.assets
+    rng = np.random.default_rng(n * 7 + len(kind))
+    base = np.resize(base_w.queries, max(n, 1))
+    q = _coherent_case(kind, n, rng, a, base)
+    ref, nbad = oracle.decode(a, q)
+    dec = decoder(3, variant, "fp16")
+    dec.reset_error_count()
+    got = dec.decode(dq(q), mode="bucketed").cpu().numpy()
+    assert np.array_equal(np.isnan(got), np.isnan(ref))
+    ok = ~np.isnan(ref).any(1)
+    check_tc(got[ok], ref[ok], f"coherent {kind} n={n}")
+    assert dec.error_count() == nbad
+    # a permutation scatters the single-decoder warps into mixed ones: every
+    # row must come out bit for bit the same either way
+    p = rng.permutation(n)
+    got_p = dec.decode(dq(q[p]), mode="bucketed").cpu().numpy()
+    assert np.array_equal(got_p[ok[p]], got[p][ok[p]])
+    dec.reset_error_count()
