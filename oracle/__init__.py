@@ -21,6 +21,9 @@ What lives here:
   (number of distinct ids per block) and the score of Eq. 1 (mean |D - 1|).
 * ``speedup_percent`` -- the reading of the "average speedup" figures printed
   under Tables 5 and 6: mean over resolutions of (t_baseline / t_shared - 1).
+* ``kmeans`` -- Alg. 2 Stage 2: k-means over per-texture embeddings into m
+  groups (the set -> decoder map c(i)); Lloyd's iteration in double, written
+  out in ``ntc_oracle.c`` with the start, tie and empty-group rules it uses.
 """
 from __future__ import annotations
 
@@ -88,6 +91,9 @@ def _load():
             lib.or_features.restype = None
             lib.or_decode.argtypes = [P, P, ctypes.c_size_t, P, ctypes.c_int]
             lib.or_decode.restype = ctypes.c_uint64
+            U = ctypes.c_uint32
+            lib.or_kmeans.argtypes = [P, U, U, U, P, U, P, P]
+            lib.or_kmeans.restype = U
             _lib = lib
     return _lib
 
@@ -223,3 +229,19 @@ def speedup_percent(t_baseline, t_shared):
     tb = np.asarray(t_baseline, dtype=np.float64)
     ts = np.asarray(t_shared, dtype=np.float64)
     return float(100.0 * np.mean(tb / ts - 1.0))
+
+
+def kmeans(features, m: int, init, max_iters: int = 100):
+    """Alg. 2, Stage 2: k-means of the rows of ``features`` [n, dim] (fp32) into
+    ``m`` groups, starting from the rows ``init`` (m distinct indices).
+    Returns (map [n] uint32, centroids [m, dim] float64, assignments made)."""
+    F = np.ascontiguousarray(features, dtype=np.float32)
+    n, dim = F.shape
+    init = np.ascontiguousarray(init, dtype=np.uint32)
+    if init.shape != (m,) or len(set(init.tolist())) != m or (init >= n).any():
+        raise ValueError("init must hold m distinct row indices")
+    out = np.empty(n, dtype=np.uint32)
+    mu = np.empty((m, dim), dtype=np.float64)
+    it = _load().or_kmeans(F.ctypes.data, n, dim, m, init.ctypes.data, max_iters, out.ctypes.data,
+                           mu.ctypes.data)
+    return out, mu, int(it)

@@ -314,3 +314,60 @@ uint64_t or_decode(const or_assets *a, const or_query *q, size_t n, double *out,
   for (size_t i = 0; i < n; ++i) bad += (uint64_t)or_query_is_bad(a, &q[i]);
   return bad;
 }
+
+/* ------------------------------------------------------------------ k-means
+ * Alg. 2, Stage 2 ("Clustering into m groups", Sec. 3.3): k-means over the
+ * per-texture embeddings F [n][dim] into m groups gives the assignment c(i),
+ * i.e. the set -> decoder map.  The paper names k-means and nothing else; this
+ * is Lloyd's iteration with the following reading:
+ *   start       mu_g = F[init[g]] for g < m (the caller picks m distinct sets)
+ *   assignment  c(i) = argmin_g sum_j (F[i][j] - mu_g[j])^2, in double, the sum
+ *               taken over j in increasing order; ties go to the smallest g
+ *   update      mu_g = (sum of F[i] over c(i) = g, i increasing) / |group g|;
+ *               an empty group keeps its centroid
+ *   stop        when an assignment equals the previous one, or after max_iters
+ *               assignments
+ * Returns the number of assignments made; map[n] is the last assignment and
+ * centroids[m][dim] the means of that assignment (the last update). */
+uint32_t or_kmeans(const float *F, uint32_t n, uint32_t dim, uint32_t m, const uint32_t *init,
+                   uint32_t max_iters, uint32_t *map, double *centroids) {
+  double *mu = centroids;
+  for (uint32_t g = 0; g < m; ++g)
+    for (uint32_t j = 0; j < dim; ++j) mu[(size_t)g * dim + j] = (double)F[(size_t)init[g] * dim + j];
+  for (uint32_t i = 0; i < n; ++i) map[i] = 0xFFFFFFFFu;
+  uint32_t t = 0;
+  while (t < max_iters) {
+    ++t;
+    int changed = 0;
+    for (uint32_t i = 0; i < n; ++i) {
+      uint32_t best = 0;
+      double best_d = 0.0;
+      for (uint32_t g = 0; g < m; ++g) {
+        double dist = 0.0;
+        for (uint32_t j = 0; j < dim; ++j) {
+          const double d = (double)F[(size_t)i * dim + j] - mu[(size_t)g * dim + j];
+          dist = dist + d * d;
+        }
+        if (g == 0 || dist < best_d) {
+          best = g;
+          best_d = dist;
+        }
+      }
+      if (map[i] != best) changed = 1;
+      map[i] = best;
+    }
+    if (!changed) break;
+    for (uint32_t g = 0; g < m; ++g) {
+      uint64_t count = 0;
+      for (uint32_t i = 0; i < n; ++i) count += map[i] == g;
+      if (count == 0) continue;
+      for (uint32_t j = 0; j < dim; ++j) {
+        double s = 0.0;
+        for (uint32_t i = 0; i < n; ++i)
+          if (map[i] == g) s = s + (double)F[(size_t)i * dim + j];
+        mu[(size_t)g * dim + j] = s / (double)count;
+      }
+    }
+  }
+  return t;
+}

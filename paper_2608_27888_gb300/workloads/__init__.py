@@ -163,6 +163,53 @@ def map_random_partition(seed, num_sets, num_decoders, tag=0):
     return m
 
 
+# Textures per category of the paper's 586-texture evaluation set (Table 1):
+# Aerial, Brick, Concrete, Fabric, Floor, Metal, Plaster/Concrete, Rock,
+# Roofing, Terrain, Wood.
+CATEGORY_SIZES = (20, 80, 40, 37, 123, 24, 19, 50, 21, 107, 65)
+
+
+def map_category(sizes=CATEGORY_SIZES):
+    """Category grouping (Sec. 4.1, "Category"): the first sizes[0] sets go to
+    decoder 0, the next sizes[1] to decoder 1, and so on."""
+    return np.repeat(np.arange(len(sizes), dtype=np.uint32), np.asarray(sizes, dtype=np.int64))
+
+
+def map_random_sizes(seed, sizes, tag=0):
+    """Random grouping with prescribed group sizes (Sec. 4.1, "Random": the same
+    group sizes as another grouping): a seeded permutation of map_category."""
+    m = map_category(sizes)
+    p = permutation(seed, 200 + tag, len(m))
+    out = np.empty_like(m)
+    out[p] = m
+    return out
+
+
+def group_sizes(set_to_decoder, num_decoders):
+    return np.bincount(np.asarray(set_to_decoder, dtype=np.int64), minlength=num_decoders)
+
+
+def embeddings(seed, sizes, dim=512, spread=0.8):
+    """Synthetic stand-in for the per-texture CLIP image embeddings of Alg. 2
+    (Stage 1, 512-d): group g (sizes[g] sets, in map_category order) has a random
+    unit centre; each set's embedding is its centre plus isotropic noise of norm
+    about `spread`, normalised to unit length (CLIP features are compared on the
+    unit sphere).  fp32 [sum(sizes), dim]."""
+    rng = np.random.default_rng(seed)
+    k = len(sizes)
+    c = rng.standard_normal((k, dim))
+    c /= np.linalg.norm(c, axis=1, keepdims=True)
+    lab = map_category(sizes)
+    x = c[lab] + spread * rng.standard_normal((len(lab), dim)) / np.sqrt(dim)
+    x /= np.linalg.norm(x, axis=1, keepdims=True)
+    return x.astype(np.float32)
+
+
+def kmeans_init(seed, n, m, tag=0):
+    """m distinct start rows for k-means: the first m of a seeded permutation."""
+    return permutation(seed, 300 + tag, n)[:m].copy()
+
+
 def queries_uniform(seed, n, num_sets):
     q = np.empty(n, dtype=QUERY_DTYPE)
     _load().gen_queries_uniform(seed, n, num_sets, q.ctypes.data)

@@ -343,3 +343,91 @@ def test_printed_average_speedups_reproduce():
 def test_table1_category_sizes_sum_to_dataset_size():
     g = json.load(open(os.path.join(GOLD, "paper_tables.json")))
     assert sum(g["table1_category_counts"].values()) == g["table1_total"] == 586
+
+
+# ------------------------------------------ map sources (Alg. 2 Stage 2, Table 1)
+
+def test_category_and_random_maps_have_table1_group_sizes():
+    gold = json.load(open(os.path.join(GOLD, "paper_tables.json")))
+    sizes = list(gold["table1_category_counts"].values())
+    assert tuple(sizes) == W.CATEGORY_SIZES
+    cat = W.map_category()
+    assert len(cat) == gold["table1_total"]
+    assert np.array_equal(np.bincount(cat), sizes)
+    assert (np.diff(cat.astype(np.int64)) >= 0).all()  # contiguous groups in category order
+    rnd = W.map_random_sizes(W.BASE_SEED, W.CATEGORY_SIZES)
+    assert np.array_equal(np.bincount(rnd, minlength=11), sizes)
+    assert not np.array_equal(rnd, cat)
+
+
+def _blobs(seed, sizes, dim, sep):
+    rng = np.random.default_rng(seed)
+    centres = rng.standard_normal((len(sizes), dim)) * sep
+    lab = np.repeat(np.arange(len(sizes)), sizes)
+    return (centres[lab] + rng.standard_normal((len(lab), dim))).astype(np.float32), lab
+
+
+def test_kmeans_recovers_well_separated_groups():
+    F, lab = _blobs(1, [30, 12, 50, 7, 21], 16, sep=40.0)
+    init = [0, 30, 42, 92, 99]  # one start row inside each group
+    m, mu, it = oracle.kmeans(F, 5, init)
+    assert np.array_equal(m, lab)
+    assert it == 2  # the second assignment repeats the first
+    for g in range(5):
+        assert np.allclose(mu[g], F[lab == g].astype(np.float64).mean(0), rtol=0, atol=1e-12)
+
+
+def test_kmeans_result_is_a_lloyd_fixed_point():
+    rng = np.random.default_rng(7)
+    F = rng.standard_normal((300, 12)).astype(np.float32)
+    m, mu, it = oracle.kmeans(F, 9, rng.permutation(300)[:9], max_iters=500)
+    assert it < 500
+    X = F.astype(np.float64)
+    d = ((X[:, None, :] - mu[None, :, :]) ** 2).sum(-1)  # brute force, every pair
+    assert np.array_equal(m, d.argmin(1))
+    for g in range(9):
+        assert np.allclose(mu[g], X[m == g].mean(0), rtol=0, atol=1e-12)
+
+
+def test_kmeans_objective_never_increases():
+    rng = np.random.default_rng(3)
+    F = rng.standard_normal((200, 6)).astype(np.float32)
+    init = rng.permutation(200)[:7]
+    X = F.astype(np.float64)
+    prev = np.inf
+    for t in range(1, 12):
+        m, mu, _ = oracle.kmeans(F, 7, init, max_iters=t)
+        J = ((X - mu[m]) ** 2).sum()
+        assert J <= prev * (1 + 1e-12)
+        prev = J
+
+
+def test_kmeans_special_cases():
+    rng = np.random.default_rng(5)
+    F = rng.standard_normal((40, 5)).astype(np.float32)
+    m, mu, _ = oracle.kmeans(F, 1, [17])
+    assert (m == 0).all()
+    assert np.allclose(mu[0], F.astype(np.float64).mean(0), rtol=0, atol=1e-12)
+    m, mu, it = oracle.kmeans(F, 40, np.arange(40))  # every row its own group
+    assert np.array_equal(m, np.arange(40)) and it == 2  # the second assignment repeats the first
+    assert np.array_equal(mu, F.astype(np.float64))
+    # two identical start rows: every distance ties, so the first assignment
+    # puts every row in group 0 (ties go to the smaller index), and the empty
+    # group 1 keeps its centroid through the update
+    G = np.concatenate([F[:10], F[:1]])
+    m, mu, it = oracle.kmeans(G, 2, [0, 10], max_iters=1)
+    assert (m == 0).all() and it == 1
+    assert np.array_equal(mu[1], G[10].astype(np.float64))
+    assert np.allclose(mu[0], G.astype(np.float64).mean(0), rtol=0, atol=1e-12)
+
+
+def test_kmeans_matches_scikit_learn_lloyd():
+    sk = pytest.importorskip("sklearn.cluster")
+    for seed, (n, dim, m) in enumerate([(500, 8, 6), (586, 32, 11), (120, 3, 4)]):
+        F, _ = _blobs(seed, np.full(m, n // m).tolist(), dim, sep=3.0)
+        init = np.random.default_rng(seed).permutation(len(F))[:m]
+        ours, mu, _ = oracle.kmeans(F, m, init, max_iters=300)
+        km = sk.KMeans(n_clusters=m, init=F[init].astype(np.float64), n_init=1, algorithm="lloyd",
+                       max_iter=300, tol=0.0).fit(F.astype(np.float64))
+        assert np.array_equal(ours, km.labels_)
+        assert np.allclose(mu, km.cluster_centers_, rtol=0, atol=1e-9)
