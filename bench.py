@@ -66,6 +66,8 @@ def parse():
     p.add_argument("--no-sweep", action="store_true", help="skip the decoders-per-warp sweep")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     p.add_argument("--no-mirror", action="store_true", help="skip the mirror of the paper's Tables 5-6")
+    p.add_argument("--maps", action="store_true",
+                   help="also decode a 586-set workload under the five groupings of Table 2")
     p.add_argument("--configs", action="store_true",
                    help="also time every full-size workload (1-5 and their maps); adds about two minutes")
     p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
@@ -365,6 +367,8 @@ def main():
         result["paper_mirror"] = paper_mirror(ntc, torch, args.precision)
     if args.configs and rank == 0:
         result["configs"] = per_config(ntc, torch, args.precision)
+    if args.maps and rank == 0:
+        result["maps"] = map_sources(ntc, torch, args.precision)
 
     if rank == 0 and not args.no_cpu and ws == 1:
         result["cpu_baseline"] = cpu_baseline(w)
@@ -434,6 +438,47 @@ def paper_mirror(ntc, torch, precision, sizes=(512, 1024, 2048, 4096, 8192), ds=
                 r[f"{k}_us"] / r["shared_us"] for r in rs) - 1.0
     return {"rows": rows, "summary": summary,
             "what": "32 sets of 1024^2, N x N texel-centre raster, d distinct sets per warp; times in us"}
+
+
+def map_sources(ntc, torch, precision):
+    """The five groupings of the paper's accuracy study (Sec. 4.1, Table 2) as a
+    decode-throughput experiment: 586 texture sets of 1024^2 (4 mips; Table 1's
+    dataset size), a 1920x1080 G-buffer with 600 regions, decoded with one
+    decoder per set ("baseline"), one for all ("single"), k-means groups of
+    synthetic 512-d embeddings computed by ntc_kmeans_map ("clustered", 11
+    groups), a random grouping with the clustered group sizes ("random") and
+    Table 1's categories ("category")."""
+    import dataclasses
+    from paper_2608_27888_gb300 import workloads as W
+    seed = W.BASE_SEED + 50
+    S, T, m = 586, 1024, len(W.CATEGORY_SIZES)
+    F = W.embeddings(seed, W.CATEGORY_SIZES)
+    km_map, _, km_it = ntc.kmeans_map(F, m, W.kmeans_init(seed, S, m))
+    km_sizes = np.bincount(km_map, minlength=m)
+    maps = {"baseline": (W.map_identity(S), S), "single": (W.map_shared(S), 1), "clustered": (km_map, m),
+            "random": (W.map_random_sizes(seed, km_sizes), m), "category": (W.map_category(), m)}
+    base = W.make_assets(seed, S, T, 4, 1, W.map_shared(S))
+    q = W.queries_gbuffer(seed, 1920, 1080, 600, S, T, lod_mode=0)
+    qd = ntc.queries_to_device(q)
+    out = torch.empty((len(q), base.out_dim), dtype=torch.float32, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    rows = []
+    for name, (mp, D) in maps.items():
+        a = dataclasses.replace(base, num_decoders=D, set_to_decoder=np.asarray(mp, dtype=np.uint32),
+                                weights=W.make_weights(seed, D, base.in_dim, base.hidden, 2, base.out_dim))
+        dec = ntc.Decoder(a, precision)
+        dd = mean_distinct(q, a)
+        row = {"map": name, "decoders": D, "group_sizes": np.bincount(mp, minlength=D).tolist() if D <= 16 else None,
+               "mean_distinct_decoders_per_warp": dd, "divergence_score_eq1": dd - 1.0}
+        row["bucketed"] = len(q) / (time_decode(torch, dec, qd, out, "bucketed", flush, flush_rd, reps=10, warm=3) / 1e3)
+        for mode in (("divergent_fma",) if precision == "fp32" else ("divergent", "divergent_fma")):
+            row[mode] = len(q) / (time_decode(torch, dec, qd, out, mode, flush, flush_rd, reps=5, warm=1) / 1e3)
+        rows.append(row)
+        dec.close()
+        torch.cuda.empty_cache()
+    return {"rows": rows, "kmeans_assignments": km_it, "queries": len(q),
+            "what": "586 sets of 1024^2, 1920x1080 G-buffer, 600 regions; Gq/s of the whole ntc_decode"}
 
 
 def per_config(ntc, torch, precision):

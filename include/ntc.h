@@ -236,6 +236,30 @@ NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder, uint32_t 
                                      uint32_t num_decoders, const ntc_query *d_queries, size_t n,
                                      uint32_t *d_perm, ntc_query *d_sorted, void *cuda_stream);
 
+/* ---------------------------------------------------------- map sources
+ *
+ * The clustered set -> decoder map of Alg. 2, Stage 2 (Sec. 3.3, "Clustering
+ * into m groups"): k-means of the per-set embeddings (the paper uses 512-d CLIP
+ * image features) into m groups; group g gets decoder g.  Lloyd's iteration in
+ * fp64 on the current CUDA device:
+ *   start       centroid g = h_features[h_init[g]] (m distinct rows < n, chosen
+ *               by the caller, e.g. from a seeded permutation);
+ *   assignment  c(i) = argmin_g sum_j (F[i][j] - mu_g[j])^2, the sum over j in
+ *               increasing order, ties to the smallest g;
+ *   update      mu_g = mean of the rows assigned to g, summed in increasing row
+ *               order; an empty group keeps its centroid;
+ *   stop        when no assignment changes, or after max_iters assignments.
+ * Every fp64 operation is rounded to nearest without contraction, in that
+ * order, so the result is reproducible bit for bit.
+ * h_features: HOST [n][dim] fp32 (finite), 1 <= n <= 2^24, 1 <= dim <= 4096;
+ * 1 <= m <= min(n, NTC_MAX_DECODERS).  Outputs (HOST, caller-owned): h_map[n]
+ * = c(i) in [0, m); h_centroids (may be NULL) [m][dim] fp64, the means of the
+ * final assignment; iters_run (may be NULL) the assignments made.
+ * Synchronous; allocates and frees its own device memory. */
+NTC_API ntc_status ntc_kmeans_map(const float *h_features, uint32_t n, uint32_t dim, uint32_t m,
+                                  const uint32_t *h_init, uint32_t max_iters, uint32_t *h_map,
+                                  double *h_centroids, uint32_t *iters_run);
+
 /* Human-readable message of the last failed call on this host thread. */
 NTC_API const char *ntc_last_error(void);
 NTC_API const char *ntc_status_string(ntc_status s);

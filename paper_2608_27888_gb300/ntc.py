@@ -28,7 +28,7 @@ MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucket
 EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps",
            "ntc_debug_features", "ntc_debug_bucket", "ntc_max_tiles", "ntc_get_error_count",
            "ntc_reset_error_count", "ntc_launch_count", "ntc_set_stage_timing", "ntc_stage_times",
-           "ntc_bucket_static", "ntc_last_error", "ntc_status_string")
+           "ntc_bucket_static", "ntc_kmeans_map", "ntc_last_error", "ntc_status_string")
 
 
 class ntc_desc(ctypes.Structure):
@@ -79,6 +79,7 @@ def _load():
         "ntc_set_stage_timing": ([P, I], I),
         "ntc_stage_times": ([P, P], I),
         "ntc_bucket_static": ([P, ctypes.c_uint32, ctypes.c_uint32, P, S, P, P, P], I),
+        "ntc_kmeans_map": ([P, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, P, ctypes.c_uint32, P, P, P], I),
         "ntc_last_error": ([], ctypes.c_char_p),
         "ntc_status_string": ([I], ctypes.c_char_p),
     }
@@ -161,6 +162,23 @@ def ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_
     """Allocation-free bucketing (no context): see include/ntc.h."""
     _check(_lib.ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm,
                                   d_sorted, stream))
+
+
+def ntc_kmeans_map(h_features, n, dim, m, h_init, max_iters, h_map, h_centroids, iters_run):
+    _check(_lib.ntc_kmeans_map(h_features, n, dim, m, h_init, max_iters, h_map, h_centroids, iters_run))
+
+
+def kmeans_map(features, m, init, max_iters=100):
+    """numpy convenience: (map [n] uint32, centroids [m, dim] float64, assignments made)."""
+    F = np.ascontiguousarray(features, dtype=np.float32)
+    n, dim = F.shape
+    init = np.ascontiguousarray(init, dtype=np.uint32)
+    out = np.empty(n, dtype=np.uint32)
+    mu = np.empty((m, dim), dtype=np.float64)
+    it = ctypes.c_uint32()
+    ntc_kmeans_map(F.ctypes.data, n, dim, m, init.ctypes.data, max_iters, out.ctypes.data, mu.ctypes.data,
+                   ctypes.byref(it))
+    return out, mu, int(it.value)
 
 
 def ntc_last_error() -> str:

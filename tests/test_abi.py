@@ -85,3 +85,29 @@ def test_descriptor_validation_before_any_device_work(lib):
         assert lib.ntc_create(ctypes.byref(desc(**bad)), ctypes.byref(ctx)) == status, bad
     keep[4][0] = 1  # map entry beyond num_decoders
     assert lib.ntc_create(ctypes.byref(desc()), ctypes.byref(ctx)) == 1
+
+
+def test_kmeans_map_validates_on_the_host():
+    import numpy as np
+    from paper_2608_27888_gb300 import ntc
+    F = np.zeros((10, 4), dtype=np.float32)
+    F[:, 0] = np.arange(10)
+    init = np.array([0, 1, 2], dtype=np.uint32)
+    out = np.empty(10, dtype=np.uint32)
+
+    def call(F=F, n=10, dim=4, m=3, init=init, iters=5, out=out):
+        return ntc._lib.ntc_kmeans_map(F.ctypes.data if F is not None else None, n, dim, m,
+                                       init.ctypes.data if init is not None else None, iters,
+                                       out.ctypes.data if out is not None else None, None, None)
+    assert call(F=None) == ntc.NTC_ERR_INVALID_ARG
+    assert call(out=None) == ntc.NTC_ERR_INVALID_ARG
+    assert call(m=11) == ntc.NTC_ERR_INVALID_ARG          # more groups than rows
+    assert call(m=0) == ntc.NTC_ERR_INVALID_ARG
+    assert call(iters=0) == ntc.NTC_ERR_INVALID_ARG
+    assert call(dim=0) == ntc.NTC_ERR_INVALID_ARG
+    assert call(init=np.array([0, 0, 2], dtype=np.uint32)) == ntc.NTC_ERR_INVALID_ARG  # duplicate start row
+    assert call(init=np.array([0, 1, 10], dtype=np.uint32)) == ntc.NTC_ERR_INVALID_ARG  # out of range
+    bad = F.copy()
+    bad[3, 2] = np.inf
+    assert call(F=bad) == ntc.NTC_ERR_INVALID_ARG
+    assert b"finite" in ntc._lib.ntc_last_error()

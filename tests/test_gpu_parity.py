@@ -342,3 +342,42 @@ def test_single_decoder_and_mixed_warps(kind, n, variant):
     got_p = dec.decode(dq(q[p]), mode="bucketed").cpu().numpy()
     assert np.array_equal(got_p[ok[p]], got[p][ok[p]])
     dec.reset_error_count()
+
+
+# ------------------------------------------------- k-means map source (Alg. 2)
+
+def _km_case(case):
+    rng = np.random.default_rng(len(case))
+    if case == "categories":  # the 586 synthetic 512-d embeddings, 11 groups
+        F = W.embeddings(W.BASE_SEED, W.CATEGORY_SIZES)
+        return F, 11, W.kmeans_init(W.BASE_SEED, len(F), 11), 100
+    if case == "many_groups":
+        F = rng.standard_normal((2000, 24)).astype(np.float32)
+        return F, 70, rng.permutation(2000)[:70], 200
+    if case == "single":
+        F = rng.standard_normal((33, 7)).astype(np.float32)
+        return F, 1, [5], 10
+    if case == "every_row":
+        F = rng.standard_normal((50, 3)).astype(np.float32)
+        return F, 50, rng.permutation(50), 10
+    if case == "dim1_ties":  # repeated values: exact distance ties
+        F = rng.integers(0, 4, (300, 1)).astype(np.float32)
+        return F, 3, [0, 1, 2] if len(set(F[:3, 0])) == 3 else rng.permutation(300)[:3], 50
+    if case == "one_iteration":
+        F = rng.standard_normal((400, 16)).astype(np.float32)
+        return F, 8, rng.permutation(400)[:8], 1
+    raise ValueError(case)
+
+
+@pytest.mark.parametrize("case", ["categories", "many_groups", "single", "every_row", "dim1_ties",
+                                  "one_iteration"])
+def test_kmeans_map_equals_oracle_bit_for_bit(case):
+    F, m, init, iters = _km_case(case)
+    init = np.asarray(init, dtype=np.uint32)
+    if len(set(init.tolist())) < m:
+        pytest.skip("start rows not distinct")
+    ref_map, ref_mu, ref_it = oracle.kmeans(F, m, init, max_iters=iters)
+    got_map, got_mu, got_it = ntc().kmeans_map(F, m, init, max_iters=iters)
+    assert got_it == ref_it
+    assert np.array_equal(got_map, ref_map)
+    assert np.array_equal(got_mu.view(np.uint64), ref_mu.view(np.uint64))
