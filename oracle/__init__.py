@@ -74,6 +74,9 @@ class _Assets(ctypes.Structure):
         ("out_dim", ctypes.c_uint32),
         ("weights", ctypes.c_void_p),
         ("set_to_decoder", ctypes.c_void_p),
+        ("pe_frequencies", ctypes.c_uint32),
+        ("activation", ctypes.c_uint32),
+        ("leaky_slope", ctypes.c_float),
     ]
 
 
@@ -121,13 +124,14 @@ class _Bound:
             a.num_sets, a.num_levels, a.num_mips, a.channels,
             dims.ctypes.data, offs.ctypes.data, lat.ctypes.data, a.address_mode,
             a.num_decoders, a.in_dim, a.hidden, a.num_hidden_layers, a.out_dim,
-            w.ctypes.data, m.ctypes.data)
+            w.ctypes.data, m.ctypes.data, getattr(a, "pe_frequencies", 0), getattr(a, "activation", 0),
+            getattr(a, "leaky_slope", 0.0))
         lib = _load()
         per = lib.or_param_count(ctypes.byref(self.s))
         if w.size != per * a.num_decoders:
             raise ValueError(f"weights hold {w.size} values, expected {per} x {a.num_decoders}")
-        if a.in_dim != a.num_levels * a.channels:
-            raise ValueError("in_dim must equal num_levels * channels")
+        if a.in_dim != a.num_levels * a.channels + 4 * getattr(a, "pe_frequencies", 0):
+            raise ValueError("in_dim must equal num_levels * channels + 4 * pe_frequencies")
 
     @property
     def ptr(self):
@@ -168,10 +172,10 @@ def taps(assets, queries):
 
 
 def features(assets, queries):
-    """MLP inputs, float64 [n][num_levels * channels] (NaN rows for bad queries)."""
+    """MLP inputs, float64 [n][in_dim] (NaN rows for bad queries)."""
     b = _Bound(assets)
     q = _queries(queries)
-    f = np.empty((q.shape[0], assets.num_levels * assets.channels), dtype=np.float64)
+    f = np.empty((q.shape[0], assets.in_dim), dtype=np.float64)
     _load().or_features(b.ptr, q.ctypes.data, q.shape[0], f.ctypes.data)
     return f
 

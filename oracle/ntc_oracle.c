@@ -31,10 +31,16 @@
  *        tap order (i0,j0), (i1,j0), (i0,j1), (i1,j1)
  *        texel index = base(s,k,m) + j*W + i
  *   4. f_k[c] = sum_taps w * L[tap][c] in double; with t > 0 the level feature
- *      is (1-t) f_k(lo) + t f_k(lo+1).  f = [f_0 | f_1 | ...].
- *   5. MLP in double: h = relu(W1 f + b1); h = relu(Wl h + bl) for each further
- *      hidden layer; o = 1 / (1 + exp(-(Wout h + bout))).  Weights are stored
- *      per decoder as W1[H][IN], b1[H], {W[H][H], b[H]}..., Wout[C][H], bout[C].
+ *      is (1-t) f_k(lo) + t f_k(lo+1).  f = [f_0 | f_1 | ... | pe].
+ *      Positional encoding (Sec. 4: the encoder output "is concatenated with
+ *      positional encoding"; its form is not given), F frequencies: with u', v'
+ *      the coordinates the taps use (wrapped into [0,1) in wrap mode, as given
+ *      in clamp mode, fp32), pe[4k..4k+3] = sin(2 pi 2^k u'), cos(2 pi 2^k u'),
+ *      sin(2 pi 2^k v'), cos(2 pi 2^k v') for k < F, in double.
+ *   5. MLP in double: h = act(W1 f + b1); h = act(Wl h + bl) for each further
+ *      hidden layer; o = 1 / (1 + exp(-(Wout h + bout))).  act is ReLU, or
+ *      LeakyReLU (Sec. 4) x > 0 ? x : slope * x.  Weights are stored per
+ *      decoder as W1[H][IN], b1[H], {W[H][H], b[H]}..., Wout[C][H], bout[C].
  */
 #include <math.h>
 #include <pthread.h>
@@ -62,6 +68,9 @@ typedef struct {
   uint32_t in_dim, hidden, num_hidden_layers, out_dim;
   const float *weights;           /* [num_decoders][params per decoder]       */
   const uint32_t *set_to_decoder; /* [num_sets]                               */
+  uint32_t pe_frequencies;        /* F: 4F positional-encoding inputs         */
+  uint32_t activation;            /* 0 = ReLU, 1 = LeakyReLU                  */
+  float leaky_slope;              /* LeakyReLU slope for x <= 0               */
 } or_assets;
 
 /* IEEE-754 binary16 -> double, written from the format's definition
@@ -155,8 +164,9 @@ static int or_query_is_bad(const or_assets *a, const or_query *q) {
   return q->set_id >= a->num_sets || !isfinite(q->u) || !isfinite(q->v);
 }
 
-/* Steps 1-4 for one query: the MLP input vector f (length num_levels*channels).
- * Returns 0 for a bad query (f untouched). */
+/* Steps 1-4 for one query: the MLP input vector f (length in_dim =
+ * num_levels*channels + 4*pe_frequencies).  Returns 0 for a bad query (f
+ * untouched). */
 static int or_features_one(const or_assets *a, const or_query *q, double *f) {
   if (or_query_is_bad(a, q)) return 0;
   float t;
@@ -180,7 +190,23 @@ static int or_features_one(const or_assets *a, const or_query *q, double *f) {
       f[k * C + c] = (nm == 2) ? (1.0 - (double)t) * acc[0][c] + (double)t * acc[1][c]
                                : acc[0][c];
   }
+  const double two_pi = 6.283185307179586476925286766559;
+  const float uw = a->address_mode == 0 ? q->u - floorf(q->u) : q->u;
+  const float vw = a->address_mode == 0 ? q->v - floorf(q->v) : q->v;
+  double *pe = f + (size_t)a->num_levels * C;
+  for (uint32_t k = 0; k < a->pe_frequencies; ++k) {
+    const double su = two_pi * ldexp((double)uw, (int)k), sv = two_pi * ldexp((double)vw, (int)k);
+    pe[4 * k + 0] = sin(su);
+    pe[4 * k + 1] = cos(su);
+    pe[4 * k + 2] = sin(sv);
+    pe[4 * k + 3] = cos(sv);
+  }
   return 1;
+}
+
+static double or_act(const or_assets *a, double x) {
+  if (x > 0.0) return x;
+  return a->activation == 1 ? (double)a->leaky_slope * x : 0.0;
 }
 
 /* Step 5: the decoder MLP in double. */
@@ -194,7 +220,7 @@ static void or_mlp(const or_assets *a, uint32_t dec, const double *f, double *o)
   for (uint32_t j = 0; j < H; ++j) {
     double acc = (double)b[j];
     for (uint32_t i = 0; i < I; ++i) acc += (double)W[(size_t)j * I + i] * f[i];
-    h[j] = acc > 0.0 ? acc : 0.0;
+    h[j] = or_act(a, acc);
   }
   p = b + H;
   /* further hidden layers */
@@ -204,7 +230,7 @@ static void or_mlp(const or_assets *a, uint32_t dec, const double *f, double *o)
     for (uint32_t j = 0; j < H; ++j) {
       double acc = (double)b[j];
       for (uint32_t i = 0; i < H; ++i) acc += (double)W[(size_t)j * H + i] * h[i];
-      g[j] = acc > 0.0 ? acc : 0.0;
+      g[j] = or_act(a, acc);
     }
     memcpy(h, g, sizeof(double) * H);
     p = b + H;
@@ -253,9 +279,9 @@ void or_taps(const or_assets *a, const or_query *q, size_t n, uint64_t *idx, flo
   }
 }
 
-/* MLP inputs of every query, f[n][num_levels*channels]; NaN rows for bad ones. */
+/* MLP inputs of every query, f[n][in_dim]; NaN rows for bad ones. */
 void or_features(const or_assets *a, const or_query *q, size_t n, double *f) {
-  const size_t F = (size_t)a->num_levels * a->channels;
+  const size_t F = a->in_dim;
   for (size_t i = 0; i < n; ++i)
     if (!or_features_one(a, &q[i], f + i * F))
       for (size_t c = 0; c < F; ++c) f[i * F + c] = NAN;
@@ -264,7 +290,7 @@ void or_features(const or_assets *a, const or_query *q, size_t n, double *f) {
 /* Decode queries [begin, end): out[i][out_dim]. */
 static void or_decode_range(const or_assets *a, const or_query *q, size_t begin,
                             size_t end, double *out) {
-  const size_t F = (size_t)a->num_levels * a->channels;
+  const size_t F = a->in_dim;
   double *f = (double *)malloc(sizeof(double) * F);
   for (size_t i = begin; i < end; ++i) {
     double *o = out + i * a->out_dim;

@@ -89,6 +89,9 @@ class Assets:
     weights: np.ndarray          # f32 [D][params]
     set_to_decoder: np.ndarray   # u32 [S]
     address_mode: int = 0        # 0 wrap, 1 clamp
+    pe_frequencies: int = 0      # F: 4F positional-encoding inputs after the latents
+    activation: int = 0          # 0 ReLU, 1 LeakyReLU
+    leaky_slope: float = 0.01    # LeakyReLU slope (the PyTorch default)
 
     @property
     def params_per_decoder(self) -> int:
@@ -246,18 +249,23 @@ def queries_gbuffer(seed, width, height, regions, num_sets, T, lod_mode=0, lod_m
 
 
 def make_assets(seed, num_sets, T, num_mips, num_decoders, set_to_decoder, hidden=64,
-                out_dim=8, layers=2, channels=8, address_mode=0):
-    """Two latent levels per set: L0 at T/2 and L1 at T/4 (square)."""
-    dims = [[(T // 2, T // 2), (T // 4, T // 4)] for _ in range(num_sets)]
+                out_dim=8, layers=2, channels=8, address_mode=0, levels=2, pe_frequencies=0,
+                activation=0, leaky_slope=0.01, grid=None):
+    """Latent levels per set: two (L0 at T/2, L1 at T/4, square) or one; `grid`
+    overrides the size of a single level (the paper's 256^2 grid)."""
+    sizes = [(T // 2, T // 2), (T // 4, T // 4)][:levels] if grid is None else [(grid, grid)]
+    dims = [sizes for _ in range(num_sets)]
     dims, offs, lat = make_latents(seed, num_sets, dims, num_mips, channels)
     L = dims.shape[1]
-    w = make_weights(seed, num_decoders, L * channels, hidden, layers, out_dim)
+    in_dim = L * channels + 4 * pe_frequencies
+    w = make_weights(seed, num_decoders, in_dim, hidden, layers, out_dim)
     return Assets(num_sets=num_sets, num_levels=L, num_mips=num_mips, channels=channels,
                   level_dims=dims, latent_offsets=offs, latents=lat,
-                  num_decoders=num_decoders, in_dim=L * channels, hidden=hidden,
+                  num_decoders=num_decoders, in_dim=in_dim, hidden=hidden,
                   num_hidden_layers=layers, out_dim=out_dim, weights=w,
                   set_to_decoder=np.asarray(set_to_decoder, dtype=np.uint32),
-                  address_mode=address_mode)
+                  address_mode=address_mode, pe_frequencies=pe_frequencies,
+                  activation=activation, leaky_slope=leaky_slope)
 
 
 # --------------------------------------------------------------- named workloads

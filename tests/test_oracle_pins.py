@@ -431,3 +431,80 @@ def test_kmeans_matches_scikit_learn_lloyd():
                        max_iter=300, tol=0.0).fit(F.astype(np.float64))
         assert np.array_equal(ours, km.labels_)
         assert np.allclose(mu, km.cluster_centers_, rtol=0, atol=1e-9)
+
+
+# ------------------- paper-faithful decoder: PE, LeakyReLU, 4-channel grid, A x B
+
+def test_positional_encoding_closed_form():
+    # dyadic coordinates where sin and cos of 2 pi 2^k u are known exactly
+    a = tiny_assets([[(4, 4)]], channels=4, pe_frequencies=3)
+    rows = [(0, 0.25, 0.125, 0.0), (0, 1.25, -0.875, 0.0), (0, 0.0, 0.5, 0.0)]
+    f = oracle.features(a, queries(rows))[:, 4:].reshape(3, 3, 4)  # [query][k][sin u, cos u, sin v, cos v]
+    def expect(u, v):
+        return np.array([[np.sin(2 * np.pi * 2 ** k * u), np.cos(2 * np.pi * 2 ** k * u),
+                          np.sin(2 * np.pi * 2 ** k * v), np.cos(2 * np.pi * 2 ** k * v)] for k in range(3)])
+    # u = 0.25: sin = 1, 0, 0 and cos = 0, -1, 1 for k = 0, 1, 2 (to rounding of pi)
+    assert np.allclose(f[0], expect(0.25, 0.125), atol=1e-15)
+    assert np.allclose(f[0][:, 0], [1, 0, 0], atol=1e-15) and np.allclose(f[0][:, 1], [0, -1, 1], atol=1e-15)
+    # wrap mode encodes the wrapped coordinate: u = 1.25 -> 0.25, v = -0.875 -> 0.125
+    assert np.array_equal(f[1], f[0])
+    assert np.allclose(f[2], expect(0.0, 0.5), atol=1e-15)
+    # clamp mode encodes the coordinate as given
+    c = tiny_assets([[(4, 4)]], channels=4, pe_frequencies=3, address_mode=1)
+    fc = oracle.features(c, queries([(0, 1.25, -0.875, 0.0)]))[0, 4:].reshape(3, 4)
+    assert np.allclose(fc, expect(1.25, -0.875), atol=1e-14)
+
+
+def test_four_channel_grid_returns_texel_values_at_centres():
+    rng = np.random.default_rng(9)
+    lat = rng.standard_normal(16 * 16 * 4).astype(np.float32)
+    a = tiny_assets([[(16, 16)]], channels=4, latents=lat)
+    ij = rng.integers(0, 16, (100, 2))
+    q = queries([(0, (i + 0.5) / 16, (j + 0.5) / 16, 0.0) for i, j in ij])
+    f = oracle.features(a, q)
+    grid = np.float16(lat).astype(np.float64).reshape(16, 16, 4)
+    assert np.array_equal(f, grid[ij[:, 1], ij[:, 0]])
+
+
+def test_leaky_relu_identity_weights_closed_form():
+    rng = np.random.default_rng(4)
+    dims = [[(8, 8), (4, 4)]]
+    _, _, total = W.pyramid_layout(1, dims, 1)
+    a = tiny_assets(dims, latents=rng.standard_normal(total * 8).astype(np.float32), hidden=16,
+                    out_dim=8, activation=1, leaky_slope=0.2)
+    a.weights[:] = 0
+    W1, b1, W2, b2, W3, b3 = split_weights(a)
+    W1[:] = np.eye(16)
+    W2[:] = np.eye(16)
+    W3[:] = np.eye(8, 16)
+    q = queries([(0, float(u), float(v), 0.0) for u, v in rng.uniform(-2, 2, (300, 2))])
+    out, _ = oracle.decode(a, q)
+    f = oracle.features(a, q)[:, :8]
+    slope = float(np.float32(0.2))
+    leaky = np.where(f > 0, f, slope * slope * f)  # two hidden layers
+    assert (f < 0).any()
+    assert np.allclose(out, sigmoid(leaky), atol=1e-15)
+
+
+@pytest.mark.parametrize("hidden,layers", [(16, 1), (32, 2), (64, 2), (64, 3), (128, 4), (32, 4)])
+def test_paper_decoder_equals_dense_torch_evaluation(hidden, layers):
+    """A x B ablation shapes with the paper's decoder: 4-channel grid, positional
+    encoding, LeakyReLU; against torch.nn.functional in fp64."""
+    rng = np.random.default_rng(hidden + layers)
+    dims = [[(16, 16)]]
+    _, _, total = W.pyramid_layout(1, dims, 2)
+    a = tiny_assets(dims, num_mips=2, channels=4, latents=rng.standard_normal(total * 4).astype(np.float32),
+                    hidden=hidden, out_dim=9, layers=layers, pe_frequencies=4, activation=1, leaky_slope=0.01)
+    a.weights[:] = rng.uniform(-0.4, 0.4, a.weights.shape).astype(np.float32)
+    q = queries([(0, float(u), float(v), float(l)) for u, v, l in
+                 zip(*rng.uniform(-2, 2, (2, 400)), rng.uniform(0, 1.5, 400))])
+    out, _ = oracle.decode(a, q)
+    x = torch.from_numpy(oracle.features(a, q))
+    assert x.shape[1] == 4 + 16
+    ps = [torch.from_numpy(p.astype(np.float64)) for p in split_weights(a)]
+    h = x
+    for l in range(layers):
+        h = torch.nn.functional.leaky_relu(torch.nn.functional.linear(h, ps[2 * l], ps[2 * l + 1]),
+                                           negative_slope=float(np.float32(0.01)))
+    o = torch.sigmoid(torch.nn.functional.linear(h, ps[-2], ps[-1])).numpy()
+    assert np.allclose(out, o, atol=1e-13, rtol=0)

@@ -12,7 +12,7 @@ def half_bits(values):
 
 def tiny_assets(level_dims, num_mips=1, channels=8, latents=None, hidden=16, out_dim=4,
                 layers=2, num_decoders=1, set_to_decoder=None, weights=None, address_mode=0,
-                num_sets=1):
+                num_sets=1, pe_frequencies=0, activation=0, leaky_slope=0.01):
     """Assets with explicit latents (float array, rounded to fp16) and weights."""
     dims, offs, total = W.pyramid_layout(num_sets, level_dims, num_mips)
     L = dims.shape[1]
@@ -20,7 +20,7 @@ def tiny_assets(level_dims, num_mips=1, channels=8, latents=None, hidden=16, out
         latents = np.zeros(total * channels, dtype=np.float32)
     lat = half_bits(np.asarray(latents, dtype=np.float32).reshape(-1))
     assert lat.size == total * channels
-    in_dim = L * channels
+    in_dim = L * channels + 4 * pe_frequencies
     per = hidden * in_dim + hidden + (layers - 1) * (hidden * hidden + hidden) + out_dim * hidden + out_dim
     if weights is None:
         weights = np.zeros((num_decoders, per), dtype=np.float32)
@@ -31,7 +31,8 @@ def tiny_assets(level_dims, num_mips=1, channels=8, latents=None, hidden=16, out
                     in_dim=in_dim, hidden=hidden, num_hidden_layers=layers, out_dim=out_dim,
                     weights=np.asarray(weights, dtype=np.float32).reshape(num_decoders, per),
                     set_to_decoder=np.asarray(set_to_decoder, dtype=np.uint32),
-                    address_mode=address_mode)
+                    address_mode=address_mode, pe_frequencies=pe_frequencies,
+                    activation=activation, leaky_slope=leaky_slope)
 
 
 def queries(rows):
