@@ -107,8 +107,9 @@ typedef enum {
 typedef struct {
   uint32_t num_sets;          /* texture sets, >= 1                            */
   uint32_t num_decoders;      /* decoders (groups), 1 .. NTC_MAX_DECODERS       */
-  uint32_t latent_channels;   /* channels per latent texel; must be 8           */
-  uint32_t num_levels;        /* latent grids per set; must be 2                */
+  uint32_t latent_channels;   /* channels per latent texel: 8, or 4 (Sec. 4's
+                                 256x256x4 grid)                                */
+  uint32_t num_levels;        /* latent grids per set: 2, or 1                  */
   uint32_t num_mips;          /* mip-chain length of every grid, 1 .. 16        */
   const uint32_t *level_dims; /* [num_sets][num_levels][2]: W, H of mip 0       */
   const uint64_t *latent_offsets; /* [num_sets][num_levels][num_mips]: first
@@ -117,19 +118,40 @@ typedef struct {
                                  row-major, channel-last                       */
   const uint16_t *latents;    /* IEEE fp16 bits, [num_texels][latent_channels] */
   uint64_t num_texels;        /* length of `latents` in texels                  */
-  uint32_t in_dim;            /* = num_levels * latent_channels (16)            */
-  uint32_t hidden;            /* hidden width: 64 or 128                        */
-  uint32_t num_hidden_layers; /* must be 2 (a 3-layer MLP)                      */
+  uint32_t in_dim;            /* = num_levels * latent_channels +
+                                 4 * pe_frequencies, at most 64                 */
+  uint32_t hidden;            /* hidden width: 16, 32, 64 or 128                */
+  uint32_t num_hidden_layers; /* 1 .. 4 (an MLP of num_hidden_layers + 1 layers;
+                                 Sec. 4 uses 2, the ablation A x B sizes vary
+                                 it)                                            */
   uint32_t out_dim;           /* output channels, 1 .. 16                       */
   const float *weights;       /* [num_decoders][P], per decoder W1[hidden][in],
-                                 b1[hidden], W2[hidden][hidden], b2[hidden],
-                                 W3[out][hidden], b3[out] (row-major [out][in]);
-                                 P = hidden*(in+1) + hidden*(hidden+1) +
+                                 b1[hidden], then per further hidden layer
+                                 W[hidden][hidden], b[hidden], then
+                                 Wout[out][hidden], bout[out] (row-major
+                                 [out][in]); P = hidden*(in+1) +
+                                 (num_hidden_layers-1)*hidden*(hidden+1) +
                                  out*(hidden+1)                                 */
   const uint32_t *set_to_decoder; /* [num_sets]: c(i), each < num_decoders      */
   ntc_precision precision;
   uint32_t address_mode;      /* 0 = wrap, 1 = clamp                            */
+  uint32_t pe_frequencies;    /* F, 0 .. 8: the MLP input ends with the
+                                 positional encoding sin/cos(2 pi 2^k u'),
+                                 sin/cos(2 pi 2^k v') for k < F (u', v' the
+                                 coordinates the taps use: wrapped into [0,1)
+                                 in wrap mode); Sec. 4 concatenates the encoder
+                                 output with a positional encoding             */
+  uint32_t activation;        /* 0 = ReLU, 1 = LeakyReLU (Sec. 4)               */
+  float leaky_slope;          /* LeakyReLU slope for x <= 0 (e.g. 0.01)         */
 } ntc_desc;
+
+/* Decoder shapes.  The standard shape (2 levels x 8 channels, no encoding, 2
+ * hidden layers of 64 or 128, ReLU) runs every mode on the specialised
+ * kernels.  Every other shape ntc_create accepts (the paper's 4-channel grid
+ * with positional encoding and LeakyReLU, the A x B ablation sizes) runs the
+ * BUCKETED mode (a general tcgen05 decode over the sorted tiles for fp16/bf16,
+ * per-lane fp32 for FP32) and the DIVERGENT_FMA mode; the other modes return
+ * NTC_ERR_UNSUPPORTED. */
 
 #define NTC_MAX_DECODERS 4095u
 #define NTC_TILE_ROWS 128u
@@ -171,8 +193,9 @@ NTC_API ntc_status ntc_destroy(ntc_ctx *ctx);
 NTC_API ntc_status ntc_debug_taps(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, uint64_t *d_idx,
                           float *d_w, float *d_t, void *cuda_stream);
 
-/* The fp32 MLP input of every query, d_feat[n][in_dim] (NaN rows for bad
- * queries).  Device pointers; async. */
+/* The fp32 MLP input of every query, d_feat[n][in_dim]: the latent features
+ * of every level, then the positional encoding (NaN rows for bad queries).
+ * Device pointers; async. */
 NTC_API ntc_status ntc_debug_features(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_feat,
                               void *cuda_stream);
 

@@ -1,0 +1,405 @@
+// Decoders of a general shape (Sec. 4's decoder and the A x B sizes of its
+// MLP ablation): num_levels x channels latent features (4- or 8-channel
+// grids) concatenated with a positional encoding of F frequencies, 1..4 hidden
+// layers of width 16..128, ReLU or LeakyReLU, sigmoid output.
+//
+//   k_decode_gen_tc   bucketed 128-query tiles on tcgen05: each of the 128
+//                     threads owns one row, writes its fp16/bf16 feature row
+//                     into a tensor-memory A operand, one thread issues each
+//                     layer's MMAs (B = the decoder's weights, staged in shared
+//                     memory by one bulk copy whenever the decoder changes),
+//                     and the epilogue adds the fp32 bias, applies the
+//                     activation and writes the next layer's A operand back to
+//                     tensor memory.  Several CTAs per SM overlap each other's
+//                     gathers and MMA round trips.
+//   k_decode_gen_fma  per-lane fp32 FMAs, one query per thread (the fp32
+//                     precision's bucketed path, and every precision's
+//                     divergent-FMA mode): the same rounding rules as the
+//                     standard per-lane kernel.
+#include <math.h>
+
+#include "tcgen05.cuh"
+
+namespace ntc {
+namespace {
+
+template <bool BF16>
+__device__ __forceinline__ uint32_t pack_act(float lo, float hi, uint32_t act, float slope) {
+  if (act == 1) {
+    lo = lo > 0.0f ? lo : slope * lo;
+    hi = hi > 0.0f ? hi : slope * hi;
+    return pack<BF16>(lo, hi);
+  }
+  return pack_relu<BF16>(__float_as_uint(lo), __float_as_uint(hi));
+}
+
+__device__ __forceinline__ void count_bad_warp(bool bad, unsigned long long *err) {
+  const unsigned m = __ballot_sync(0xFFFFFFFFu, bad);
+  if (m && (threadIdx.x & 31) == __ffs(m) - 1) atomicAdd(err, (unsigned long long)__popc(m));
+}
+
+// byte offset of hidden layer l's weights (l >= 1) and of the output layer's
+__device__ __forceinline__ uint32_t gen_w_off(const GenWeights &G, uint32_t l) {
+  return G.hidden * G.k1 * 2 + (l - 1) * G.hidden * G.hidden * 2;
+}
+
+template <bool BF16>
+__global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
+                                                       unsigned long long *err, unsigned int *status,
+                                                       uint32_t tmem_cols, uint32_t img_bytes) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ uint64_t bars[2];  // [0] MMA completion, [1] weight copy
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile uint32_t abort_flag;
+  const uint32_t row = threadIdx.x, warp = row >> 5;
+  const uint32_t lanes = (warp * 32) << 16;  // this warp's TMEM lane quadrant
+  const uint32_t D = A.num_decoders, H = G.hidden, K1 = G.k1, C = G.out_dim, NL = G.layers;
+  const float *bias = reinterpret_cast<const float *>(smem + (size_t)gen_w_off(G, NL) + 16u * H * 2u);
+  const uint32_t mma_bar = saddr(&bars[0]), w_bar = saddr(&bars[1]);
+  if (row == 0) {
+    mbar_init(mma_bar, 1);
+    mbar_init(w_bar, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(saddr(&tmem_slot)),
+                 "r"(tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tAcc = tmem_slot;      // H fp32 columns
+  const uint32_t tA = tmem_slot + H;    // A operand: max(K1, H) / 2 columns
+  const uint32_t sW = saddr(smem);
+  const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
+  const uint32_t T = __ldg(B.meta);
+  uint32_t cur = 0xFFFFFFFFu, mph = 0, wph = 0;
+  auto wait = [&](uint32_t bar, uint32_t parity) {
+    if (!mbar_wait(bar, parity)) {
+      atomicOr(status, 1u);
+      abort_flag = 1;
+    }
+  };
+  for (uint32_t t = blockIdx.x; t < T; t += gridDim.x) {
+    uint32_t dec, start, len;
+    tile_info(B.meta, D, t, dec, start, len);
+    const bool valid = row < len;
+    ntc_query q;
+    uint32_t oi = 0;
+    if (valid) {
+      q = load_query(B.sorted + start + row);
+      oi = __ldg(B.perm + start + row);
+    }
+    const bool good = valid && dec < D && !query_bad(A, q);
+    const bool bad = valid && !good;
+    count_bad_warp(bad, err);
+    if (bad)
+      for (uint32_t c = 0; c < C; ++c) out[(size_t)oi * C + c] = __int_as_float(0x7fc00000);
+    if (dec >= D) continue;  // a tile of the bad bucket (CTA-uniform)
+    if (dec != cur) {
+      // every MMA of the previous tile has completed: the weights may change
+      if (row == 0) {
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(w_bar), "r"(img_bytes)
+                     : "memory");
+        asm volatile(
+            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(sW),
+            "l"(G.tc + (size_t)dec * G.tc_stride), "r"(img_bytes), "r"(w_bar)
+            : "memory");
+      }
+      wait(w_bar, wph);
+      wph ^= 1;
+      cur = dec;
+    }
+    // layer-1 A operand: this row's features, K1 columns of fp16/bf16
+    {
+      float f[kGenMaxIn];
+      if (good) gen_features(A, q, f);
+      else
+#pragma unroll
+        for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
+#pragma unroll
+      for (int kc = 0; kc < kGenMaxIn / 16; ++kc) {
+        if ((uint32_t)kc * 16 >= K1) break;
+        uint32_t p[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) p[i] = pack<BF16>(f[16 * kc + 2 * i], f[16 * kc + 2 * i + 1]);
+        tmem_st8(tA + lanes + 8 * kc, p);
+      }
+    }
+    tmem_wait_st();
+    fence_before();
+    __syncthreads();
+    if (abort_flag) break;
+    if (row == 0) {
+      fence_after();
+      const uint64_t d1 = smem_desc(sW, K1);
+      for (uint32_t kc = 0; kc < K1 / 16; ++kc) umma_ta(tAcc, tA + 8 * kc, d1 + 16 * kc, id_h, kc);
+      umma_commit(mma_bar);
+    }
+    for (uint32_t l = 0; l < NL; ++l) {
+      // hidden layer l is in the accumulator: bias, activation, next A operand
+      wait(mma_bar, mph);
+      mph ^= 1;
+      fence_after();
+      const float *bl = bias + l * H;
+      for (uint32_t c0 = 0; c0 < H; c0 += 16) {
+        uint32_t v[16];
+        tmem_ld16(tAcc + lanes + c0, v);
+        tmem_wait_ld();
+        uint32_t p[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[c0 + 2 * i],
+                                __uint_as_float(v[2 * i + 1]) + bl[c0 + 2 * i + 1], G.activation, G.slope);
+        tmem_st8(tA + lanes + c0 / 2, p);
+      }
+      tmem_wait_st();
+      fence_before();
+      __syncthreads();
+      if (abort_flag) break;
+      if (row == 0) {
+        fence_after();
+        const bool last = l + 1 == NL;
+        const uint64_t dw = smem_desc(sW + gen_w_off(G, l + 1), H);
+        for (uint32_t kc = 0; kc < H / 16; ++kc) umma_ta(tAcc, tA + 8 * kc, dw + 16 * kc, last ? id_o : id_h, kc);
+        umma_commit(mma_bar);
+      }
+    }
+    if (abort_flag) break;
+    wait(mma_bar, mph);
+    mph ^= 1;
+    fence_after();
+    uint32_t o[16];
+    tmem_ld16(tAcc + lanes, o);
+    tmem_wait_ld();
+    if (good) {
+      const float *bo = bias + NL * H;
+      float *dst = out + (size_t)oi * C;
+#pragma unroll
+      for (int c = 0; c < 16; ++c)
+        if (c < (int)C) dst[c] = 1.0f / (1.0f + expf(-(__uint_as_float(o[c]) + bo[c])));
+    }
+    fence_before();
+    __syncthreads();  // the next tile overwrites the A operand and the accumulator
+    if (abort_flag) break;
+  }
+  fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_slot), "r"(tmem_cols)
+                 : "memory");
+  }
+}
+
+template <typename T>
+struct Op;
+template <>
+struct Op<float> {
+  static __device__ __forceinline__ float ld(const float *p) { return __ldg(p); }
+  static __device__ __forceinline__ float round(float x) { return x; }
+  static __device__ __forceinline__ float cvt(float x) { return x; }
+};
+template <>
+struct Op<__half> {
+  static __device__ __forceinline__ float ld(const __half *p) { return __half2float(__ldg(p)); }
+  static __device__ __forceinline__ float round(float x) { return __half2float(__float2half_rn(x)); }
+  static __device__ __forceinline__ __half cvt(float x) { return __float2half_rn(x); }
+};
+template <>
+struct Op<__nv_bfloat16> {
+  static __device__ __forceinline__ float ld(const __nv_bfloat16 *p) { return __bfloat162float(__ldg(p)); }
+  static __device__ __forceinline__ float round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+  static __device__ __forceinline__ __nv_bfloat16 cvt(float x) { return __float2bfloat16_rn(x); }
+};
+
+__device__ __forceinline__ float act_f(float x, uint32_t act, float slope) {
+  return x > 0.0f ? x : (act == 1 ? slope * x : 0.0f);
+}
+
+// Per-lane decode of a general shape; row i is sorted[i] written to out[perm[i]]
+// (or query i itself when perm is null).
+template <typename T>
+__global__ void __launch_bounds__(128) k_decode_gen_fma(Assets A, GenWeights G, const ntc_query *qs,
+                                                        const uint32_t *perm, size_t n, float *out,
+                                                        unsigned long long *err) {
+  using E = Op<T>;
+  const uint32_t H = G.hidden, I = G.in_dim, C = G.out_dim, NL = G.layers, CP = out_pad(C);
+  const size_t wbytes = (((size_t)H * I + (size_t)(NL - 1) * H * H + (size_t)H * CP) * sizeof(T) + 15) / 16 * 16;
+  const size_t step = (size_t)gridDim.x * blockDim.x;
+  const size_t nr = (n + 31) & ~(size_t)31;  // whole warps iterate together
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nr; i += step) {
+    const bool valid = i < n;
+    ntc_query q;
+    uint32_t oi = 0;
+    bool bad = false;
+    if (valid) {
+      q = load_query(qs + i);
+      oi = perm ? __ldg(perm + i) : (uint32_t)i;
+      bad = query_bad(A, q);
+    }
+    count_bad_warp(valid && bad, err);
+    if (!valid) continue;
+    float *o_row = out + (size_t)oi * C;
+    if (bad) {
+      for (uint32_t c = 0; c < C; ++c) o_row[c] = __int_as_float(0x7fc00000);
+      continue;
+    }
+    const uint8_t *img = G.fma + (size_t)__ldg(A.map + q.set_id) * G.fma_stride;
+    const T *W = reinterpret_cast<const T *>(img);
+    const float *bias = reinterpret_cast<const float *>(img + wbytes);
+    float f[kGenMaxIn];
+    gen_features(A, q, f);
+    float h[kGenMaxHidden], g[kGenMaxHidden];
+    for (uint32_t j = 0; j < H; ++j) {
+      float acc = 0.0f;
+      for (uint32_t k = 0; k < I; ++k) acc = fmaf(E::ld(W + (size_t)j * I + k), E::round(f[k]), acc);
+      h[j] = E::round(act_f(acc + __ldg(bias + j), G.activation, G.slope));
+    }
+    const T *Wl = W + (size_t)H * I;
+    for (uint32_t l = 1; l < NL; ++l) {
+      for (uint32_t j = 0; j < H; ++j) {
+        float acc = 0.0f;
+        for (uint32_t k = 0; k < H; ++k) acc = fmaf(E::ld(Wl + (size_t)j * H + k), h[k], acc);
+        g[j] = E::round(act_f(acc + __ldg(bias + l * H + j), G.activation, G.slope));
+      }
+      for (uint32_t j = 0; j < H; ++j) h[j] = g[j];
+      Wl += (size_t)H * H;
+    }
+    const T *Wo = Wl;  // W_out^T [H][CP]
+    for (uint32_t c = 0; c < C; ++c) {
+      float acc = 0.0f;
+      for (uint32_t j = 0; j < H; ++j) acc = fmaf(E::ld(Wo + (size_t)j * CP + c), h[j], acc);
+      o_row[c] = 1.0f / (1.0f + expf(-(acc + __ldg(bias + NL * H + c))));
+    }
+  }
+}
+
+// One CTA per decoder: fp32 weights (W1, b1, {W_l, b_l}..., Wout, bout) ->
+// the tcgen05 image (if tc) and the per-lane image of type T.
+template <typename T>
+__global__ void k_pack_gen(const float *w32, GenWeights G, uint8_t *tc, uint8_t *fma) {
+  using E = Op<T>;
+  const uint32_t d = blockIdx.x, H = G.hidden, I = G.in_dim, C = G.out_dim, NL = G.layers, K1 = G.k1;
+  const uint32_t CP = out_pad(C);
+  const size_t P = (size_t)H * I + H + (size_t)(NL - 1) * (H * H + H) + (size_t)C * H + C;
+  const float *p = w32 + (size_t)d * P;
+  // source offsets of each layer
+  auto Wsrc = [&](uint32_t l) -> const float * {  // l = 0: W1; 1..NL-1: hidden; NL: output
+    return l == 0 ? p : p + (size_t)H * I + H + (size_t)(l - 1) * (H * H + H);
+  };
+  auto bsrc = [&](uint32_t l) -> const float * {
+    return l == 0 ? p + (size_t)H * I : Wsrc(l) + (size_t)(l < NL ? H : C) * H;
+  };
+  if (tc) {
+    uint8_t *img = tc + (size_t)d * G.tc_stride;
+    // W1 [H][K1]
+    for (uint32_t e = threadIdx.x; e < H * K1; e += blockDim.x) {
+      const uint32_t r = e / K1, k = e % K1;
+      const float x = k < I ? Wsrc(0)[(size_t)r * I + k] : 0.0f;
+      *reinterpret_cast<T *>(img + core_off(r, k, K1)) = E::cvt(x);
+    }
+    for (uint32_t l = 1; l <= NL; ++l) {
+      const uint32_t rows = l < NL ? H : 16;
+      uint8_t *base = img + (size_t)H * K1 * 2 + (size_t)(l - 1) * H * H * 2;
+      for (uint32_t e = threadIdx.x; e < rows * H; e += blockDim.x) {
+        const uint32_t r = e / H, k = e % H;
+        const float x = (l < NL || r < C) ? Wsrc(l)[(size_t)r * H + k] : 0.0f;
+        *reinterpret_cast<T *>(base + core_off(r, k, H)) = E::cvt(x);
+      }
+    }
+    float *b = reinterpret_cast<float *>(img + gen_tc_weight_bytes(I, H, NL));
+    for (uint32_t e = threadIdx.x; e < NL * H + 16; e += blockDim.x) {
+      const uint32_t l = e / H;
+      b[e] = l < NL ? bsrc(l)[e % H] : (e - NL * H < C ? bsrc(NL)[e - NL * H] : 0.0f);
+    }
+  }
+  T *o = reinterpret_cast<T *>(fma + (size_t)d * G.fma_stride);
+  for (uint32_t e = threadIdx.x; e < H * I; e += blockDim.x) o[e] = E::cvt(Wsrc(0)[e]);
+  T *ol = o + (size_t)H * I;
+  for (uint32_t l = 1; l < NL; ++l, ol += (size_t)H * H)
+    for (uint32_t e = threadIdx.x; e < H * H; e += blockDim.x) ol[e] = E::cvt(Wsrc(l)[e]);
+  for (uint32_t e = threadIdx.x; e < H * CP; e += blockDim.x) {
+    const uint32_t j = e / CP, c = e % CP;
+    ol[e] = E::cvt(c < C ? Wsrc(NL)[(size_t)c * H + j] : 0.0f);
+  }
+  const size_t wbytes = (((size_t)H * I + (size_t)(NL - 1) * H * H + (size_t)H * CP) * sizeof(T) + 15) / 16 * 16;
+  float *ob = reinterpret_cast<float *>(fma + (size_t)d * G.fma_stride + wbytes);
+  for (uint32_t e = threadIdx.x; e < NL * H + CP; e += blockDim.x) {
+    const uint32_t l = e / H;
+    ob[e] = l < NL ? bsrc(l)[e % H] : (e - NL * H < C ? bsrc(NL)[e - NL * H] : 0.0f);
+  }
+}
+
+uint32_t gen_tmem_cols(const GenWeights &G) {
+  const uint32_t need = G.hidden + (G.k1 > G.hidden ? G.k1 : G.hidden) / 2;
+  uint32_t c = 32;
+  while (c < need) c <<= 1;
+  return c;
+}
+
+template <bool BF16>
+cudaError_t launch_gen_tc_t(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+                            unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
+  const uint32_t img = (uint32_t)gen_tc_image_bytes(G.in_dim, G.hidden, G.layers);
+  const uint32_t cols = gen_tmem_cols(G);
+  cudaError_t e = cudaFuncSetAttribute(k_decode_gen_tc<BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)img);
+  if (e != cudaSuccess) return e;
+  int occ = 1;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_gen_tc<BF16>, 128, img);
+  if (occ < 1) occ = 1;
+  if ((uint32_t)occ > 512 / cols) occ = (int)(512 / cols);  // tensor memory: every resident CTA allocates
+  const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
+  size_t grid = (size_t)num_sms * occ;
+  if (grid > max_tiles) grid = max_tiles;
+  k_decode_gen_tc<BF16><<<(unsigned)grid, 128, img, st>>>(A, G, B, out, err, status, cols, img);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_gen_fma_t(const Assets &A, const GenWeights &G, const Buckets *B, const ntc_query *q, size_t n,
+                             float *out, unsigned long long *err, int num_sms, cudaStream_t st) {
+  int occ = 1;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_gen_fma<T>, 128, 0);
+  if (occ < 1) occ = 1;
+  const size_t blocks = (n + 127) / 128;
+  size_t grid = (size_t)num_sms * occ * 4;
+  if (grid > blocks) grid = blocks;
+  k_decode_gen_fma<T><<<(unsigned)grid, 128, 0, st>>>(A, G, B ? B->sorted : q, B ? B->perm : nullptr, n, out, err);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+                                 unsigned long long *err, unsigned int *status, bool bf16, int num_sms,
+                                 cudaStream_t st, int *launches) {
+  *launches += 1;
+  return bf16 ? launch_gen_tc_t<true>(A, G, B, n, out, err, status, num_sms, st)
+              : launch_gen_tc_t<false>(A, G, B, n, out, err, status, num_sms, st);
+}
+
+cudaError_t launch_decode_gen_fma(const Assets &A, const GenWeights &G, const Buckets *B, const ntc_query *q,
+                                  size_t n, float *out, unsigned long long *err, ntc_precision prec, int num_sms,
+                                  cudaStream_t st, int *launches) {
+  *launches += 1;
+  if (prec == NTC_PREC_FP32) return launch_gen_fma_t<float>(A, G, B, q, n, out, err, num_sms, st);
+  if (prec == NTC_PREC_TC_BF16) return launch_gen_fma_t<__nv_bfloat16>(A, G, B, q, n, out, err, num_sms, st);
+  return launch_gen_fma_t<__half>(A, G, B, q, n, out, err, num_sms, st);
+}
+
+cudaError_t launch_pack_gen(const float *w32, uint32_t D, const GenWeights &G, ntc_precision prec, uint8_t *tc,
+                            uint8_t *fma, cudaStream_t st) {
+  if (prec == NTC_PREC_FP32)
+    k_pack_gen<float><<<D, 256, 0, st>>>(w32, G, nullptr, fma);
+  else if (prec == NTC_PREC_TC_BF16)
+    k_pack_gen<__nv_bfloat16><<<D, 256, 0, st>>>(w32, G, tc, fma);
+  else
+    k_pack_gen<__half><<<D, 256, 0, st>>>(w32, G, tc, fma);
+  return cudaGetLastError();
+}
+
+}  // namespace ntc

@@ -111,9 +111,10 @@ __global__ void k_debug_taps(Assets A, const ntc_query *qs, size_t n, unsigned l
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const ntc_query q = load_query(qs + i);
-  unsigned long long *I = idx + i * kLevels * 8;
-  float *Wt = w + i * kLevels * 8;
-  for (int e = 0; e < kLevels * 8; ++e) {
+  const uint32_t L = A.num_levels;
+  unsigned long long *I = idx + i * L * 8;
+  float *Wt = w + i * L * 8;
+  for (uint32_t e = 0; e < L * 8; ++e) {
     I[e] = ~0ull;
     Wt[e] = 0.0f;
   }
@@ -122,8 +123,8 @@ __global__ void k_debug_taps(Assets A, const ntc_query *qs, size_t n, unsigned l
   float t;
   const int lo = select_mip(q.lod, A.num_mips, t);
   t_out[i] = t;
-  const GridDesc *g = A.grids + (size_t)q.set_id * kLevels * A.num_mips;
-  for (int k = 0; k < kLevels; ++k) {
+  const GridDesc *g = A.grids + (size_t)q.set_id * L * A.num_mips;
+  for (uint32_t k = 0; k < L; ++k) {
     unsigned long long ix[4];
     float wt[4];
     grid_taps(g[k * A.num_mips + lo], q.u, q.v, A.address_mode, ix, wt);
@@ -141,17 +142,29 @@ __global__ void k_debug_taps(Assets A, const ntc_query *qs, size_t n, unsigned l
   }
 }
 
+// The MLP input of every query: the standard kernels' feature code for the
+// standard input (2 levels x 8 channels), the general one otherwise.
 __global__ void k_debug_features(Assets A, const ntc_query *qs, size_t n, float *f_out) {
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const ntc_query q = load_query(qs + i);
-  float f[kInDim];
+  const uint32_t in = A.num_levels * A.channels + 4 * A.pe_frequencies;
+  const bool standard = A.num_levels == kLevels && A.channels == kChannels && A.pe_frequencies == 0;
+  float f[kGenMaxIn];
   if (query_bad(A, q)) {
-    for (int c = 0; c < kInDim; ++c) f[c] = __int_as_float(0x7fc00000);
+#pragma unroll
+    for (int c = 0; c < kGenMaxIn; ++c) f[c] = __int_as_float(0x7fc00000);
+  } else if (standard) {
+    float s[kInDim];
+    query_features(A, q, s);
+#pragma unroll
+    for (int c = 0; c < kGenMaxIn; ++c) f[c] = c < kInDim ? s[c] : 0.0f;
   } else {
-    query_features(A, q, f);
+    gen_features(A, q, f);
   }
-  for (int c = 0; c < kInDim; ++c) f_out[i * kInDim + c] = f[c];
+#pragma unroll
+  for (int c = 0; c < kGenMaxIn; ++c)
+    if (c < (int)in) f_out[i * in + c] = f[c];
 }
 
 template <typename T>

@@ -20,6 +20,13 @@ struct ntc_ctx {
   int device = 0;
   int num_sms = 0;
   uint32_t S = 0, D = 0, M = 0, H = 0, C = 0, address_mode = 0;
+  // decoder shape; `general` is every shape but the standard one (2 levels x 8
+  // channels, no encoding, 2 hidden layers of 64 or 128, ReLU)
+  uint32_t L = kLevels, LC = kChannels, F = 0, NL = 2, in_dim = kInDim, act = 0;
+  float slope = 0.0f;
+  bool general = false;
+  uint8_t *d_gtc = nullptr, *d_gfma = nullptr;
+  size_t gtc_stride = 0, gfma_stride = 0;
   ntc_precision prec = NTC_PREC_TC_FP16;
   uint64_t num_texels = 0;
   uint4 *d_lat = nullptr;
@@ -104,7 +111,26 @@ Assets assets_of(const ntc_ctx *c) {
   A.num_decoders = c->D;
   A.num_mips = c->M;
   A.address_mode = c->address_mode;
+  A.num_levels = c->L;
+  A.channels = c->LC;
+  A.pe_frequencies = c->F;
   return A;
+}
+
+GenWeights gen_of(const ntc_ctx *c) {
+  GenWeights G;
+  G.tc = c->d_gtc;
+  G.tc_stride = c->gtc_stride;
+  G.fma = c->d_gfma;
+  G.fma_stride = c->gfma_stride;
+  G.in_dim = c->in_dim;
+  G.k1 = gen_k1(c->in_dim);
+  G.hidden = c->H;
+  G.layers = c->NL;
+  G.out_dim = c->C;
+  G.activation = c->act;
+  G.slope = c->slope;
+  return G;
 }
 
 WeightImages weights_of(const ntc_ctx *c) {
@@ -141,6 +167,8 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_f32);
   cudaFree(c->d_tc);
   cudaFree(c->d_fma);
+  cudaFree(c->d_gtc);
+  cudaFree(c->d_gfma);
   cudaFree(c->d_err);
   cudaFree(c->d_status);
   cudaFree(c->d_counts);
@@ -225,33 +253,42 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   if (d->num_sets < 1) return fail(NTC_ERR_INVALID_ARG, "num_sets must be >= 1");
   if (d->num_decoders < 1 || d->num_decoders > NTC_MAX_DECODERS)
     return fail(NTC_ERR_INVALID_ARG, "num_decoders must be in 1..%u", NTC_MAX_DECODERS);
-  if (d->latent_channels != kChannels)
-    return fail(NTC_ERR_UNSUPPORTED, "latent_channels must be %d", kChannels);
-  if (d->num_levels != kLevels) return fail(NTC_ERR_UNSUPPORTED, "num_levels must be %d", kLevels);
+  if (d->latent_channels != 4 && d->latent_channels != 8)
+    return fail(NTC_ERR_UNSUPPORTED, "latent_channels must be 4 or 8");
+  if (d->num_levels != 1 && d->num_levels != 2) return fail(NTC_ERR_UNSUPPORTED, "num_levels must be 1 or 2");
   if (d->num_mips < 1 || d->num_mips > kMaxMips)
     return fail(NTC_ERR_INVALID_ARG, "num_mips must be in 1..%d", kMaxMips);
-  if (d->in_dim != kInDim) return fail(NTC_ERR_INVALID_ARG, "in_dim must be num_levels * latent_channels");
-  if (d->hidden != 64 && d->hidden != 128) return fail(NTC_ERR_UNSUPPORTED, "hidden must be 64 or 128");
-  if (d->num_hidden_layers != 2) return fail(NTC_ERR_UNSUPPORTED, "num_hidden_layers must be 2");
+  if (d->pe_frequencies > (uint32_t)kGenMaxPe)
+    return fail(NTC_ERR_UNSUPPORTED, "pe_frequencies must be at most %d", kGenMaxPe);
+  if (d->in_dim != d->num_levels * d->latent_channels + 4 * d->pe_frequencies)
+    return fail(NTC_ERR_INVALID_ARG, "in_dim must be num_levels * latent_channels + 4 * pe_frequencies");
+  if (d->in_dim > (uint32_t)kGenMaxIn) return fail(NTC_ERR_UNSUPPORTED, "in_dim must be at most %d", kGenMaxIn);
+  if (d->hidden != 16 && d->hidden != 32 && d->hidden != 64 && d->hidden != 128)
+    return fail(NTC_ERR_UNSUPPORTED, "hidden must be 16, 32, 64 or 128");
+  if (d->num_hidden_layers < 1 || d->num_hidden_layers > (uint32_t)kGenMaxLayers)
+    return fail(NTC_ERR_UNSUPPORTED, "num_hidden_layers must be in 1..%d", kGenMaxLayers);
   if (d->out_dim < 1 || d->out_dim > 16) return fail(NTC_ERR_UNSUPPORTED, "out_dim must be in 1..16");
+  if (d->activation > 1) return fail(NTC_ERR_INVALID_ARG, "activation must be 0 (ReLU) or 1 (LeakyReLU)");
+  if (d->activation == 1 && !(d->leaky_slope - d->leaky_slope == 0.0f))
+    return fail(NTC_ERR_INVALID_ARG, "leaky_slope must be finite");
   if (d->precision != NTC_PREC_TC_FP16 && d->precision != NTC_PREC_TC_BF16 && d->precision != NTC_PREC_FP32)
     return fail(NTC_ERR_INVALID_ARG, "unknown precision");
   if (d->address_mode > 1) return fail(NTC_ERR_INVALID_ARG, "address_mode must be 0 (wrap) or 1 (clamp)");
   if (d->num_texels < 1) return fail(NTC_ERR_INVALID_ARG, "num_texels must be >= 1");
-  const uint32_t S = d->num_sets, M = d->num_mips;
-  std::vector<GridDesc> grids((size_t)S * kLevels * M);
+  const uint32_t S = d->num_sets, M = d->num_mips, L = d->num_levels;
+  std::vector<GridDesc> grids((size_t)S * L * M);
   for (uint32_t s = 0; s < S; ++s)
-    for (uint32_t k = 0; k < kLevels; ++k) {
-      const uint32_t W0 = d->level_dims[((size_t)s * kLevels + k) * 2];
-      const uint32_t H0 = d->level_dims[((size_t)s * kLevels + k) * 2 + 1];
+    for (uint32_t k = 0; k < L; ++k) {
+      const uint32_t W0 = d->level_dims[((size_t)s * L + k) * 2];
+      const uint32_t H0 = d->level_dims[((size_t)s * L + k) * 2 + 1];
       if (W0 < 1 || H0 < 1 || W0 > (1u << 24) || H0 > (1u << 24) || (uint64_t)W0 * H0 > 0xFFFFFFFFull)
         return fail(NTC_ERR_INVALID_ARG, "set %u level %u: bad grid size %ux%u", s, k, W0, H0);
       for (uint32_t m = 0; m < M; ++m) {
         const uint32_t W = W0 >> m ? W0 >> m : 1, H = H0 >> m ? H0 >> m : 1;
-        const uint64_t base = d->latent_offsets[((size_t)s * kLevels + k) * M + m];
+        const uint64_t base = d->latent_offsets[((size_t)s * L + k) * M + m];
         if (base > d->num_texels || (uint64_t)W * H > d->num_texels - base)
           return fail(NTC_ERR_INVALID_ARG, "set %u level %u mip %u lies outside the latents", s, k, m);
-        GridDesc &g = grids[((size_t)s * kLevels + k) * M + m];
+        GridDesc &g = grids[((size_t)s * L + k) * M + m];
         g.base = base;
         g.W = W;
         g.H = H;
@@ -275,16 +312,29 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   c->address_mode = d->address_mode;
   c->prec = d->precision;
   c->num_texels = d->num_texels;
-  const size_t P = (size_t)c->H * (kInDim + 1) + (size_t)c->H * (c->H + 1) + (size_t)c->C * (c->H + 1);
+  c->L = L;
+  c->LC = d->latent_channels;
+  c->F = d->pe_frequencies;
+  c->NL = d->num_hidden_layers;
+  c->in_dim = d->in_dim;
+  c->act = d->activation;
+  c->slope = d->activation == 1 ? d->leaky_slope : 0.0f;
+  c->general = !(c->L == kLevels && c->LC == kChannels && c->F == 0 && c->NL == 2 && c->act == 0 &&
+                 (c->H == 64 || c->H == 128));
+  const size_t P = (size_t)c->H * (c->in_dim + 1) + (size_t)(c->NL - 1) * c->H * (c->H + 1) +
+                   (size_t)c->C * (c->H + 1);
   c->mma_stride = round16(mma_image_bytes(c->H));
   c->f32_stride = (f32_image_floats(c->H, c->C) + 3) & ~(size_t)3;
   c->tc_stride = round16(tc_image_bytes(c->H));
   c->fma_stride = round16(fma_image_bytes(c->H, c->C, c->prec == NTC_PREC_FP32 ? 4u : 2u));
-  // the row-pair copy: grids back to back, built in chunks of kPairChunk texels
-  std::vector<GridDesc> pgrids(grids.size());
+  c->gtc_stride = round16(gen_tc_image_bytes(c->in_dim, c->H, c->NL));
+  c->gfma_stride = round16(gen_fma_image_bytes(c->in_dim, c->H, c->NL, c->C, c->prec == NTC_PREC_FP32 ? 4u : 2u));
+  // the row-pair copy (standard shape only): grids back to back, built in
+  // chunks of kPairChunk texels
+  std::vector<GridDesc> pgrids(c->general ? 0 : grids.size());
   std::vector<uint32_t> chunk_grid, chunk_start;
   uint64_t num_pairs = 0;
-  for (size_t g = 0; g < grids.size(); ++g) {
+  for (size_t g = 0; g < pgrids.size(); ++g) {
     pgrids[g] = grids[g];
     pgrids[g].base = num_pairs;
     const uint64_t nt = (uint64_t)grids[g].W * grids[g].H;
@@ -300,36 +350,48 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   auto step = [&](cudaError_t r) {
     if (e == cudaSuccess) e = r;
   };
-  step(cudaMalloc((void **)&c->d_lat, d->num_texels * 16));
+  const size_t lat_bytes = d->num_texels * d->latent_channels * 2;
+  step(cudaMalloc((void **)&c->d_lat, lat_bytes));
   step(cudaMalloc((void **)&c->d_grids, grids.size() * sizeof(GridDesc)));
   step(cudaMalloc((void **)&c->d_map, (size_t)S * 4));
-  step(cudaMalloc((void **)&c->d_mma, c->mma_stride * c->D));
-  step(cudaMalloc((void **)&c->d_f32, c->f32_stride * 4 * c->D));
-  step(cudaMalloc((void **)&c->d_tc, c->tc_stride * c->D));
-  step(cudaMalloc((void **)&c->d_fma, c->fma_stride * c->D));
   step(cudaMalloc((void **)&c->d_err, sizeof(unsigned long long)));
   step(cudaMalloc((void **)&c->d_status, sizeof(unsigned int)));
   step(cudaMalloc((void **)&d_w32, P * 4 * c->D));
-  step(cudaMalloc((void **)&c->d_pair, num_pairs * 32));
-  step(cudaMalloc((void **)&c->d_pgrids, pgrids.size() * sizeof(GridDesc)));
-  step(cudaMalloc((void **)&d_chunks, chunk_grid.size() * 2 * sizeof(uint32_t)));
+  if (!c->general) {
+    step(cudaMalloc((void **)&c->d_mma, c->mma_stride * c->D));
+    step(cudaMalloc((void **)&c->d_f32, c->f32_stride * 4 * c->D));
+    step(cudaMalloc((void **)&c->d_tc, c->tc_stride * c->D));
+    step(cudaMalloc((void **)&c->d_fma, c->fma_stride * c->D));
+    step(cudaMalloc((void **)&c->d_pair, num_pairs * 32));
+    step(cudaMalloc((void **)&c->d_pgrids, pgrids.size() * sizeof(GridDesc)));
+    step(cudaMalloc((void **)&d_chunks, chunk_grid.size() * 2 * sizeof(uint32_t)));
+  } else {
+    if (c->prec != NTC_PREC_FP32) step(cudaMalloc((void **)&c->d_gtc, c->gtc_stride * c->D));
+    step(cudaMalloc((void **)&c->d_gfma, c->gfma_stride * c->D));
+  }
   if (e == cudaSuccess) {
-    step(cudaMemcpy(c->d_lat, d->latents, d->num_texels * 16, cudaMemcpyHostToDevice));
+    step(cudaMemcpy(c->d_lat, d->latents, lat_bytes, cudaMemcpyHostToDevice));
     step(cudaMemcpy(c->d_grids, grids.data(), grids.size() * sizeof(GridDesc), cudaMemcpyHostToDevice));
     step(cudaMemcpy(c->d_map, d->set_to_decoder, (size_t)S * 4, cudaMemcpyHostToDevice));
     step(cudaMemcpy(d_w32, d->weights, P * 4 * c->D, cudaMemcpyHostToDevice));
-    step(cudaMemcpy(c->d_pgrids, pgrids.data(), pgrids.size() * sizeof(GridDesc), cudaMemcpyHostToDevice));
-    step(cudaMemcpy(d_chunks, chunk_grid.data(), chunk_grid.size() * sizeof(uint32_t), cudaMemcpyHostToDevice));
-    step(cudaMemcpy(d_chunks + chunk_grid.size(), chunk_start.data(), chunk_start.size() * sizeof(uint32_t),
-                    cudaMemcpyHostToDevice));
-    step(launch_build_pairs(assets_of(c), d_chunks, d_chunks + chunk_grid.size(), (uint32_t)chunk_grid.size(),
-                            c->d_pair, 0));
     step(cudaMemset(c->d_err, 0, sizeof(unsigned long long)));
     step(cudaMemset(c->d_status, 0, sizeof(unsigned int)));
-    step(cudaMemset(c->d_tc, 0, c->tc_stride * c->D));
-    step(launch_pack_weights(d_w32, c->D, c->H, c->C, c->prec == NTC_PREC_TC_BF16, c->d_mma,
-                             c->mma_stride, c->d_f32, c->f32_stride, c->d_tc, c->tc_stride, 0));
-    step(launch_pack_fma(d_w32, c->D, c->H, c->C, c->prec, c->d_fma, c->fma_stride, 0));
+    if (!c->general) {
+      step(cudaMemcpy(c->d_pgrids, pgrids.data(), pgrids.size() * sizeof(GridDesc), cudaMemcpyHostToDevice));
+      step(cudaMemcpy(d_chunks, chunk_grid.data(), chunk_grid.size() * sizeof(uint32_t), cudaMemcpyHostToDevice));
+      step(cudaMemcpy(d_chunks + chunk_grid.size(), chunk_start.data(), chunk_start.size() * sizeof(uint32_t),
+                      cudaMemcpyHostToDevice));
+      step(launch_build_pairs(assets_of(c), d_chunks, d_chunks + chunk_grid.size(), (uint32_t)chunk_grid.size(),
+                              c->d_pair, 0));
+      step(cudaMemset(c->d_tc, 0, c->tc_stride * c->D));
+      step(launch_pack_weights(d_w32, c->D, c->H, c->C, c->prec == NTC_PREC_TC_BF16, c->d_mma,
+                               c->mma_stride, c->d_f32, c->f32_stride, c->d_tc, c->tc_stride, 0));
+      step(launch_pack_fma(d_w32, c->D, c->H, c->C, c->prec, c->d_fma, c->fma_stride, 0));
+    } else {
+      if (c->d_gtc) step(cudaMemset(c->d_gtc, 0, c->gtc_stride * c->D));
+      step(cudaMemset(c->d_gfma, 0, c->gfma_stride * c->D));
+      step(launch_pack_gen(d_w32, c->D, gen_of(c), c->prec, c->d_gtc, c->d_gfma, 0));
+    }
     step(cudaDeviceSynchronize());
   }
   cudaFree(d_w32);
@@ -364,6 +426,8 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   const bool fp32 = c->prec == NTC_PREC_FP32;
   if (fp32 && mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT_FMA)
     return fail(NTC_ERR_UNSUPPORTED, "the fp32 precision has only the bucketed and divergent FMA modes");
+  if (c->general && mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT_FMA)
+    return fail(NTC_ERR_UNSUPPORTED, "this decoder shape has only the bucketed and divergent FMA modes");
   if (n == 0) return NTC_OK;
   DeviceGuard g(c->device);
   if (!g.ok) return fail(NTC_ERR_CUDA, "cannot select the context's device");
@@ -377,13 +441,15 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   // one decoder shared by every set (the paper's shared decoder): there is no
   // divergence to remove, so the tensor-core decode takes the queries in their
   // own order and nothing is sorted
-  const bool shared = mode == NTC_MODE_BUCKETED && !fp32 && c->D == 1;
+  const bool shared = mode == NTC_MODE_BUCKETED && !fp32 && !c->general && c->D == 1;
   s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
   if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
   if (unsorted) {
     if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
-    if (mode == NTC_MODE_DIVERGENT)
+    if (c->general)
+      e = launch_decode_gen_fma(A, gen_of(c), nullptr, q, n, out, c->d_err, c->prec, c->num_sms, st, &launches);
+    else if (mode == NTC_MODE_DIVERGENT)
       e = launch_decode_divergent(A, W, q, n, out, c->d_err, bf16, c->num_sms, st, &launches);
     else
       e = launch_decode_divergent_fma(A, W, q, n, out, c->d_err, c->prec, c->num_sms, st, &launches);
@@ -412,7 +478,11 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     B.meta = c->d_meta;
   }
   if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
-  if (fp32)
+  if (c->general && fp32)
+    e = launch_decode_gen_fma(A, gen_of(c), &B, nullptr, n, out, c->d_err, c->prec, c->num_sms, st, &launches);
+  else if (c->general)
+    e = launch_decode_gen_tc(A, gen_of(c), B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
+  else if (fp32)
     e = launch_decode_fp32(A, W, B, n, out, c->d_err, c->num_sms, st, &launches);
   else if (mode == NTC_MODE_BUCKETED_MMA)
     e = launch_decode_mma(A, W, B, n, out, c->d_err, bf16, c->num_sms, st, &launches);

@@ -35,6 +35,9 @@ struct Assets {
   const GridDesc *pgrids;
   const uint32_t *map;      // [num_sets] set -> decoder
   uint32_t num_sets, num_decoders, num_mips, address_mode;
+  // the decoder input (the general-shape kernels read these; the standard
+  // kernels are compiled for 2 levels x 8 channels and no encoding)
+  uint32_t num_levels = kLevels, channels = kChannels, pe_frequencies = 0;
 };
 
 // Per-decoder weight images.
@@ -71,6 +74,48 @@ inline __host__ __device__ size_t f32_image_floats(uint32_t H, uint32_t C) {
 inline __host__ __device__ size_t fma_image_bytes(uint32_t H, uint32_t C, uint32_t elem) {
   const size_t CP = out_pad(C);
   return ((size_t)H * 16 + (size_t)H * H + (size_t)H * CP) * elem + (2 * (size_t)H + CP) * 4;
+}
+
+// General decoder shapes (any shape ntc_create accepts besides the standard
+// 2 x 8 latent channels -> 2 hidden layers of 64 or 128 with ReLU): inputs of
+// num_levels x channels latents plus 4F positional-encoding values, 1..4
+// hidden layers of 16..128, ReLU or LeakyReLU.
+constexpr int kGenMaxIn = 64;      // in_dim limit
+constexpr int kGenMaxHidden = 128;
+constexpr int kGenMaxLayers = 4;   // hidden layers
+constexpr int kGenMaxPe = 8;       // encoding frequencies
+
+// Per-decoder images of a general shape.
+//  tc image (fp16/bf16 tcgen05 B operands, no-swizzle K-major core matrices):
+//    W1 [H][K1] (K1 = in_dim rounded up to 16, zero padded), W_l [H][H] for
+//    each further hidden layer, Wout [16][H] (rows >= C zero), then fp32 b1[H],
+//    b_l[H]..., bout[16].
+//  fma image (the precision's type T, row-major): W1 [H][in], W_l [H][H]...,
+//    Wout^T [H][CP], then fp32 biases as above (bout padded to CP).
+struct GenWeights {
+  const uint8_t *tc;
+  size_t tc_stride;
+  const uint8_t *fma;
+  size_t fma_stride;
+  uint32_t in_dim, k1, hidden, layers, out_dim, activation;
+  float slope;
+};
+
+inline __host__ __device__ uint32_t gen_k1(uint32_t in_dim) { return (in_dim + 15) / 16 * 16; }
+inline __host__ __device__ size_t gen_tc_weight_bytes(uint32_t in_dim, uint32_t H, uint32_t layers) {
+  return ((size_t)H * gen_k1(in_dim) + (size_t)(layers - 1) * H * H + (size_t)16 * H) * 2;
+}
+inline __host__ __device__ size_t gen_bias_floats(uint32_t H, uint32_t layers) {
+  return (size_t)layers * H + 16;
+}
+inline __host__ __device__ size_t gen_tc_image_bytes(uint32_t in_dim, uint32_t H, uint32_t layers) {
+  return gen_tc_weight_bytes(in_dim, H, layers) + gen_bias_floats(H, layers) * 4;
+}
+inline __host__ __device__ size_t gen_fma_image_bytes(uint32_t in_dim, uint32_t H, uint32_t layers, uint32_t C,
+                                                      uint32_t elem) {
+  const size_t CP = out_pad(C);
+  const size_t w = ((size_t)H * in_dim + (size_t)(layers - 1) * H * H + (size_t)H * CP) * elem;
+  return (w + 15) / 16 * 16 + ((size_t)layers * H + CP) * 4;
 }
 
 // Bucketing results on the device.  identity_n != 0: one decoder and no
@@ -206,6 +251,93 @@ __device__ __forceinline__ void query_features(const Assets &A, const ntc_query 
   }
 }
 
+// Positional encoding of one coordinate pair at input offset BASE: for k < F,
+// sin / cos of 2 pi 2^k u and of 2 pi 2^k v (u, v as the taps see them).
+template <int BASE>
+__device__ __forceinline__ void pe_features(float u, float v, uint32_t F, float (&f)[kGenMaxIn]) {
+#pragma unroll
+  for (int k = 0; k < kGenMaxPe; ++k) {
+    if (BASE + 4 * k + 3 >= kGenMaxIn) break;
+    if (k < (int)F) {
+      float su, cu, sv, cv;
+      sincospif(ldexpf(u, k + 1), &su, &cu);
+      sincospif(ldexpf(v, k + 1), &sv, &cv);
+      f[BASE + 4 * k + 0] = su;
+      f[BASE + 4 * k + 1] = cu;
+      f[BASE + 4 * k + 2] = sv;
+      f[BASE + 4 * k + 3] = cv;
+    }
+  }
+}
+
+// The latent features of level K of a good query, C channels per texel, at
+// input offset K * C; with t > 0 the two mips are blended (weights scaled by
+// 1 - t and t, as in query_features).
+template <int K, int C>
+__device__ __forceinline__ void gen_level(const Assets &A, const GridDesc *g, int lo, float t, const ntc_query &q,
+                                          float (&f)[kGenMaxIn]) {
+  const int nm = t > 0.0f ? 2 : 1;
+  for (int mi = 0; mi < nm; ++mi) {
+    unsigned long long idx[4];
+    float w[4];
+    grid_taps(g[K * A.num_mips + lo + mi], q.u, q.v, A.address_mode, idx, w);
+    const float s = nm == 1 ? 1.0f : (mi == 0 ? __fsub_rn(1.0f, t) : t);
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      const float wp = nm == 1 ? w[p] : w[p] * s;
+      if (C == 8) {
+        const uint4 raw = __ldg(A.lat + idx[p]);
+        const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const float2 x = __half22float2(h[c]);
+          f[K * C + 2 * c] = fmaf(wp, x.x, f[K * C + 2 * c]);
+          f[K * C + 2 * c + 1] = fmaf(wp, x.y, f[K * C + 2 * c + 1]);
+        }
+      } else {
+        const uint2 raw = __ldg(reinterpret_cast<const uint2 *>(A.lat) + idx[p]);
+        const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const float2 x = __half22float2(h[c]);
+          f[K * C + 2 * c] = fmaf(wp, x.x, f[K * C + 2 * c]);
+          f[K * C + 2 * c + 1] = fmaf(wp, x.y, f[K * C + 2 * c + 1]);
+        }
+      }
+    }
+  }
+}
+
+// The MLP input of a good query for a general shape: num_levels x channels
+// latent features, then the positional encoding; zero beyond in_dim.
+__device__ __forceinline__ void gen_features(const Assets &A, const ntc_query &q, float (&f)[kGenMaxIn]) {
+#pragma unroll
+  for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
+  float t;
+  const int lo = select_mip(q.lod, A.num_mips, t);
+  const GridDesc *g = A.grids + (size_t)q.set_id * A.num_levels * A.num_mips;
+  const float u = A.address_mode == 0 ? __fsub_rn(q.u, floorf(q.u)) : q.u;
+  const float v = A.address_mode == 0 ? __fsub_rn(q.v, floorf(q.v)) : q.v;
+  const uint32_t F = A.pe_frequencies;
+  if (A.channels == 8) {
+    gen_level<0, 8>(A, g, lo, t, q, f);
+    if (A.num_levels == 2) {
+      gen_level<1, 8>(A, g, lo, t, q, f);
+      pe_features<16>(u, v, F, f);
+    } else {
+      pe_features<8>(u, v, F, f);
+    }
+  } else {
+    gen_level<0, 4>(A, g, lo, t, q, f);
+    if (A.num_levels == 2) {
+      gen_level<1, 4>(A, g, lo, t, q, f);
+      pe_features<8>(u, v, F, f);
+    } else {
+      pe_features<4>(u, v, F, f);
+    }
+  }
+}
+
 __device__ __forceinline__ ntc_query load_query(const ntc_query *q) {
   uint4 r = __ldg(reinterpret_cast<const uint4 *>(q));
   ntc_query out;
@@ -264,6 +396,17 @@ cudaError_t launch_decode_divergent_fma(const Assets &A, const WeightImages &W, 
                                         int num_sms, cudaStream_t st, int *launches);
 cudaError_t launch_pack_fma(const float *w32, uint32_t D, uint32_t H, uint32_t C, ntc_precision prec,
                             uint8_t *fma, size_t fma_stride, cudaStream_t st);
+// General shapes: the tcgen05 decode over bucketed tiles, and the per-lane
+// FMA decode over the queries in bucket order (B non-null) or in their own
+// order (B null).
+cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+                                 unsigned long long *err, unsigned int *status, bool bf16, int num_sms,
+                                 cudaStream_t st, int *launches);
+cudaError_t launch_decode_gen_fma(const Assets &A, const GenWeights &G, const Buckets *B, const ntc_query *q,
+                                  size_t n, float *out, unsigned long long *err, ntc_precision prec, int num_sms,
+                                  cudaStream_t st, int *launches);
+cudaError_t launch_pack_gen(const float *w32, uint32_t D, const GenWeights &G, ntc_precision prec, uint8_t *tc,
+                            uint8_t *fma, cudaStream_t st);
 cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
                              float *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches);

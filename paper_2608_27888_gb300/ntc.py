@@ -50,6 +50,9 @@ class ntc_desc(ctypes.Structure):
         ("set_to_decoder", ctypes.c_void_p),
         ("precision", ctypes.c_int),
         ("address_mode", ctypes.c_uint32),
+        ("pe_frequencies", ctypes.c_uint32),
+        ("activation", ctypes.c_uint32),
+        ("leaky_slope", ctypes.c_float),
     ]
 
 
@@ -234,6 +237,9 @@ class Decoder:
         d.set_to_decoder = m.ctypes.data
         d.precision = PRECISIONS[precision]
         d.address_mode = assets.address_mode
+        d.pe_frequencies = getattr(assets, "pe_frequencies", 0)
+        d.activation = getattr(assets, "activation", 0)
+        d.leaky_slope = getattr(assets, "leaky_slope", 0.0)
         self.desc = d
         self.out_dim = assets.out_dim
         self.num_decoders = assets.num_decoders

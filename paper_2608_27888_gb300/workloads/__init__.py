@@ -318,6 +318,28 @@ def config(k: int, size: str = "full", variant: str | None = None) -> Workload:
     raise ValueError(f"unknown workload {k}")
 
 
+def paper_decoder(size: str = "full", hidden=64, layers=2, levels=1, channels=4, pe=4, activation=1,
+                  leaky_slope=0.01, num_sets=16, num_decoders=4, out_dim=9, trilinear=True) -> Workload:
+    """The decoder of the paper's experiments (Sec. 4): one 256x256x4 latent grid
+    per set (64^2 small) with a 4-level mip chain, its bilinear (trilinear when
+    the lod is fractional) features concatenated with a positional encoding of
+    `pe` frequencies, an MLP of `layers` hidden layers of `hidden` neurons with
+    LeakyReLU (the A x B ablation varies both), sigmoid output; the sets grouped
+    into `num_decoders` clusters.  Queries: a 1920x1080 G-buffer (240x136
+    small) with 200 (40) regions and a continuous lod in [0, 3] per region."""
+    full = size == "full"
+    seed = BASE_SEED + 40 + hidden + 7 * layers + levels + channels + pe + activation
+    grid = 256 if full else 64
+    W_, H_, R = (1920, 1080, 200) if full else (240, 136, 40)
+    m = map_random_partition(seed, num_sets, num_decoders)
+    a = make_assets(seed, num_sets, 2 * grid, 4, num_decoders, m, hidden=hidden, out_dim=out_dim,
+                    layers=layers, channels=channels, levels=levels, pe_frequencies=pe,
+                    activation=activation, leaky_slope=leaky_slope, grid=grid if levels == 1 else None)
+    q = queries_gbuffer(seed, W_, H_, R, num_sets, grid, lod_mode=1 if trilinear else 0, lod_max=3.0)
+    name = f"paper-A{hidden}xB{layers + 1}-L{levels}C{channels}F{pe}{'leaky' if activation else 'relu'}-{size}"
+    return Workload(name, a, q, {"grid": grid})
+
+
 def sweep(d: int, N: int = 4096, size: str = "full") -> Workload:
     """Controlled-divergence sweep: 32 sets of 1024^2 (128^2 small), 32 decoders,
     identity map, N x N texel-centre raster, exactly d distinct sets per warp."""

@@ -78,10 +78,14 @@ def test_descriptor_validation_before_any_device_work(lib):
             setattr(d, k, v)
         return d
     ctx = ctypes.c_void_p()
-    for bad, status in [(dict(hidden=96), 2), (dict(latent_channels=4), 2), (dict(num_levels=3), 2),
+    for bad, status in [(dict(hidden=96), 2), (dict(latent_channels=6), 2), (dict(num_levels=3), 2),
                         (dict(out_dim=17), 2), (dict(num_decoders=0), 1), (dict(num_mips=0), 1),
                         (dict(num_texels=10), 1), (dict(address_mode=2), 1), (dict(precision=9), 1),
-                        (dict(num_hidden_layers=3), 2)]:
+                        (dict(num_hidden_layers=5), 2), (dict(num_hidden_layers=0), 2),
+                        (dict(latent_channels=4), 1),          # in_dim no longer levels x channels
+                        (dict(pe_frequencies=2), 1),           # in_dim misses the 8 encoding inputs
+                        (dict(pe_frequencies=9, in_dim=52), 2), (dict(activation=2), 1),
+                        (dict(activation=1, leaky_slope=float("inf")), 1)]:
         assert lib.ntc_create(ctypes.byref(desc(**bad)), ctypes.byref(ctx)) == status, bad
     keep[4][0] = 1  # map entry beyond num_decoders
     assert lib.ntc_create(ctypes.byref(desc()), ctypes.byref(ctx)) == 1
