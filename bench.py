@@ -68,6 +68,8 @@ def parse():
     p.add_argument("--no-mirror", action="store_true", help="skip the mirror of the paper's Tables 5-6")
     p.add_argument("--maps", action="store_true",
                    help="also decode a 586-set workload under the five groupings of Table 2")
+    p.add_argument("--variants", action="store_true",
+                   help="also time Sec. 4's decoder and the A x B sizes of its MLP ablation")
     p.add_argument("--configs", action="store_true",
                    help="also time every full-size workload (1-5 and their maps); adds about two minutes")
     p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
@@ -369,6 +371,8 @@ def main():
         result["configs"] = per_config(ntc, torch, args.precision)
     if args.maps and rank == 0:
         result["maps"] = map_sources(ntc, torch, args.precision)
+    if args.variants and rank == 0:
+        result["variants"] = decoder_variants(ntc, torch, args.precision)
 
     if rank == 0 and not args.no_cpu and ws == 1:
         result["cpu_baseline"] = cpu_baseline(w)
@@ -438,6 +442,43 @@ def paper_mirror(ntc, torch, precision, sizes=(512, 1024, 2048, 4096, 8192), ds=
                 r[f"{k}_us"] / r["shared_us"] for r in rs) - 1.0
     return {"rows": rows, "summary": summary,
             "what": "32 sets of 1024^2, N x N texel-centre raster, d distinct sets per warp; times in us"}
+
+
+def decoder_variants(ntc, torch, precision):
+    """Sec. 4's decoder (one 256x256x4 grid per set with a 4-mip chain,
+    positional encoding of 4 frequencies, LeakyReLU, 64 x 3) and the A x B sizes
+    of its MLP ablation (A neurons, B layers), 16 sets in 4 clusters, on a
+    1920x1080 G-buffer with a continuous lod (trilinear).  Queries/s of the
+    whole ntc_decode (bucketed: the general tcgen05 kernel for fp16/bf16) and of
+    the per-lane FMA mode, with the HBM-bound rate of the algorithmic bytes."""
+    from paper_2608_27888_gb300 import workloads as W
+    peak, _ = peaks()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    rows = []
+    shapes = [(64, 3)] + [(a, b) for a in (32, 64, 128) for b in (2, 3, 4, 5) if (a, b) != (64, 3)]
+    for A_, B_ in shapes:
+        w = W.paper_decoder("full", hidden=A_, layers=B_ - 1)
+        a, q = w.assets, w.queries
+        n = len(q)
+        dec = ntc.Decoder(a, precision)
+        qd = ntc.queries_to_device(q)
+        out = torch.empty((n, a.out_dim), dtype=torch.float32, device="cuda")
+        tri = bool((q["lod"] != np.floor(q["lod"])).any())
+        bpq = 16 + (2 if tri else 1) * a.num_levels * 4 * a.channels * 2 + 4 * a.out_dim
+        flops = 2 * (a.in_dim * A_ + (B_ - 2) * A_ * A_ + A_ * a.out_dim)
+        row = {"A": A_, "B": B_, "in_dim": a.in_dim, "queries": n, "bytes_per_query": bpq,
+               "flops_per_query": flops, "roofline_rate": peak * 1e9 / bpq}
+        row["bucketed"] = n / (time_decode(torch, dec, qd, out, "bucketed", flush, flush_rd, reps=10, warm=3) / 1e3)
+        row["frac_of_roofline"] = row["bucketed"] / row["roofline_rate"]
+        row["divergent_fma"] = n / (time_decode(torch, dec, qd, out, "divergent_fma", flush, flush_rd, reps=3,
+                                                warm=1) / 1e3)
+        rows.append(row)
+        dec.close()
+        del qd, out
+        torch.cuda.empty_cache()
+    return {"rows": rows, "what": "16 sets of 256^2x4 (4 mips), PE 4 frequencies, LeakyReLU, 4 decoders; "
+                                  "1920x1080 G-buffer, lod in [0, 3]"}
 
 
 def map_sources(ntc, torch, precision):

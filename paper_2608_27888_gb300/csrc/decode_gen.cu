@@ -10,8 +10,9 @@
 //                     memory by one bulk copy whenever the decoder changes),
 //                     and the epilogue adds the fp32 bias, applies the
 //                     activation and writes the next layer's A operand back to
-//                     tensor memory.  Several CTAs per SM overlap each other's
-//                     gathers and MMA round trips.
+//                     tensor memory.  The next tile's rows are gathered into a
+//                     second layer-1 operand while the current tile's MMA chain
+//                     runs, and several CTAs per SM overlap each other.
 //   k_decode_gen_fma  per-lane fp32 FMAs, one query per thread (the fp32
 //                     precision's bucketed path, and every precision's
 //                     divergent-FMA mode): the same rounding rules as the
@@ -43,6 +44,19 @@ __device__ __forceinline__ uint32_t gen_w_off(const GenWeights &G, uint32_t l) {
   return G.hidden * G.k1 * 2 + (l - 1) * G.hidden * G.hidden * 2;
 }
 
+// Dynamic shared memory: the decoder image, then (when they fit) copies of the
+// tile table and of the grid table.
+constexpr uint32_t kGenTileTable = 1024;  // D + 2 entries
+constexpr uint32_t kGenGrids = 1024;      // sets x levels x mips entries
+inline __host__ __device__ size_t gen_smem_bytes(uint32_t img_bytes) {
+  return ((size_t)img_bytes + 15) / 16 * 16 + 2 * kGenTileTable * 4 + (size_t)kGenGrids * sizeof(GridDesc);
+}
+
+// Tensor memory: the accumulator (H columns), the hidden layers' A operand
+// (H / 2 columns) and two layer-1 A operands (K1 / 2 columns each): while one
+// tile's MMA chain runs, the next tile's feature rows go into the other one.
+__host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) { return H + H / 2 + K1; }
+
 template <bool BF16>
 __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
                                                        unsigned long long *err, unsigned int *status,
@@ -56,6 +70,7 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
   const uint32_t D = A.num_decoders, H = G.hidden, K1 = G.k1, C = G.out_dim, NL = G.layers;
   const float *bias = reinterpret_cast<const float *>(smem + (size_t)gen_w_off(G, NL) + 16u * H * 2u);
   const uint32_t mma_bar = saddr(&bars[0]), w_bar = saddr(&bars[1]);
+  uint8_t *tables = smem + ((size_t)img_bytes + 15) / 16 * 16;
   if (row == 0) {
     mbar_init(mma_bar, 1);
     mbar_init(w_bar, 1);
@@ -68,11 +83,30 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
   }
+  // tile and grid tables in shared memory when they fit
+  const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
+  if (D + 2 <= kGenTileTable) {
+    uint32_t *s_seg = reinterpret_cast<uint32_t *>(tables), *s_tst = s_seg + kGenTileTable;
+    for (uint32_t i = row; i < D + 2; i += blockDim.x) {
+      s_seg[i] = __ldg(seg + i);
+      s_tst[i] = __ldg(tst + i);
+    }
+    seg = s_seg;
+    tst = s_tst;
+  }
+  const GridDesc *grids = A.grids;
+  const uint32_t ngrids = A.num_sets * A.num_levels * A.num_mips;
+  if (ngrids <= kGenGrids) {
+    GridDesc *s_grids = reinterpret_cast<GridDesc *>(tables + 2 * kGenTileTable * 4);
+    for (uint32_t i = row; i < ngrids; i += blockDim.x) s_grids[i] = A.grids[i];
+    grids = s_grids;
+  }
   fence_before();
   __syncthreads();
   fence_after();
-  const uint32_t tAcc = tmem_slot;      // H fp32 columns
-  const uint32_t tA = tmem_slot + H;    // A operand: max(K1, H) / 2 columns
+  const uint32_t tAcc = tmem_slot;               // H fp32 columns
+  const uint32_t tAH = tmem_slot + H;            // hidden A operand, H / 2 columns
+  const uint32_t tA1 = tmem_slot + H + H / 2;    // two layer-1 A operands, K1 / 2 columns each
   const uint32_t sW = saddr(smem);
   const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
   const uint32_t T = __ldg(B.meta);
@@ -83,108 +117,129 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
       abort_flag = 1;
     }
   };
-  for (uint32_t t = blockIdx.x; t < T; t += gridDim.x) {
-    uint32_t dec, start, len;
-    tile_info(B.meta, D, t, dec, start, len);
-    const bool valid = row < len;
+  TileWalk walk;
+  // Tile tt's row of this thread: its query, bad-row handling, and the feature
+  // row written into layer-1 A operand `buf` (zeros for rows that are not good).
+  auto fetch = [&](uint32_t tt, uint32_t buf, uint32_t &d_, uint32_t &oi_, bool &good_) {
+    uint32_t st_, ln_;
+    walk.at(seg, tst, D, tt, d_, st_, ln_);
+    const bool valid = row < ln_;
     ntc_query q;
-    uint32_t oi = 0;
+    oi_ = 0;
     if (valid) {
-      q = load_query(B.sorted + start + row);
-      oi = __ldg(B.perm + start + row);
+      q = load_query(B.sorted + st_ + row);
+      oi_ = __ldg(B.perm + st_ + row);
     }
-    const bool good = valid && dec < D && !query_bad(A, q);
-    const bool bad = valid && !good;
+    good_ = valid && d_ < D && !query_bad(A, q);
+    const bool bad = valid && !good_;
     count_bad_warp(bad, err);
     if (bad)
-      for (uint32_t c = 0; c < C; ++c) out[(size_t)oi * C + c] = __int_as_float(0x7fc00000);
-    if (dec >= D) continue;  // a tile of the bad bucket (CTA-uniform)
-    if (dec != cur) {
-      // every MMA of the previous tile has completed: the weights may change
-      if (row == 0) {
-        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(w_bar), "r"(img_bytes)
-                     : "memory");
-        asm volatile(
-            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(sW),
-            "l"(G.tc + (size_t)dec * G.tc_stride), "r"(img_bytes), "r"(w_bar)
-            : "memory");
-      }
-      wait(w_bar, wph);
-      wph ^= 1;
-      cur = dec;
+      for (uint32_t c = 0; c < C; ++c) out[(size_t)oi_ * C + c] = __int_as_float(0x7fc00000);
+    if (d_ >= D) return;  // a tile of the bad bucket (CTA-uniform): nothing to multiply
+    float f[kGenMaxIn];
+    if (good_) gen_features(A, grids, q, f);
+    else
+#pragma unroll
+      for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
+#pragma unroll
+    for (int kc = 0; kc < kGenMaxIn / 16; ++kc) {
+      if ((uint32_t)kc * 16 >= K1) break;
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) p[i] = pack<BF16>(f[16 * kc + 2 * i], f[16 * kc + 2 * i + 1]);
+      tmem_st8(tA1 + buf * (K1 / 2) + lanes + 8 * kc, p);
     }
-    // layer-1 A operand: this row's features, K1 columns of fp16/bf16
-    {
-      float f[kGenMaxIn];
-      if (good) gen_features(A, q, f);
-      else
-#pragma unroll
-        for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
-#pragma unroll
-      for (int kc = 0; kc < kGenMaxIn / 16; ++kc) {
-        if ((uint32_t)kc * 16 >= K1) break;
-        uint32_t p[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) p[i] = pack<BF16>(f[16 * kc + 2 * i], f[16 * kc + 2 * i + 1]);
-        tmem_st8(tA + lanes + 8 * kc, p);
+  };
+  uint32_t t = blockIdx.x, buf = 0, dec = D, oi = 0;
+  bool good = false;
+  if (t < T) fetch(t, buf, dec, oi, good);
+  while (t < T) {
+    if (dec < D) {
+      if (dec != cur) {
+        // every MMA of the previous tile has completed: the weights may change
+        if (row == 0) {
+          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(w_bar), "r"(img_bytes)
+                       : "memory");
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(sW),
+              "l"(G.tc + (size_t)dec * G.tc_stride), "r"(img_bytes), "r"(w_bar)
+              : "memory");
+        }
+        wait(w_bar, wph);
+        wph ^= 1;
+        cur = dec;
       }
-    }
-    tmem_wait_st();
-    fence_before();
-    __syncthreads();
-    if (abort_flag) break;
-    if (row == 0) {
-      fence_after();
-      const uint64_t d1 = smem_desc(sW, K1);
-      for (uint32_t kc = 0; kc < K1 / 16; ++kc) umma_ta(tAcc, tA + 8 * kc, d1 + 16 * kc, id_h, kc);
-      umma_commit(mma_bar);
-    }
-    for (uint32_t l = 0; l < NL; ++l) {
-      // hidden layer l is in the accumulator: bias, activation, next A operand
-      wait(mma_bar, mph);
-      mph ^= 1;
-      fence_after();
-      const float *bl = bias + l * H;
-      for (uint32_t c0 = 0; c0 < H; c0 += 16) {
-        uint32_t v[16];
-        tmem_ld16(tAcc + lanes + c0, v);
-        tmem_wait_ld();
-        uint32_t p[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[c0 + 2 * i],
-                                __uint_as_float(v[2 * i + 1]) + bl[c0 + 2 * i + 1], G.activation, G.slope);
-        tmem_st8(tA + lanes + c0 / 2, p);
-      }
-      tmem_wait_st();
+      tmem_wait_st();  // this tile's feature rows (written by the previous fetch)
       fence_before();
       __syncthreads();
       if (abort_flag) break;
       if (row == 0) {
         fence_after();
-        const bool last = l + 1 == NL;
-        const uint64_t dw = smem_desc(sW + gen_w_off(G, l + 1), H);
-        for (uint32_t kc = 0; kc < H / 16; ++kc) umma_ta(tAcc, tA + 8 * kc, dw + 16 * kc, last ? id_o : id_h, kc);
+        const uint64_t d1 = smem_desc(sW, K1);
+        for (uint32_t kc = 0; kc < K1 / 16; ++kc)
+          umma_ta(tAcc, tA1 + buf * (K1 / 2) + 8 * kc, d1 + 16 * kc, id_h, kc);
         umma_commit(mma_bar);
       }
     }
-    if (abort_flag) break;
-    wait(mma_bar, mph);
-    mph ^= 1;
-    fence_after();
-    uint32_t o[16];
-    tmem_ld16(tAcc + lanes, o);
-    tmem_wait_ld();
-    if (good) {
-      const float *bo = bias + NL * H;
-      float *dst = out + (size_t)oi * C;
+    // the next tile's rows are gathered while this tile's MMA chain runs
+    const uint32_t tn = t + gridDim.x;
+    uint32_t ndec = D, noi = 0;
+    bool ngood = false;
+    if (tn < T) fetch(tn, buf ^ 1u, ndec, noi, ngood);
+    if (dec < D) {
+      for (uint32_t l = 0; l < NL; ++l) {
+        // hidden layer l is in the accumulator: bias, activation, next A operand
+        wait(mma_bar, mph);
+        mph ^= 1;
+        fence_after();
+        const float *bl = bias + l * H;
+        for (uint32_t c0 = 0; c0 < H; c0 += 16) {
+          uint32_t v[16];
+          tmem_ld16(tAcc + lanes + c0, v);
+          tmem_wait_ld();
+          uint32_t p[8];
 #pragma unroll
-      for (int c = 0; c < 16; ++c)
-        if (c < (int)C) dst[c] = 1.0f / (1.0f + expf(-(__uint_as_float(o[c]) + bo[c])));
+          for (int i = 0; i < 8; ++i)
+            p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[c0 + 2 * i],
+                                  __uint_as_float(v[2 * i + 1]) + bl[c0 + 2 * i + 1], G.activation, G.slope);
+          tmem_st8(tAH + lanes + c0 / 2, p);
+        }
+        tmem_wait_st();
+        fence_before();
+        __syncthreads();
+        if (abort_flag) break;
+        if (row == 0) {
+          fence_after();
+          const bool last = l + 1 == NL;
+          const uint64_t dw = smem_desc(sW + gen_w_off(G, l + 1), H);
+          for (uint32_t kc = 0; kc < H / 16; ++kc)
+            umma_ta(tAcc, tAH + 8 * kc, dw + 16 * kc, last ? id_o : id_h, kc);
+          umma_commit(mma_bar);
+        }
+      }
+      if (abort_flag) break;
+      wait(mma_bar, mph);
+      mph ^= 1;
+      fence_after();
+      uint32_t o[16];
+      tmem_ld16(tAcc + lanes, o);
+      tmem_wait_ld();
+      if (good) {
+        const float *bo = bias + NL * H;
+        float *dst = out + (size_t)oi * C;
+#pragma unroll
+        for (int c = 0; c < 16; ++c)
+          if (c < (int)C) dst[c] = 1.0f / (1.0f + expf(-(__uint_as_float(o[c]) + bo[c])));
+      }
+      fence_before();
+      __syncthreads();  // the next tile overwrites the accumulator and the hidden operand
+      if (abort_flag) break;
     }
-    fence_before();
-    __syncthreads();  // the next tile overwrites the A operand and the accumulator
-    if (abort_flag) break;
+    t = tn;
+    buf ^= 1u;
+    dec = ndec;
+    oi = noi;
+    good = ngood;
   }
   fence_before();
   __syncthreads();
@@ -252,7 +307,7 @@ __global__ void __launch_bounds__(128) k_decode_gen_fma(Assets A, GenWeights G, 
     const T *W = reinterpret_cast<const T *>(img);
     const float *bias = reinterpret_cast<const float *>(img + wbytes);
     float f[kGenMaxIn];
-    gen_features(A, q, f);
+    gen_features(A, A.grids, q, f);
     float h[kGenMaxHidden], g[kGenMaxHidden];
     for (uint32_t j = 0; j < H; ++j) {
       float acc = 0.0f;
@@ -335,7 +390,7 @@ __global__ void k_pack_gen(const float *w32, GenWeights G, uint8_t *tc, uint8_t 
 }
 
 uint32_t gen_tmem_cols(const GenWeights &G) {
-  const uint32_t need = G.hidden + (G.k1 > G.hidden ? G.k1 : G.hidden) / 2;
+  const uint32_t need = gen_tmem_need(G.hidden, G.k1);
   uint32_t c = 32;
   while (c < need) c <<= 1;
   return c;
@@ -345,17 +400,18 @@ template <bool BF16>
 cudaError_t launch_gen_tc_t(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
                             unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
   const uint32_t img = (uint32_t)gen_tc_image_bytes(G.in_dim, G.hidden, G.layers);
+  const size_t smem = gen_smem_bytes(img);
   const uint32_t cols = gen_tmem_cols(G);
-  cudaError_t e = cudaFuncSetAttribute(k_decode_gen_tc<BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)img);
+  cudaError_t e = cudaFuncSetAttribute(k_decode_gen_tc<BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   int occ = 1;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_gen_tc<BF16>, 128, img);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_gen_tc<BF16>, 128, smem);
   if (occ < 1) occ = 1;
   if ((uint32_t)occ > 512 / cols) occ = (int)(512 / cols);  // tensor memory: every resident CTA allocates
   const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms * occ;
   if (grid > max_tiles) grid = max_tiles;
-  k_decode_gen_tc<BF16><<<(unsigned)grid, 128, img, st>>>(A, G, B, out, err, status, cols, img);
+  k_decode_gen_tc<BF16><<<(unsigned)grid, 128, smem, st>>>(A, G, B, out, err, status, cols, img);
   return cudaGetLastError();
 }
 

@@ -160,7 +160,7 @@ __global__ void k_debug_features(Assets A, const ntc_query *qs, size_t n, float 
 #pragma unroll
     for (int c = 0; c < kGenMaxIn; ++c) f[c] = c < kInDim ? s[c] : 0.0f;
   } else {
-    gen_features(A, q, f);
+    gen_features(A, A.grids, q, f);
   }
 #pragma unroll
   for (int c = 0; c < kGenMaxIn; ++c)

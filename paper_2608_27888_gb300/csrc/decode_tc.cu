@@ -200,28 +200,6 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
       : "memory");
 }
 
-// The tiles of one role in increasing order: the decoder index only moves
-// forward, so a lookup is a few compares instead of a binary search.  With
-// ident_n != 0 (one decoder, nothing sorted) tile t is queries 128t .. of the
-// caller's array.
-struct TileWalk {
-  uint32_t d = 0;
-  uint32_t ident_n = 0;
-  __device__ __forceinline__ void at(const uint32_t *seg, const uint32_t *tst, uint32_t D, uint32_t t,
-                                     uint32_t &dec, uint32_t &start, uint32_t &len) {
-    if (ident_n) {
-      dec = 0;
-      start = t * kTile;
-      len = min((uint32_t)kTile, ident_n - start);
-      return;
-    }
-    while (d < D && tst[d + 1] <= t) ++d;
-    dec = d;
-    start = seg[d] + (t - tst[d]) * kTile;
-    len = min((uint32_t)kTile, seg[d + 1] - start);
-  }
-};
-
 constexpr uint32_t kSmemTileTable = 1024;  // staged when D + 2 <= this
 constexpr uint32_t kSmemGrids = 1024;      // staged when S * 2 * M <= this
 

@@ -309,13 +309,15 @@ __device__ __forceinline__ void gen_level(const Assets &A, const GridDesc *g, in
 }
 
 // The MLP input of a good query for a general shape: num_levels x channels
-// latent features, then the positional encoding; zero beyond in_dim.
-__device__ __forceinline__ void gen_features(const Assets &A, const ntc_query &q, float (&f)[kGenMaxIn]) {
+// latent features, then the positional encoding; zero beyond in_dim.  grids:
+// A.grids, or a copy of it (in shared memory).
+__device__ __forceinline__ void gen_features(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                             float (&f)[kGenMaxIn]) {
 #pragma unroll
   for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
   float t;
   const int lo = select_mip(q.lod, A.num_mips, t);
-  const GridDesc *g = A.grids + (size_t)q.set_id * A.num_levels * A.num_mips;
+  const GridDesc *g = grids + (size_t)q.set_id * A.num_levels * A.num_mips;
   const float u = A.address_mode == 0 ? __fsub_rn(q.u, floorf(q.u)) : q.u;
   const float v = A.address_mode == 0 ? __fsub_rn(q.v, floorf(q.v)) : q.v;
   const uint32_t F = A.pe_frequencies;
@@ -364,6 +366,28 @@ __device__ __forceinline__ void tile_info(const uint32_t *meta, uint32_t D, uint
   uint32_t end = __ldg(seg + lo + 1);
   len = min((uint32_t)kTile, end - start);
 }
+
+// The tiles of one role in increasing order: the decoder index only moves
+// forward, so a lookup is a few compares instead of a binary search.  With
+// ident_n != 0 (one decoder, nothing sorted) tile t is queries 128t .. of the
+// caller's array.
+struct TileWalk {
+  uint32_t d = 0;
+  uint32_t ident_n = 0;
+  __device__ __forceinline__ void at(const uint32_t *seg, const uint32_t *tst, uint32_t D, uint32_t t,
+                                     uint32_t &dec, uint32_t &start, uint32_t &len) {
+    if (ident_n) {
+      dec = 0;
+      start = t * kTile;
+      len = min((uint32_t)kTile, ident_n - start);
+      return;
+    }
+    while (d < D && tst[d + 1] <= t) ++d;
+    dec = d;
+    start = seg[d] + (t - tst[d]) * kTile;
+    len = min((uint32_t)kTile, seg[d + 1] - start);
+  }
+};
 
 // ---------------------------------------------------------------- launchers
 
