@@ -174,7 +174,7 @@ cudaError_t launch_fma_t(const Assets &A, const WeightImages &W, const ntc_query
                          unsigned long long *err, int num_sms, cudaStream_t st) {
   static int occ = -1;
   if (occ < 0) {
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_divergent_fma<H, CP, T>, 128, 0);
+    occ = resident_ctas(k_decode_divergent_fma<H, CP, T>, 128, 0);
     if (occ < 1) occ = 1;
   }
   const size_t blocks = (n + 127) / 128;

@@ -3,16 +3,16 @@
 // grids) concatenated with a positional encoding of F frequencies, 1..4 hidden
 // layers of width 16..128, ReLU or LeakyReLU, sigmoid output.
 //
-//   k_decode_gen_tc   bucketed 128-query tiles on tcgen05: each of the 128
-//                     threads owns one row, writes its fp16/bf16 feature row
-//                     into a tensor-memory A operand, one thread issues each
-//                     layer's MMAs (B = the decoder's weights, staged in shared
-//                     memory by one bulk copy whenever the decoder changes),
-//                     and the epilogue adds the fp32 bias, applies the
-//                     activation and writes the next layer's A operand back to
-//                     tensor memory.  The next tile's rows are gathered into a
-//                     second layer-1 operand while the current tile's MMA chain
-//                     runs, and several CTAs per SM overlap each other.
+//   k_decode_gen_tc   bucketed 128-query tiles on tcgen05, warp-specialised:
+//                     a producer warpgroup gathers each row's fp16/bf16
+//                     feature row into a tensor-memory ring stage; a consumer
+//                     warpgroup issues each layer's MMAs (B = the decoder's
+//                     weights, staged in shared memory by one bulk copy
+//                     whenever the decoder changes) and runs the epilogues:
+//                     fp32 bias, activation, the next layer's A operand back
+//                     into tensor memory, sigmoid and the scattered store.
+//                     The producer gathers the next tiles while the consumer
+//                     runs a tile's MMA chain; several CTAs per SM overlap.
 //   k_decode_gen_fma  per-lane fp32 FMAs, one query per thread (the fp32
 //                     precision's bucketed path, and every precision's
 //                     divergent-FMA mode): the same rounding rules as the
@@ -45,39 +45,62 @@ __device__ __forceinline__ uint32_t gen_w_off(const GenWeights &G, uint32_t l) {
 }
 
 // Dynamic shared memory: the decoder image, then (when they fit) copies of the
-// tile table and of the grid table.
+// tile table and of the grid table, then the ring's output rows.
 constexpr uint32_t kGenTileTable = 1024;  // D + 2 entries
 constexpr uint32_t kGenGrids = 1024;      // sets x levels x mips entries
+constexpr uint32_t kGenStages = 2;        // tiles between the producer and the consumer
+inline __host__ __device__ size_t gen_tables_off(uint32_t img_bytes) { return ((size_t)img_bytes + 15) / 16 * 16; }
+inline __host__ __device__ size_t gen_oidx_off(uint32_t img_bytes) {
+  return gen_tables_off(img_bytes) + 2 * kGenTileTable * 4 + (size_t)kGenGrids * sizeof(GridDesc);
+}
 inline __host__ __device__ size_t gen_smem_bytes(uint32_t img_bytes) {
-  return ((size_t)img_bytes + 15) / 16 * 16 + 2 * kGenTileTable * 4 + (size_t)kGenGrids * sizeof(GridDesc);
+  return gen_oidx_off(img_bytes) + (size_t)kGenStages * 128 * 4;
 }
 
 // Tensor memory: the accumulator (H columns), the hidden layers' A operand
-// (H / 2 columns) and two layer-1 A operands (K1 / 2 columns each): while one
-// tile's MMA chain runs, the next tile's feature rows go into the other one.
-__host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) { return H + H / 2 + K1; }
+// (H / 2 columns) and the ring's layer-1 A operands (K1 / 2 columns each).
+__host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) {
+  return H + H / 2 + kGenStages * (K1 / 2);
+}
 
-template <bool BF16>
-__global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
+// Warp-specialised: warpgroup 0 produces, warpgroup 1 consumes.  The CTA's
+// tiles are t_j = blockIdx.x + j * gridDim.x; tile j goes through ring stage
+// j mod kGenStages.  Producer thread r gathers row r of tile j into the stage's
+// A operand (TMEM lane r) and its output row into oidx; each producer warp
+// arrives on full[s].  The consumer's thread 0 issues layer 1 from the stage
+// (its completion empties the stage) and every further layer from the hidden
+// operand; consumer thread r runs row r's epilogues.
+template <bool BF16, int L, int C>
+__global__ void __launch_bounds__(256, 2) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
                                                        unsigned long long *err, unsigned int *status,
                                                        uint32_t tmem_cols, uint32_t img_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ uint64_t bars[2];  // [0] MMA completion, [1] weight copy
+  __shared__ uint64_t bars[2 * kGenStages + 2];  // full[S], empty[S], MMA completion, weight copy
   __shared__ uint32_t tmem_slot;
   __shared__ volatile uint32_t abort_flag;
-  const uint32_t row = threadIdx.x, warp = row >> 5;
-  const uint32_t lanes = (warp * 32) << 16;  // this warp's TMEM lane quadrant
-  const uint32_t D = A.num_decoders, H = G.hidden, K1 = G.k1, C = G.out_dim, NL = G.layers;
+  const uint32_t tid = threadIdx.x, row = tid & 127, wg = tid >> 7;
+  const uint32_t lanes = ((row >> 5) * 32) << 16;  // this warp's TMEM lane quadrant
+  constexpr int NF = L * C + 4 * kGenMaxPe;  // feature values this input layout can have
+  constexpr int NP = (NF + 15) / 16 * 16;
+  const uint32_t D = A.num_decoders, H = G.hidden, K1 = G.k1, NL = G.layers;
+  const uint32_t OC = G.out_dim;
   const float *bias = reinterpret_cast<const float *>(smem + (size_t)gen_w_off(G, NL) + 16u * H * 2u);
-  const uint32_t mma_bar = saddr(&bars[0]), w_bar = saddr(&bars[1]);
-  uint8_t *tables = smem + ((size_t)img_bytes + 15) / 16 * 16;
-  if (row == 0) {
+  uint8_t *tables = smem + gen_tables_off(img_bytes);
+  uint32_t *oidx = reinterpret_cast<uint32_t *>(smem + gen_oidx_off(img_bytes));
+  auto full_bar = [&](uint32_t s) { return saddr(&bars[s]); };
+  auto empty_bar = [&](uint32_t s) { return saddr(&bars[kGenStages + s]); };
+  const uint32_t mma_bar = saddr(&bars[2 * kGenStages]), w_bar = saddr(&bars[2 * kGenStages + 1]);
+  if (tid == 0) {
+    for (uint32_t i = 0; i < kGenStages; ++i) {
+      mbar_init(full_bar(i), 4);   // one arrival per producer warp
+      mbar_init(empty_bar(i), 1);  // the layer-1 commit (or the consumer, for a tile of bad rows)
+    }
     mbar_init(mma_bar, 1);
     mbar_init(w_bar, 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
-  if (warp == 0) {
+  if (tid < 32) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(saddr(&tmem_slot)),
                  "r"(tmem_cols)
                  : "memory");
@@ -87,7 +110,7 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
   const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
   if (D + 2 <= kGenTileTable) {
     uint32_t *s_seg = reinterpret_cast<uint32_t *>(tables), *s_tst = s_seg + kGenTileTable;
-    for (uint32_t i = row; i < D + 2; i += blockDim.x) {
+    for (uint32_t i = tid; i < D + 2; i += blockDim.x) {
       s_seg[i] = __ldg(seg + i);
       s_tst[i] = __ldg(tst + i);
     }
@@ -98,63 +121,114 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
   const uint32_t ngrids = A.num_sets * A.num_levels * A.num_mips;
   if (ngrids <= kGenGrids) {
     GridDesc *s_grids = reinterpret_cast<GridDesc *>(tables + 2 * kGenTileTable * 4);
-    for (uint32_t i = row; i < ngrids; i += blockDim.x) s_grids[i] = A.grids[i];
+    for (uint32_t i = tid; i < ngrids; i += blockDim.x) s_grids[i] = A.grids[i];
     grids = s_grids;
   }
   fence_before();
   __syncthreads();
   fence_after();
-  const uint32_t tAcc = tmem_slot;               // H fp32 columns
-  const uint32_t tAH = tmem_slot + H;            // hidden A operand, H / 2 columns
-  const uint32_t tA1 = tmem_slot + H + H / 2;    // two layer-1 A operands, K1 / 2 columns each
-  const uint32_t sW = saddr(smem);
-  const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
+  const uint32_t tAcc = tmem_slot;             // H fp32 columns
+  const uint32_t tAH = tmem_slot + H;          // hidden A operand, H / 2 columns
+  const uint32_t tA1 = tmem_slot + H + H / 2;  // ring stages, K1 / 2 columns each
   const uint32_t T = __ldg(B.meta);
-  uint32_t cur = 0xFFFFFFFFu, mph = 0, wph = 0;
-  auto wait = [&](uint32_t bar, uint32_t parity) {
-    if (!mbar_wait(bar, parity)) {
-      atomicOr(status, 1u);
-      abort_flag = 1;
-    }
-  };
-  TileWalk walk;
-  // Tile tt's row of this thread: its query, bad-row handling, and the feature
-  // row written into layer-1 A operand `buf` (zeros for rows that are not good).
-  auto fetch = [&](uint32_t tt, uint32_t buf, uint32_t &d_, uint32_t &oi_, bool &good_) {
-    uint32_t st_, ln_;
-    walk.at(seg, tst, D, tt, d_, st_, ln_);
-    const bool valid = row < ln_;
+  const uint32_t grid = gridDim.x;
+  const uint32_t K = blockIdx.x < T ? (T - blockIdx.x + grid - 1) / grid : 0;  // this CTA's tiles
+  if (wg == 0) {
+    // ------------------------------------------------------------- producer
+    TileWalk walk;
+    // tile j's query record and output row; the next tile's are loaded while
+    // tile j is gathered
+    auto load_row = [&](uint32_t jj, uint32_t &d_, uint32_t &len_, ntc_query &q_, uint32_t &oi_) {
+      uint32_t st_;
+      walk.at(seg, tst, D, blockIdx.x + jj * grid, d_, st_, len_);
+      oi_ = 0;
+      if (row < len_) {
+        q_ = load_query(B.sorted + st_ + row);
+        oi_ = __ldg(B.perm + st_ + row);
+      }
+    };
+    uint32_t dec = D, len = 0, oi = 0;
     ntc_query q;
-    oi_ = 0;
-    if (valid) {
-      q = load_query(B.sorted + st_ + row);
-      oi_ = __ldg(B.perm + st_ + row);
+    if (K) load_row(0, dec, len, q, oi);
+    for (uint32_t j = 0; j < K; ++j) {
+      if (abort_flag) break;
+      const uint32_t s = j % kGenStages, use = j / kGenStages;
+      uint32_t ndec = D, nlen = 0, noi = 0;
+      ntc_query nq;
+      if (j + 1 < K) load_row(j + 1, ndec, nlen, nq, noi);
+      const bool valid = row < len;
+      const bool good = valid && dec < D && !query_bad(A, q);
+      const bool bad = valid && !good;
+      count_bad_warp(bad, err);
+      if (bad)
+        for (uint32_t c = 0; c < OC; ++c) out[(size_t)oi * OC + c] = __int_as_float(0x7fc00000);
+      float f[NP];
+      if (good) gen_features_t<L, C, NP>(A, grids, q, f);
+      else
+#pragma unroll
+        for (int i = 0; i < NP; ++i) f[i] = 0.0f;
+      if (!mbar_wait(empty_bar(s), (use & 1u) ^ 1u)) {  // the stage's previous tile has left layer 1
+        atomicOr(status, 1u);
+        abort_flag = 1;
+      }
+      fence_after();
+      if (dec < D) {
+#pragma unroll
+        for (int kc = 0; kc < NP / 16; ++kc) {
+          if ((uint32_t)kc * 16 >= K1) break;
+          uint32_t p[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) p[i] = pack<BF16>(f[16 * kc + 2 * i], f[16 * kc + 2 * i + 1]);
+          tmem_st8(tA1 + s * (K1 / 2) + lanes + 8 * kc, p);
+        }
+        tmem_wait_st();
+      }
+      oidx[s * 128 + row] = good ? oi : 0xFFFFFFFFu;
+      fence_before();
+      __syncwarp();
+      if ((row & 31) == 0) mbar_arrive(full_bar(s));
+      dec = ndec;
+      len = nlen;
+      q = nq;
+      oi = noi;
     }
-    good_ = valid && d_ < D && !query_bad(A, q);
-    const bool bad = valid && !good_;
-    count_bad_warp(bad, err);
-    if (bad)
-      for (uint32_t c = 0; c < C; ++c) out[(size_t)oi_ * C + c] = __int_as_float(0x7fc00000);
-    if (d_ >= D) return;  // a tile of the bad bucket (CTA-uniform): nothing to multiply
-    float f[kGenMaxIn];
-    if (good_) gen_features(A, grids, q, f);
-    else
-#pragma unroll
-      for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
-#pragma unroll
-    for (int kc = 0; kc < kGenMaxIn / 16; ++kc) {
-      if ((uint32_t)kc * 16 >= K1) break;
-      uint32_t p[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) p[i] = pack<BF16>(f[16 * kc + 2 * i], f[16 * kc + 2 * i + 1]);
-      tmem_st8(tA1 + buf * (K1 / 2) + lanes + 8 * kc, p);
-    }
-  };
-  uint32_t t = blockIdx.x, buf = 0, dec = D, oi = 0;
-  bool good = false;
-  if (t < T) fetch(t, buf, dec, oi, good);
-  while (t < T) {
-    if (dec < D) {
+  } else {
+    // ------------------------------------------------------------- consumer
+    uint32_t cur = 0xFFFFFFFFu, mph = 0, wph = 0;
+    const uint32_t sW = saddr(smem);
+    TileWalk cwalk;
+    const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
+    auto wait = [&](uint32_t bar, uint32_t parity) {
+      if (!mbar_wait(bar, parity)) {
+        atomicOr(status, 1u);
+        abort_flag = 1;
+      }
+    };
+    // the MMA chain: one warp polls without suspending (lower wake-up
+    // latency), the named barrier releases the rest of the warpgroup
+    auto wait_mma = [&]() {
+      if (row < 32 && !mbar_spin(mma_bar, mph)) {
+        atomicOr(status, 1u);
+        abort_flag = 1;
+      }
+      mph ^= 1;
+      wg_bar(1);
+    };
+    for (uint32_t j = 0; j < K; ++j) {
+      const uint32_t s = j % kGenStages, use = j / kGenStages;
+      uint32_t dec, st, len;
+      cwalk.at(seg, tst, D, blockIdx.x + j * grid, dec, st, len);
+      if (row < 32) wait(full_bar(s), use & 1u);
+      wg_bar(1);
+      fence_after();
+      const uint32_t oi = oidx[s * 128 + row];
+      const bool good = oi != 0xFFFFFFFFu;
+      wg_bar(1);  // every consumer thread has read its output row
+      if (abort_flag) break;
+      if (dec >= D) {  // a tile of bad rows: nothing to multiply
+        if (row == 0) mbar_arrive(empty_bar(s));
+        continue;
+      }
       if (dec != cur) {
         // every MMA of the previous tile has completed: the weights may change
         if (row == 0) {
@@ -169,44 +243,45 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
         wph ^= 1;
         cur = dec;
       }
-      tmem_wait_st();  // this tile's feature rows (written by the previous fetch)
-      fence_before();
-      __syncthreads();
-      if (abort_flag) break;
       if (row == 0) {
         fence_after();
         const uint64_t d1 = smem_desc(sW, K1);
         for (uint32_t kc = 0; kc < K1 / 16; ++kc)
-          umma_ta(tAcc, tA1 + buf * (K1 / 2) + 8 * kc, d1 + 16 * kc, id_h, kc);
+          umma_ta(tAcc, tA1 + s * (K1 / 2) + 8 * kc, d1 + 16 * kc, id_h, kc);
         umma_commit(mma_bar);
+        umma_commit(empty_bar(s));
       }
-    }
-    // the next tile's rows are gathered while this tile's MMA chain runs
-    const uint32_t tn = t + gridDim.x;
-    uint32_t ndec = D, noi = 0;
-    bool ngood = false;
-    if (tn < T) fetch(tn, buf ^ 1u, ndec, noi, ngood);
-    if (dec < D) {
       for (uint32_t l = 0; l < NL; ++l) {
         // hidden layer l is in the accumulator: bias, activation, next A operand
-        wait(mma_bar, mph);
-        mph ^= 1;
+        wait_mma();
         fence_after();
         const float *bl = bias + l * H;
-        for (uint32_t c0 = 0; c0 < H; c0 += 16) {
+        if (H == 16) {
           uint32_t v[16];
-          tmem_ld16(tAcc + lanes + c0, v);
+          tmem_ld16(tAcc + lanes, v);
           tmem_wait_ld();
           uint32_t p[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[c0 + 2 * i],
-                                  __uint_as_float(v[2 * i + 1]) + bl[c0 + 2 * i + 1], G.activation, G.slope);
-          tmem_st8(tAH + lanes + c0 / 2, p);
+            p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[2 * i], __uint_as_float(v[2 * i + 1]) + bl[2 * i + 1],
+                                  G.activation, G.slope);
+          tmem_st8(tAH + lanes, p);
+        } else {
+          for (uint32_t c0 = 0; c0 < H; c0 += 32) {
+            uint32_t v[32];
+            tmem_ld32(tAcc + lanes + c0, v);
+            tmem_wait_ld();
+            uint32_t p[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+              p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[c0 + 2 * i],
+                                    __uint_as_float(v[2 * i + 1]) + bl[c0 + 2 * i + 1], G.activation, G.slope);
+            tmem_st16(tAH + lanes + c0 / 2, p);
+          }
         }
         tmem_wait_st();
         fence_before();
-        __syncthreads();
+        wg_bar(1);
         if (abort_flag) break;
         if (row == 0) {
           fence_after();
@@ -218,32 +293,25 @@ __global__ void __launch_bounds__(128) k_decode_gen_tc(Assets A, GenWeights G, B
         }
       }
       if (abort_flag) break;
-      wait(mma_bar, mph);
-      mph ^= 1;
+      wait_mma();
       fence_after();
       uint32_t o[16];
       tmem_ld16(tAcc + lanes, o);
       tmem_wait_ld();
       if (good) {
         const float *bo = bias + NL * H;
-        float *dst = out + (size_t)oi * C;
+        float *dst = out + (size_t)oi * OC;
 #pragma unroll
         for (int c = 0; c < 16; ++c)
-          if (c < (int)C) dst[c] = 1.0f / (1.0f + expf(-(__uint_as_float(o[c]) + bo[c])));
+          if (c < (int)OC) dst[c] = 1.0f / (1.0f + expf(-(__uint_as_float(o[c]) + bo[c])));
       }
       fence_before();
-      __syncthreads();  // the next tile overwrites the accumulator and the hidden operand
-      if (abort_flag) break;
+      wg_bar(1);  // the next tile overwrites the accumulator and the hidden operand
     }
-    t = tn;
-    buf ^= 1u;
-    dec = ndec;
-    oi = noi;
-    good = ngood;
   }
   fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (tid < 32) {
     fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_slot), "r"(tmem_cols)
                  : "memory");
@@ -396,30 +464,42 @@ uint32_t gen_tmem_cols(const GenWeights &G) {
   return c;
 }
 
-template <bool BF16>
+template <bool BF16, int L, int C>
 cudaError_t launch_gen_tc_t(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
                             unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
   const uint32_t img = (uint32_t)gen_tc_image_bytes(G.in_dim, G.hidden, G.layers);
   const size_t smem = gen_smem_bytes(img);
   const uint32_t cols = gen_tmem_cols(G);
-  cudaError_t e = cudaFuncSetAttribute(k_decode_gen_tc<BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e =
+      cudaFuncSetAttribute(k_decode_gen_tc<BF16, L, C>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  int occ = 1;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_gen_tc<BF16>, 128, smem);
+  // resident CTAs per SM: registers, shared memory, threads, and tensor memory
+  // (every resident CTA allocates `cols` of the SM's 512 columns)
+  int occ = resident_ctas(k_decode_gen_tc<BF16, L, C>, 256, smem);
+  occ = min(occ, (int)(512 / cols));
   if (occ < 1) occ = 1;
-  if ((uint32_t)occ > 512 / cols) occ = (int)(512 / cols);  // tensor memory: every resident CTA allocates
   const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms * occ;
   if (grid > max_tiles) grid = max_tiles;
-  k_decode_gen_tc<BF16><<<(unsigned)grid, 128, smem, st>>>(A, G, B, out, err, status, cols, img);
+  k_decode_gen_tc<BF16, L, C><<<(unsigned)grid, 256, smem, st>>>(A, G, B, out, err, status, cols, img);
   return cudaGetLastError();
+}
+
+template <bool BF16>
+cudaError_t launch_gen_tc_b(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+                            unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
+  if (A.channels == 8)
+    return A.num_levels == 2 ? launch_gen_tc_t<BF16, 2, 8>(A, G, B, n, out, err, status, num_sms, st)
+                             : launch_gen_tc_t<BF16, 1, 8>(A, G, B, n, out, err, status, num_sms, st);
+  return A.num_levels == 2 ? launch_gen_tc_t<BF16, 2, 4>(A, G, B, n, out, err, status, num_sms, st)
+                           : launch_gen_tc_t<BF16, 1, 4>(A, G, B, n, out, err, status, num_sms, st);
 }
 
 template <typename T>
 cudaError_t launch_gen_fma_t(const Assets &A, const GenWeights &G, const Buckets *B, const ntc_query *q, size_t n,
                              float *out, unsigned long long *err, int num_sms, cudaStream_t st) {
   int occ = 1;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_gen_fma<T>, 128, 0);
+  occ = resident_ctas(k_decode_gen_fma<T>, 128, 0);
   if (occ < 1) occ = 1;
   const size_t blocks = (n + 127) / 128;
   size_t grid = (size_t)num_sms * occ * 4;
@@ -434,8 +514,8 @@ cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buc
                                  unsigned long long *err, unsigned int *status, bool bf16, int num_sms,
                                  cudaStream_t st, int *launches) {
   *launches += 1;
-  return bf16 ? launch_gen_tc_t<true>(A, G, B, n, out, err, status, num_sms, st)
-              : launch_gen_tc_t<false>(A, G, B, n, out, err, status, num_sms, st);
+  return bf16 ? launch_gen_tc_b<true>(A, G, B, n, out, err, status, num_sms, st)
+              : launch_gen_tc_b<false>(A, G, B, n, out, err, status, num_sms, st);
 }
 
 cudaError_t launch_decode_gen_fma(const Assets &A, const GenWeights &G, const Buckets *B, const ntc_query *q,

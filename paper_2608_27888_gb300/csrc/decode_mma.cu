@@ -395,7 +395,7 @@ cudaError_t launch_mma_t(const Assets &A, const WeightImages &W, const Buckets &
   static int occ = -1;
   if (occ < 0) {
     cudaFuncSetAttribute(k_decode_mma<H, NT3, BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_mma<H, NT3, BF16>, kTile, smem);
+    occ = resident_ctas(k_decode_mma<H, NT3, BF16>, kTile, smem);
     if (occ < 1) occ = 1;
   }
   size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
@@ -410,7 +410,7 @@ cudaError_t launch_div_t(const Assets &A, const WeightImages &W, const ntc_query
                          float *out, unsigned long long *err, int num_sms, cudaStream_t st) {
   static int occ = -1;
   if (occ < 0) {
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_divergent<H, NT3, BF16>, 128, 0);
+    occ = resident_ctas(k_decode_divergent<H, NT3, BF16>, 128, 0);
     if (occ < 1) occ = 1;
   }
   size_t blocks = (n + 127) / 128;

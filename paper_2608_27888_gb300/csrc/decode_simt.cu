@@ -230,7 +230,7 @@ cudaError_t launch_fp32_t(const Assets &A, const WeightImages &W, const Buckets 
   static int occ = -1;
   if (occ < 0) {
     cudaFuncSetAttribute(k_decode_fp32<H, CP>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_decode_fp32<H, CP>, kTile, smem);
+    occ = resident_ctas(k_decode_fp32<H, CP>, kTile, smem);
     if (occ < 1) occ = 1;
   }
   size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;

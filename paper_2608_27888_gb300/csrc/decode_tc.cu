@@ -203,9 +203,6 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
 constexpr uint32_t kSmemTileTable = 1024;  // staged when D + 2 <= this
 constexpr uint32_t kSmemGrids = 1024;      // staged when S * 2 * M <= this
 
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
-}
 
 // Shared-memory plan of the warp-specialised kernel: only the decoders' weights
 // (the B operands) and bookkeeping live in shared memory; every A operand and

@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "../../include/ntc.h"
 
 namespace ntc {
@@ -252,91 +254,96 @@ __device__ __forceinline__ void query_features(const Assets &A, const ntc_query 
 }
 
 // Positional encoding of one coordinate pair at input offset BASE: for k < F,
-// sin / cos of 2 pi 2^k u and of 2 pi 2^k v (u, v as the taps see them).
-template <int BASE>
-__device__ __forceinline__ void pe_features(float u, float v, uint32_t F, float (&f)[kGenMaxIn]) {
+// sin / cos of 2 pi 2^k u and of 2 pi 2^k v (u, v as the taps see them).  One
+// sincospif per coordinate gives k = 0; every further frequency doubles the
+// angle (sin 2a = 2 sin a cos a, cos 2a = cos^2 a - sin^2 a), which keeps the
+// error within a few ulp for the at most 8 frequencies.
+template <int BASE, int N>
+__device__ __forceinline__ void pe_features(float u, float v, uint32_t F, float (&f)[N]) {
+  if (F == 0) return;
+  float su, cu, sv, cv;
+  sincospif(2.0f * u, &su, &cu);
+  sincospif(2.0f * v, &sv, &cv);
 #pragma unroll
   for (int k = 0; k < kGenMaxPe; ++k) {
-    if (BASE + 4 * k + 3 >= kGenMaxIn) break;
+    if (BASE + 4 * k + 3 >= N) break;
     if (k < (int)F) {
-      float su, cu, sv, cv;
-      sincospif(ldexpf(u, k + 1), &su, &cu);
-      sincospif(ldexpf(v, k + 1), &sv, &cv);
       f[BASE + 4 * k + 0] = su;
       f[BASE + 4 * k + 1] = cu;
       f[BASE + 4 * k + 2] = sv;
       f[BASE + 4 * k + 3] = cv;
+      const float su2 = 2.0f * su * cu, cu2 = cu * cu - su * su;
+      const float sv2 = 2.0f * sv * cv, cv2 = cv * cv - sv * sv;
+      su = su2, cu = cu2, sv = sv2, cv = cv2;
     }
   }
 }
 
 // The latent features of level K of a good query, C channels per texel, at
 // input offset K * C; with t > 0 the two mips are blended (weights scaled by
-// 1 - t and t, as in query_features).
-template <int K, int C>
+// 1 - t and t, as in query_features).  Every tap load of the level (both mips)
+// is issued before any is consumed.
+template <int K, int C, int N>
 __device__ __forceinline__ void gen_level(const Assets &A, const GridDesc *g, int lo, float t, const ntc_query &q,
-                                          float (&f)[kGenMaxIn]) {
-  const int nm = t > 0.0f ? 2 : 1;
-  for (int mi = 0; mi < nm; ++mi) {
-    unsigned long long idx[4];
-    float w[4];
-    grid_taps(g[K * A.num_mips + lo + mi], q.u, q.v, A.address_mode, idx, w);
-    const float s = nm == 1 ? 1.0f : (mi == 0 ? __fsub_rn(1.0f, t) : t);
+                                          float (&f)[N]) {
+  using Raw = typename std::conditional<C == 8, uint4, uint2>::type;
+  const bool two = t > 0.0f;
+  unsigned long long idx[2][4];
+  float w[2][4];
+  grid_taps(g[K * A.num_mips + lo], q.u, q.v, A.address_mode, idx[0], w[0]);
+  if (two) grid_taps(g[K * A.num_mips + lo + 1], q.u, q.v, A.address_mode, idx[1], w[1]);
+  Raw raw[2][4];
+#pragma unroll
+  for (int m = 0; m < 2; ++m)
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+      if (m == 0 || two) raw[m][p] = __ldg(reinterpret_cast<const Raw *>(A.lat) + idx[m][p]);
+#pragma unroll
+  for (int m = 0; m < 2; ++m) {
+    if (m == 1 && !two) break;
+    const float s = !two ? 1.0f : (m == 0 ? __fsub_rn(1.0f, t) : t);
 #pragma unroll
     for (int p = 0; p < 4; ++p) {
-      const float wp = nm == 1 ? w[p] : w[p] * s;
-      if (C == 8) {
-        const uint4 raw = __ldg(A.lat + idx[p]);
-        const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
+      const float wp = !two ? w[m][p] : w[m][p] * s;
+      const __half2 *h = reinterpret_cast<const __half2 *>(&raw[m][p]);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const float2 x = __half22float2(h[c]);
-          f[K * C + 2 * c] = fmaf(wp, x.x, f[K * C + 2 * c]);
-          f[K * C + 2 * c + 1] = fmaf(wp, x.y, f[K * C + 2 * c + 1]);
-        }
-      } else {
-        const uint2 raw = __ldg(reinterpret_cast<const uint2 *>(A.lat) + idx[p]);
-        const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          const float2 x = __half22float2(h[c]);
-          f[K * C + 2 * c] = fmaf(wp, x.x, f[K * C + 2 * c]);
-          f[K * C + 2 * c + 1] = fmaf(wp, x.y, f[K * C + 2 * c + 1]);
-        }
+      for (int c = 0; c < C / 2; ++c) {
+        const float2 x = __half22float2(h[c]);
+        f[K * C + 2 * c] = fmaf(wp, x.x, f[K * C + 2 * c]);
+        f[K * C + 2 * c + 1] = fmaf(wp, x.y, f[K * C + 2 * c + 1]);
       }
     }
   }
 }
 
-// The MLP input of a good query for a general shape: num_levels x channels
-// latent features, then the positional encoding; zero beyond in_dim.  grids:
-// A.grids, or a copy of it (in shared memory).
-__device__ __forceinline__ void gen_features(const Assets &A, const GridDesc *grids, const ntc_query &q,
-                                             float (&f)[kGenMaxIn]) {
+// The MLP input of a good query for a general shape with L levels of C
+// channels: the latent features, then the positional encoding; zero up to N.
+// grids: A.grids, or a copy of it (in shared memory).
+template <int L, int C, int N>
+__device__ __forceinline__ void gen_features_t(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                               float (&f)[N]) {
+  static_assert(N >= L * C + 4 * kGenMaxPe && N <= kGenMaxIn, "feature array too small");
 #pragma unroll
-  for (int i = 0; i < kGenMaxIn; ++i) f[i] = 0.0f;
+  for (int i = 0; i < N; ++i) f[i] = 0.0f;
   float t;
   const int lo = select_mip(q.lod, A.num_mips, t);
-  const GridDesc *g = grids + (size_t)q.set_id * A.num_levels * A.num_mips;
+  const GridDesc *g = grids + (size_t)q.set_id * L * A.num_mips;
   const float u = A.address_mode == 0 ? __fsub_rn(q.u, floorf(q.u)) : q.u;
   const float v = A.address_mode == 0 ? __fsub_rn(q.v, floorf(q.v)) : q.v;
-  const uint32_t F = A.pe_frequencies;
+  gen_level<0, C, N>(A, g, lo, t, q, f);
+  if (L == 2) gen_level<1, C, N>(A, g, lo, t, q, f);
+  pe_features<L * C, N>(u, v, A.pe_frequencies, f);
+}
+
+// Any general shape, dispatched at run time (kGenMaxIn values).
+__device__ __forceinline__ void gen_features(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                             float (&f)[kGenMaxIn]) {
   if (A.channels == 8) {
-    gen_level<0, 8>(A, g, lo, t, q, f);
-    if (A.num_levels == 2) {
-      gen_level<1, 8>(A, g, lo, t, q, f);
-      pe_features<16>(u, v, F, f);
-    } else {
-      pe_features<8>(u, v, F, f);
-    }
+    if (A.num_levels == 2) gen_features_t<2, 8, kGenMaxIn>(A, grids, q, f);
+    else gen_features_t<1, 8, kGenMaxIn>(A, grids, q, f);
   } else {
-    gen_level<0, 4>(A, g, lo, t, q, f);
-    if (A.num_levels == 2) {
-      gen_level<1, 4>(A, g, lo, t, q, f);
-      pe_features<8>(u, v, F, f);
-    } else {
-      pe_features<4>(u, v, F, f);
-    }
+    if (A.num_levels == 2) gen_features_t<2, 4, kGenMaxIn>(A, grids, q, f);
+    else gen_features_t<1, 4, kGenMaxIn>(A, grids, q, f);
   }
 }
 
@@ -440,6 +447,29 @@ cudaError_t launch_debug_taps(const Assets &A, const ntc_query *q, size_t n, uns
                               float *w, float *t, cudaStream_t st, int *launches);
 cudaError_t launch_debug_features(const Assets &A, const ntc_query *q, size_t n, float *f,
                                   cudaStream_t st, int *launches);
+// CTAs of `kernel` that fit on one SM at once (threads, registers, shared
+// memory), computed from the kernel's own attributes and the device's limits.
+template <typename Kernel>
+inline int resident_ctas(Kernel kernel, int threads, size_t dyn_smem) {
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess) return 1;
+  int dev = 0, regs_sm = 65536, smem_sm = 233472, thr_sm = 2048, cta_sm = 32;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev);
+  cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+  cudaDeviceGetAttribute(&thr_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev);
+  cudaDeviceGetAttribute(&cta_sm, cudaDevAttrMaxBlocksPerMultiprocessor, dev);
+  const int warps = (threads + 31) / 32;
+  const int regs_cta = warps * ((fa.numRegs + 7) / 8 * 8) * 32;  // 256-register allocation units per warp
+  int occ = regs_cta > 0 ? regs_sm / regs_cta : cta_sm;
+  occ = occ < thr_sm / (warps * 32) ? occ : thr_sm / (warps * 32);
+  const size_t smem_cta = dyn_smem + fa.sharedSizeBytes + 1024;  // 1 KB per CTA reserved by the system
+  const int by_smem = (int)((size_t)smem_sm / smem_cta);
+  occ = occ < by_smem ? occ : by_smem;
+  occ = occ < cta_sm ? occ : cta_sm;
+  return occ < 1 ? 1 : occ;
+}
+
 // Launch with programmatic stream serialisation (see pdl_wait).
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,

@@ -381,3 +381,22 @@ def test_kmeans_map_equals_oracle_bit_for_bit(case):
     assert got_it == ref_it
     assert np.array_equal(got_map, ref_map)
     assert np.array_equal(got_mu.view(np.uint64), ref_mu.view(np.uint64))
+
+
+def test_bucketing_with_the_most_decoders():
+    """4095 decoders (the most the library accepts): the bucketing kernels'
+    per-warp counters then take most of their shared memory."""
+    D = 4095
+    a = tiny_assets([[(4, 4), (2, 2)]] * D, hidden=16, out_dim=4, num_decoders=D, num_sets=D,
+                    set_to_decoder=np.random.default_rng(0).permutation(D))
+    dec = ntc().Decoder(a, "fp16")
+    rng = np.random.default_rng(1)
+    for n in (1, 2049, 70001):
+        sets = rng.integers(0, D + 3, n)  # a few out-of-range ids: the extra bucket
+        q = queries([(int(s), 0.5, 0.5, 0.0) for s in sets])
+        perm, counts, tiles = dec.bucket(dq(q))
+        p, c, _, t = oracle.bucket(q["set_id"], a.set_to_decoder, D)
+        assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
+        assert np.array_equal(counts.cpu().numpy().astype(np.uint32), c)
+        assert np.array_equal(tiles.cpu().numpy().astype(np.uint32), t)
+    dec.close()
