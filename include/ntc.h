@@ -30,8 +30,12 @@
  * Memory: the context owns device copies of latents, weights and map.  Query
  * and output buffers of ntc_decode are DEVICE pointers owned by the caller.
  * Scratch (bucket counts, permutation, sorted queries) is owned by the context
- * and grows on demand with cudaMallocAsync on the call's stream.  One context
- * must not run two decodes concurrently (on different streams or threads).
+ * and grows on demand with cudaMallocAsync on the call's stream.  The
+ * tensor-core BUCKETED decode sorts in one pass when (num_decoders + 1) * n
+ * rows of 20 bytes fit in 24 GiB, giving every decoder a region of n rows
+ * (e.g. 1.4 GB for 16 decoders and 4M queries); otherwise it runs the stable
+ * three-kernel sort, which needs n rows.  One context must not run two
+ * decodes concurrently (on different streams or threads).
  *
  * Errors: host-detectable problems return a status and enqueue nothing; the
  * message is available from ntc_last_error().  A query whose set id is out of

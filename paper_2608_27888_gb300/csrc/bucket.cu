@@ -234,10 +234,21 @@ __device__ void block_scan_256(uint32_t *a, uint32_t len) {
   __syncthreads();
 }
 
+// SPREAD (the single-pass bucketing of the tensor-core decode): no k_hist or
+// k_scan runs first.  Decoder d owns region [d * cap, d * cap + cap) of perm
+// and sorted (cap = n); each chunk reserves room for its run of decoder d with
+// one atomicAdd on cursor[d], so runs of one decoder keep chunk order only as
+// far as the atomics happen to, and the permutation is not the stable one
+// (every decoded row is independent of the others in its tile, so outputs do
+// not change).  The last CTA to finish (atomic ticket, no waiting) writes meta
+// with seg[d] = the decoder's count and the tile starts, and clears cursor and
+// ticket for the next call.
+template <bool SPREAD>
 __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_query *q, size_t n,
                                                             const uint32_t *counts, uint32_t chunks,
-                                                            const uint32_t *meta, uint32_t *perm,
-                                                            ntc_query *sorted, unsigned int *status) {
+                                                            uint32_t *meta, uint32_t *perm,
+                                                            ntc_query *sorted, unsigned int *status,
+                                                            uint32_t *cursor, uint32_t cap) {
   // shared memory: the chunk's records [chunk] (16 B), the chunk-local index
   // [chunk] (u16) and decoder [chunk] (u16) of every sorted slot, then per-warp
   // counters [kWarps][D+1] and the chunk's per-decoder local offsets and global
@@ -256,7 +267,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
   const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
   bulk_issue(srec, q + cbase, valid * 16u, &bar);  // the queries do not depend on k_scan
-  pdl_wait();                                        // the scanned counts and segment starts
+  if (!SPREAD) pdl_wait();                           // the scanned counts and segment starts
   pdl_trigger();                                     // the decode may launch (it waits for this grid)
   if (!bulk_wait(&bar)) atomicOr(status, 2u);
   const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
@@ -292,7 +303,8 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
       run += c;
     }
     loff[d] = run;
-    gbase[d] = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
+    if (SPREAD) gbase[d] = run ? d * cap + atomicAdd(cursor + d, run) : 0u;
+    else gbase[d] = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
   }
   __syncthreads();
   block_scan_256(loff, D1);  // exclusive scan of the chunk totals over decoders
@@ -313,6 +325,38 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
     const uint32_t pos = gbase[d] + (i - loff[d]);
     perm[pos] = (uint32_t)(cbase + j);
     reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
+  }
+  if (SPREAD) {
+    __shared__ bool last;
+    uint32_t *ticket = cursor + D1;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();  // this CTA's reservations before its ticket
+      last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    // every chunk has reserved its runs: counts per decoder and tile starts
+    uint32_t *segc = meta + 1, *tst = meta + 1 + (D1 + 1);
+    for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
+      const uint32_t c = ((volatile uint32_t *)cursor)[d];
+      segc[d] = c;
+      loff[d] = (c + kTile - 1) / kTile;
+      cursor[d] = 0;
+    }
+    __syncthreads();
+    const uint32_t last_tiles = loff[D1 - 1];
+    __syncthreads();
+    block_scan_256(loff, D1);
+    for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) tst[d] = loff[d];
+    if (threadIdx.x == 0) {
+      const uint32_t T = loff[D1 - 1] + last_tiles;
+      tst[D1] = T;
+      segc[D1] = 0;
+      meta[0] = T;
+      *ticket = 0;
+    }
   }
 }
 
@@ -350,18 +394,26 @@ cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const S
   static bool attr_done = false;
   if (!attr_done) {
     cudaFuncSetAttribute(k_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    cudaFuncSetAttribute(k_scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    cudaFuncSetAttribute(k_scatter<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
     attr_done = true;
   }
   // totals[D+1] and the ticket live after meta
   uint32_t *totals = s.meta + meta_words(D);
   uint32_t *ticket = totals + (D + 1);
+  if (s.cursor) {  // single pass: reserve runs in per-decoder regions
+    cudaFuncSetAttribute(k_scatter<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    k_scatter<true><<<chunks, kBucketThreads, smem_scatter, st>>>(A, q, n, nullptr, chunks, s.meta, s.perm,
+                                                                   s.sorted, status, s.cursor, s.cap);
+    *launches += 1;
+    return cudaGetLastError();
+  }
   k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks, status);
   cudaError_t e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, (uint32_t)n, totals,
                              s.meta, ticket);
   if (e == cudaSuccess)
-    e = launch_pdl(k_scatter, dim3(chunks), dim3(kBucketThreads), smem_scatter, st, A, q, n,
-                   (const uint32_t *)s.counts, chunks, (const uint32_t *)s.meta, s.perm, s.sorted, status);
+    e = launch_pdl(k_scatter<false>, dim3(chunks), dim3(kBucketThreads), smem_scatter, st, A, q, n,
+                   (const uint32_t *)s.counts, chunks, s.meta, s.perm, s.sorted, status, (uint32_t *)nullptr,
+                   0u);
   *launches += 3;
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

@@ -136,6 +136,7 @@ __global__ void __launch_bounds__(256, 2) k_decode_gen_tc(Assets A, GenWeights G
   if (wg == 0) {
     // ------------------------------------------------------------- producer
     TileWalk walk;
+    walk.cap = B.spread_cap;
     // tile j's query record and output row; the next tile's are loaded while
     // tile j is gathered
     auto load_row = [&](uint32_t jj, uint32_t &d_, uint32_t &len_, ntc_query &q_, uint32_t &oi_) {
@@ -197,6 +198,7 @@ __global__ void __launch_bounds__(256, 2) k_decode_gen_tc(Assets A, GenWeights G
     uint32_t cur = 0xFFFFFFFFu, mph = 0, wph = 0;
     const uint32_t sW = saddr(smem);
     TileWalk cwalk;
+    cwalk.cap = B.spread_cap;
     const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
     auto wait = [&](uint32_t bar, uint32_t parity) {
       if (!mbar_wait(bar, parity)) {

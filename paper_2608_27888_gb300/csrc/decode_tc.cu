@@ -356,6 +356,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     ntc_query q;
     TileWalk walk;
     walk.ident_n = B.identity_n;
+    walk.cap = B.spread_cap;
     if (tile_of(j) < K) {
       walk.at(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
       if ((uint32_t)row < len) {
@@ -436,6 +437,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     uint32_t ph = 0, wph = 0, cur = 0xFFFFFFFFu;
     TileWalk cwalk;
     cwalk.ident_n = B.identity_n;
+    cwalk.cap = B.spread_cap;
     constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
     const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
     auto wait_bar = [&](uint32_t b, uint32_t parity) {

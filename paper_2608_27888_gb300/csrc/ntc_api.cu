@@ -45,6 +45,7 @@ struct ntc_ctx {
   size_t cap_n = 0, cap_counts = 0;
   uint32_t *d_counts = nullptr, *d_perm = nullptr, *d_meta = nullptr;
   ntc_query *d_sorted = nullptr;
+  uint32_t *d_cursor = nullptr;  // single-pass bucketing: [D+1] cursors + ticket, zero between calls
   // staging for ntc_decode_host, and its copy streams and chunk events
   size_t cap_host = 0;
   ntc_query *d_hq = nullptr;
@@ -175,14 +176,26 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_perm);
   cudaFree(c->d_sorted);
   cudaFree(c->d_meta);
+  cudaFree(c->d_cursor);
   cudaFree(c->d_hq);
   cudaFree(c->d_hout);
 }
 
 size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
 
-// Make sure the bucketing scratch holds n queries (stream-ordered allocation).
-ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
+// Single-pass bucketing gives every decoder a region of n rows: used when
+// that fits this budget (the stable three-kernel sort needs n rows in all).
+constexpr size_t kSpreadBudgetBytes = 24ull << 30;
+
+bool use_spread(const ntc_ctx *c, size_t n) {
+  const size_t rows = ((size_t)c->D + 1) * n;
+  return rows * (sizeof(ntc_query) + 4) <= kSpreadBudgetBytes && rows < 0xFFFFFF00ull;
+}
+
+// Make sure the bucketing scratch holds n queries (stream-ordered allocation);
+// `rows` entries of perm and sorted (n, or (D+1) * n for the single pass).
+ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st, size_t rows = 0) {
+  if (rows < n) rows = n;
   const size_t chunks = (n + kBucketChunk - 1) / kBucketChunk;
   const size_t counts = (size_t)(c->D + 1) * (chunks ? chunks : 1);
   if (!c->d_meta) {
@@ -197,15 +210,19 @@ ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
     CK(cudaMallocAsync((void **)&c->d_counts, counts * 4, st), "scratch allocation");
     c->cap_counts = counts;
   }
-  if (n > c->cap_n) {
+  if (rows > c->cap_n) {
     if (c->d_perm) CK(cudaFreeAsync(c->d_perm, st), "scratch free");
     if (c->d_sorted) CK(cudaFreeAsync(c->d_sorted, st), "scratch free");
     c->d_perm = nullptr;
     c->d_sorted = nullptr;
     c->cap_n = 0;
-    CK(cudaMallocAsync((void **)&c->d_perm, n * 4, st), "scratch allocation");
-    CK(cudaMallocAsync((void **)&c->d_sorted, n * sizeof(ntc_query), st), "scratch allocation");
-    c->cap_n = n;
+    CK(cudaMallocAsync((void **)&c->d_perm, rows * 4, st), "scratch allocation");
+    CK(cudaMallocAsync((void **)&c->d_sorted, rows * sizeof(ntc_query), st), "scratch allocation");
+    c->cap_n = rows;
+  }
+  if (!c->d_cursor) {
+    CK(cudaMallocAsync((void **)&c->d_cursor, ((size_t)c->D + 2) * 4, st), "scratch allocation");
+    CK(cudaMemsetAsync(c->d_cursor, 0, ((size_t)c->D + 2) * 4, st), "scratch clear");
   }
   return NTC_OK;
 }
@@ -442,7 +459,9 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   // divergence to remove, so the tensor-core decode takes the queries in their
   // own order and nothing is sorted
   const bool shared = mode == NTC_MODE_BUCKETED && !fp32 && !c->general && c->D == 1;
-  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st);
+  // the tensor-core decodes need no stable order: single-pass bucketing
+  const bool spread = mode == NTC_MODE_BUCKETED && !fp32 && !shared && use_spread(c, n);
+  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st, spread ? ((size_t)c->D + 1) * n : n);
   if (s != NTC_OK) return s;
   if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
   if (unsorted) {
@@ -468,7 +487,12 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     B.meta = nullptr;
     B.identity_n = (uint32_t)n;
   } else {
-    e = launch_bucket(A, q, n, scratch_of(c), st, &launches, c->d_status);
+    Scratch sc = scratch_of(c);
+    if (spread) {
+      sc.cursor = c->d_cursor;
+      sc.cap = (uint32_t)n;
+    }
+    e = launch_bucket(A, q, n, sc, st, &launches, c->d_status);
     if (e != cudaSuccess) {
       c->launches += launches;
       return cuda_fail(e, "bucketing launch");
@@ -476,6 +500,7 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     B.sorted = c->d_sorted;
     B.perm = c->d_perm;
     B.meta = c->d_meta;
+    B.spread_cap = spread ? (uint32_t)n : 0u;
   }
   if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
   if (c->general && fp32)

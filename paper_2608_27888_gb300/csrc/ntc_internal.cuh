@@ -128,6 +128,9 @@ struct Buckets {
   const uint32_t *perm;     // original index of each sorted query
   const uint32_t *meta;     // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
   uint32_t identity_n = 0;
+  // spread_cap != 0: single-pass bucketing; decoder d's sorted rows are at
+  // d * spread_cap .. and meta's seg[d] holds the decoder's count
+  uint32_t spread_cap = 0;
 };
 inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2); }
 
@@ -377,10 +380,12 @@ __device__ __forceinline__ void tile_info(const uint32_t *meta, uint32_t D, uint
 // The tiles of one role in increasing order: the decoder index only moves
 // forward, so a lookup is a few compares instead of a binary search.  With
 // ident_n != 0 (one decoder, nothing sorted) tile t is queries 128t .. of the
-// caller's array.
+// caller's array; with cap != 0 (single-pass bucketing) decoder d's rows start
+// at d * cap and seg[d] is their count.
 struct TileWalk {
   uint32_t d = 0;
   uint32_t ident_n = 0;
+  uint32_t cap = 0;
   __device__ __forceinline__ void at(const uint32_t *seg, const uint32_t *tst, uint32_t D, uint32_t t,
                                      uint32_t &dec, uint32_t &start, uint32_t &len) {
     if (ident_n) {
@@ -391,8 +396,14 @@ struct TileWalk {
     }
     while (d < D && tst[d + 1] <= t) ++d;
     dec = d;
-    start = seg[d] + (t - tst[d]) * kTile;
-    len = min((uint32_t)kTile, seg[d + 1] - start);
+    const uint32_t off = (t - tst[d]) * kTile;
+    if (cap) {
+      start = d * cap + off;
+      len = min((uint32_t)kTile, seg[d] - off);
+    } else {
+      start = seg[d] + off;
+      len = min((uint32_t)kTile, seg[d + 1] - start);
+    }
   }
 };
 
@@ -400,9 +411,13 @@ struct TileWalk {
 
 struct Scratch {
   uint32_t *counts;   // [(D+1) * chunks]
-  uint32_t *perm;     // [n]
-  ntc_query *sorted;  // [n]
+  uint32_t *perm;     // [n], or [(D+1) * cap] with cursor
+  ntc_query *sorted;  // [n], or [(D+1) * cap] with cursor
   uint32_t *meta;     // meta_words(D)
+  // single-pass bucketing (see k_scatter<true>): decoder d's runs go to
+  // [d * cap, d * cap + cap); cursor [D+1] + ticket [1], zero between calls
+  uint32_t *cursor = nullptr;
+  uint32_t cap = 0;
 };
 
 constexpr int kBucketThreads = 256;
