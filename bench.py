@@ -44,8 +44,6 @@ METRIC = "decoded queries/sec on 1 GB300 vs distinct decoders per warp; % of roo
 UNIT = "queries/s"
 WORKLOAD = ("config2: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16), 16 decoders "
             "16->64->64->8 (one per set), 4,194,304 queries: uniform set id, uniform UV, lod 0")
-BYTES_PER_QUERY = 16 + 8 * 16 + 8 * 4  # query record + 8 taps of 16 B + 8 fp32 outputs
-FLOPS_PER_QUERY = 2 * (16 * 64 + 64 * 64 + 64 * 8)
 L2_FLUSH_BYTES = 256 << 20
 KERNEL_NAMES = {("bucketed", False): "k_decode_tc (tcgen05/TMEM gather-decode)",
                 ("bucketed", True): "k_decode_fp32 (FFMA gather-decode)",
@@ -73,6 +71,9 @@ def parse():
     p.add_argument("--configs", action="store_true",
                    help="also time every full-size workload (1-5 and their maps); adds about two minutes")
     p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
+    p.add_argument("--workload", default="config2", choices=["config2", "paper-decoder"],
+                   help="the timed batch: the 4M-query 16-decoder workload (default), or Sec. 4's "
+                        "decoder (256^2x4 grid, positional encoding, LeakyReLU, 64x3) on a 1080p G-buffer")
     return p.parse_args()
 
 
@@ -146,7 +147,7 @@ def peaks():
 
 def kernel_source_hash():
     h = hashlib.sha1()
-    for f in ("decode_tc.cu", "ntc_internal.cuh"):
+    for f in ("decode_tc.cu", "decode_gen.cu", "tcgen05.cuh", "ntc_internal.cuh"):
         with open(os.path.join(ROOT, "paper_2608_27888_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
@@ -174,10 +175,24 @@ def dist_env():
     return ws, rank, local
 
 
-def workload(small: bool, rank: int):
+def shape_costs(a, q):
+    """Algorithmic bytes and FLOPs per query of a workload: the query record,
+    every tap's latent texel (both mips when the lod is fractional), the fp32
+    outputs; 2 x the MACs of the MLP."""
+    tri = a.num_mips > 1 and bool((q["lod"] != np.floor(q["lod"])).any())
+    bpq = 16 + (2 if tri else 1) * a.num_levels * 4 * a.channels * 2 + 4 * a.out_dim
+    H = a.hidden
+    flops = 2 * (a.in_dim * H + (a.num_hidden_layers - 1) * H * H + H * a.out_dim)
+    w_bytes = a.num_decoders * (a.in_dim * H + (a.num_hidden_layers - 1) * H * H + a.out_dim * H) * 2
+    return bpq, flops, w_bytes
+
+
+def workload(small: bool, rank: int, name: str = "config2"):
     """The benchmark batch of one rank: the same assets on every rank, a
     rank-specific query stream (queries are sharded, assets replicated)."""
     from paper_2608_27888_gb300 import workloads as W
+    if name == "paper-decoder":
+        return W.paper_decoder("small" if small else "full")
     seed = W.BASE_SEED + 2
     S, T, n = (16, 128, 40_077) if small else (16, 1024, 4_194_304)
     a = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
@@ -212,7 +227,7 @@ def run_reference(args, ws, rank):
     if rank != 0:
         return
     import oracle
-    w = workload(args.small, 0)
+    w = workload(args.small, 0, args.workload)
     n = len(w.queries)
     cores = os.cpu_count() or 1
     sample = min(n, 1 << 20)
@@ -231,7 +246,7 @@ def run_reference(args, ws, rank):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "sample_queries": sample},
+        "config": {"workload": WORKLOAD if args.workload == "config2" else w.name, "sample_queries": sample},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
@@ -253,7 +268,7 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     from paper_2608_27888_gb300 import ntc
 
-    w = workload(args.small, rank)
+    w = workload(args.small, rank, args.workload)
     n = len(w.queries)
     C = w.assets.out_dim
     dec = ntc.Decoder(w.assets, args.precision)
@@ -310,13 +325,14 @@ def main():
 
     # roofline of the dominant kernel (the gather-decode)
     peak, peak_kind = peaks()
-    w_bytes = w.assets.num_decoders * (64 * 16 + 64 * 64 + 8 * 64) * 2
-    alg_bytes = n * BYTES_PER_QUERY + w_bytes
+    bpq, flops_q, w_bytes = shape_costs(w.assets, w.queries)
+    alg_bytes = n * bpq + w_bytes
     achieved = alg_bytes / (decode_ms / 1e3) / 1e9
-    kernel_tag = f"{args.mode}-{args.precision}"
+    kernel_tag = f"{args.mode}-{args.precision}" + ("" if args.workload == "config2" else f"-{args.workload}")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": recorded_traffic(kernel_tag),
-                "kernel": KERNEL_NAMES[(args.mode, args.precision == "fp32")],
+                "kernel": KERNEL_NAMES[(args.mode, args.precision == "fp32")] if args.workload == "config2"
+                else "k_decode_gen_tc (general-shape tcgen05 gather-decode)",
                 "kernel_ms": decode_ms, "bucketing_ms": bucket_ms,
                 "peak_kind": f"{peak_kind} HBM copy bandwidth",
                 "algorithmic_bytes_per_launch": alg_bytes}
@@ -339,7 +355,7 @@ def main():
     # the in-run comparison: the unsorted divergent kernel on the same batch
     extra = {}
     for other in ("divergent", "divergent_fma"):
-        if args.mode == other or (args.precision == "fp32" and other == "divergent"):
+        if args.mode == other or (other == "divergent" and (args.precision == "fp32" or args.workload != "config2")):
             continue
         dms, _, _ = timed_steps(other, max(5, args.steps // 2), 2)
         extra[other] = {"value": n * ws / (statistics.mean(dms) / 1e3), "unit": UNIT,
@@ -353,13 +369,14 @@ def main():
         "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f16" if args.precision == "fp16" else args.precision.replace("fp", "f"),
         "data": "synthetic",
-        "config": {"workload": WORKLOAD if not args.small else "config2-small", "queries_per_gpu": n,
+        "config": {"workload": (WORKLOAD if args.workload == "config2" else w.name) if not args.small else w.name,
+                   "queries_per_gpu": n,
                    "decoders": w.assets.num_decoders, "mode": args.mode, "precision": args.precision,
                    "mean_distinct_decoders_per_warp": dd,
                    "l2": "flushed before every timed step (256 MiB write, then a 256 MiB read of another buffer; outside the step events)",
                    "parallelism": f"{ws} independent replicas (queries sharded, no collective)"},
         "roofline": roofline, "e2e": e2e, "gpu_launches": launches, "clocks": clocks,
-        "flops_per_query": FLOPS_PER_QUERY,
+        "flops_per_query": flops_q, "bytes_per_query": bpq,
         **extra,
     }
 
