@@ -71,7 +71,7 @@ __host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) {
 // (its completion empties the stage) and every further layer from the hidden
 // operand; consumer thread r runs row r's epilogues.
 template <bool BF16, int L, int C>
-__global__ void __launch_bounds__(256, 2) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
+__global__ void __launch_bounds__(256, L * C <= 8 ? 3 : 2) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
                                                        unsigned long long *err, unsigned int *status,
                                                        uint32_t tmem_cols, uint32_t img_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -163,11 +163,38 @@ __global__ void __launch_bounds__(256, 2) k_decode_gen_tc(Assets A, GenWeights G
       count_bad_warp(bad, err);
       if (bad)
         for (uint32_t c = 0; c < OC; ++c) out[(size_t)oi * OC + c] = __int_as_float(0x7fc00000);
-      float f[NP];
-      if (good) gen_features_t<L, C, NP>(A, grids, q, f);
-      else
+      // the feature row, packed to fp16/bf16 pairs as it is produced: the
+      // latent features, then sin/cos pairs of the encoding (zeros beyond)
+      constexpr int LW = L * C / 2, NW = NP / 2;
+      uint32_t pk[NW];
 #pragma unroll
-        for (int i = 0; i < NP; ++i) f[i] = 0.0f;
+      for (int i = 0; i < NW; ++i) pk[i] = 0u;
+      if (good) {
+        {
+          float fl[L * C];
+          gen_latents_t<L, C>(A, grids, q, fl);
+#pragma unroll
+          for (int i = 0; i < LW; ++i) pk[i] = pack<BF16>(fl[2 * i], fl[2 * i + 1]);
+        }
+        const uint32_t F = A.pe_frequencies;
+        if (F) {
+          float u, v, su, cu, sv, cv;
+          pe_coords(A, q, u, v);
+          sincospif(2.0f * u, &su, &cu);
+          sincospif(2.0f * v, &sv, &cv);
+#pragma unroll
+          for (int k = 0; k < kGenMaxPe; ++k) {
+            if (LW + 2 * k + 1 >= NW) break;
+            if (k < (int)F) {
+              pk[LW + 2 * k] = pack<BF16>(su, cu);
+              pk[LW + 2 * k + 1] = pack<BF16>(sv, cv);
+              const float su2 = 2.0f * su * cu, cu2 = cu * cu - su * su;
+              const float sv2 = 2.0f * sv * cv, cv2 = cv * cv - sv * sv;
+              su = su2, cu = cu2, sv = sv2, cv = cv2;
+            }
+          }
+        }
+      }
       if (!mbar_wait(empty_bar(s), (use & 1u) ^ 1u)) {  // the stage's previous tile has left layer 1
         atomicOr(status, 1u);
         abort_flag = 1;
@@ -179,7 +206,7 @@ __global__ void __launch_bounds__(256, 2) k_decode_gen_tc(Assets A, GenWeights G
           if ((uint32_t)kc * 16 >= K1) break;
           uint32_t p[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) p[i] = pack<BF16>(f[16 * kc + 2 * i], f[16 * kc + 2 * i + 1]);
+          for (int i = 0; i < 8; ++i) p[i] = pk[8 * kc + i];
           tmem_st8(tA1 + s * (K1 / 2) + lanes + 8 * kc, p);
         }
         tmem_wait_st();

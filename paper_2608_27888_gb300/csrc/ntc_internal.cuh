@@ -338,6 +338,25 @@ __device__ __forceinline__ void gen_features_t(const Assets &A, const GridDesc *
   pe_features<L * C, N>(u, v, A.pe_frequencies, f);
 }
 
+// Only the latent features of a good query: L levels of C channels.
+template <int L, int C>
+__device__ __forceinline__ void gen_latents_t(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                              float (&f)[L * C]) {
+#pragma unroll
+  for (int i = 0; i < L * C; ++i) f[i] = 0.0f;
+  float t;
+  const int lo = select_mip(q.lod, A.num_mips, t);
+  const GridDesc *g = grids + (size_t)q.set_id * L * A.num_mips;
+  gen_level<0, C, L * C>(A, g, lo, t, q, f);
+  if (L == 2) gen_level<1, C, L * C>(A, g, lo, t, q, f);
+}
+
+// The coordinates the taps see (the positional encoding's input).
+__device__ __forceinline__ void pe_coords(const Assets &A, const ntc_query &q, float &u, float &v) {
+  u = A.address_mode == 0 ? __fsub_rn(q.u, floorf(q.u)) : q.u;
+  v = A.address_mode == 0 ? __fsub_rn(q.v, floorf(q.v)) : q.v;
+}
+
 // Any general shape, dispatched at run time (kGenMaxIn values).
 __device__ __forceinline__ void gen_features(const Assets &A, const GridDesc *grids, const ntc_query &q,
                                              float (&f)[kGenMaxIn]) {
