@@ -71,7 +71,7 @@ __host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) {
 // (its completion empties the stage) and every further layer from the hidden
 // operand; consumer thread r runs row r's epilogues.
 template <bool BF16, int L, int C>
-__global__ void __launch_bounds__(256, L * C <= 8 ? 3 : 2) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
+__global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
                                                        unsigned long long *err, unsigned int *status,
                                                        uint32_t tmem_cols, uint32_t img_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
