@@ -292,8 +292,13 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
     __syncwarp();
   }
   __syncthreads();
-  // per decoder: warp prefix (in place), chunk total and global base
+  // per decoder: warp prefix (in place), chunk total and global base.  SPREAD
+  // with D + 1 <= blockDim.x: thread d keeps its reservation in a register
+  // until the copy-out, so the atomic's round trip overlaps the scan and the
+  // local sort
   const uint32_t *seg = meta + 1;
+  const bool reg_base = SPREAD && D1 <= blockDim.x;
+  uint32_t my_base = 0;
   for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
     uint32_t run = 0;
 #pragma unroll
@@ -303,8 +308,13 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
       run += c;
     }
     loff[d] = run;
-    if (SPREAD) gbase[d] = run ? d * cap + atomicAdd(cursor + d, run) : 0u;
-    else gbase[d] = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
+    if (SPREAD) {
+      const uint32_t b = run ? d * cap + atomicAdd(cursor + d, run) : 0u;
+      if (reg_base) my_base = b;
+      else gbase[d] = b;
+    } else {
+      gbase[d] = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
+    }
   }
   __syncthreads();
   block_scan_256(loff, D1);  // exclusive scan of the chunk totals over decoders
@@ -317,6 +327,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
     sidx[lp] = (uint16_t)(wbase + it * 32 + lane);
     sdec[lp] = (uint16_t)d;
   }
+  if (reg_base && threadIdx.x < D1) gbase[threadIdx.x] = my_base;
   __syncthreads();
   // coalesced copy-out: consecutive slots of one decoder go to consecutive
   // positions of that decoder's segment
