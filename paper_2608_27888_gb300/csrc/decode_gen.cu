@@ -233,10 +233,11 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
         abort_flag = 1;
       }
     };
-    // the MMA chain: one warp polls without suspending (lower wake-up
-    // latency), the named barrier releases the rest of the warpgroup
+    // the MMA chain: one warp waits (suspended in the barrier wait, so it
+    // takes no issue slots from the producer), the named barrier releases the
+    // rest of the warpgroup
     auto wait_mma = [&]() {
-      if (row < 32 && !mbar_spin(mma_bar, mph)) {
+      if (row < 32 && !mbar_wait(mma_bar, mph)) {
         atomicOr(status, 1u);
         abort_flag = 1;
       }

@@ -428,7 +428,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     // ------------------------------------------------------------ consumer
     const int c = role - NP;
     const int wgid = role;  // named barrier id role + 1
-    const bool poller = (row >> 5) == (c & 3);  // pollers spread over the sub-partitions
+    const bool poller = (row >> 5) == (c & 3);  // one waiting warp per consumer, spread over the sub-partitions
     const uint32_t tD = tmem_base + TC::acc(c);  // accumulator
     const uint32_t tH = tmem_base + TC::hid(c);  // hidden A operand
     const uint32_t tOnes = tmem_base + TC::ONES; // the bias K step's A operand
@@ -441,7 +441,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
     const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
     auto wait_bar = [&](uint32_t b, uint32_t parity) {
-      if (poller && !mbar_spin(b, parity)) {
+      if (poller && !mbar_wait(b, parity)) {
         atomicOr(status, 1u);
         *abort_flag = 1;
       }
