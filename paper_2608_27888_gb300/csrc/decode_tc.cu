@@ -158,24 +158,21 @@ __device__ __forceinline__ void issue_level_hi(const Assets &A, const GridDesc *
   }
 }
 
-// acc[c/2] += w * tap[c] over the 8 channels of one tap, as packed fp32 pairs
-// (fma.rn.f32x2; the first tap multiplies, which rounds the same as an fma
-// into zero).
+// acc[c/2] += w * tap[c] over the 8 channels of one tap, in packed fp16 pairs
+// (the latents' own type; hfma2, the first tap multiplies): the feature row
+// becomes the fp16/bf16 A operand, so the blend needs no fp32 conversions.
 template <bool FIRST>
-__device__ __forceinline__ void accum_tap_x2(float2 (&acc)[4], uint4 raw, float w) {
-  const float2 ww = make_float2(w, w);
+__device__ __forceinline__ void accum_tap_x2(__half2 (&acc)[4], uint4 raw, float w) {
+  const __half2 ww = __float2half2_rn(w);
   const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
 #pragma unroll
-  for (int p = 0; p < 4; ++p) {
-    const float2 x = __half22float2(h[p]);
-    acc[p] = FIRST ? __fmul2_rn(ww, x) : __ffma2_rn(ww, x, acc[p]);
-  }
+  for (int p = 0; p < 4; ++p) acc[p] = FIRST ? __hmul2(ww, h[p]) : __hfma2(ww, h[p], acc[p]);
 }
 
 // Feature accumulation: acc[k][c/2] over the 8 channels of level k, all taps
 // of mip lo first (FIRST: the first tap multiplies), then those of mip lo + 1.
 template <bool FIRST>
-__device__ __forceinline__ void accum_taps(const Taps &tp, float2 (&acc)[kLevels][4]) {
+__device__ __forceinline__ void accum_taps(const Taps &tp, __half2 (&acc)[kLevels][4]) {
 #pragma unroll
   for (int k = 0; k < kLevels; ++k) {
     accum_tap_x2<FIRST>(acc[k], tp.raw[k * 4], tp.w[k * 4]);
@@ -185,11 +182,18 @@ __device__ __forceinline__ void accum_taps(const Taps &tp, float2 (&acc)[kLevels
 }
 
 template <bool BF16>
-__device__ __forceinline__ void pack_row(const float2 (&acc)[kLevels][4], uint32_t (&packed)[8]) {
+__device__ __forceinline__ void pack_row(const __half2 (&acc)[kLevels][4], uint32_t (&packed)[8]) {
 #pragma unroll
   for (int k = 0; k < kLevels; ++k)
 #pragma unroll
-    for (int p = 0; p < 4; ++p) packed[k * 4 + p] = pack<BF16>(acc[k][p].x, acc[k][p].y);
+    for (int p = 0; p < 4; ++p) {
+      if (BF16) {
+        const float2 x = __half22float2(acc[k][p]);
+        packed[k * 4 + p] = pack<true>(x.x, x.y);
+      } else {
+        packed[k * 4 + p] = *reinterpret_cast<const uint32_t *>(&acc[k][p]);
+      }
+    }
 }
 
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
@@ -392,7 +396,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
       if (bad)
         for (uint32_t cc = 0; cc < C; ++cc) out[(size_t)oi * C + cc] = __int_as_float(0x7fc00000);
-      float2 acc[kLevels][4];
+      __half2 acc[kLevels][4];
       accum_taps<true>(taps, acc);
       if (TRI) prefetch();
       if (TRI && __any_sync(0xFFFFFFFFu, good && mp.t > 0.0f)) {  // some row blends two mips
