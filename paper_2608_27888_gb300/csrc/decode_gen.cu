@@ -171,10 +171,17 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
       for (int i = 0; i < NW; ++i) pk[i] = 0u;
       if (good) {
         {
-          float fl[L * C];
-          gen_latents_t<L, C>(A, grids, q, fl);
+          __half2 hl[LW];
+          gen_latents_h2<L, C>(A, grids, q, hl);
 #pragma unroll
-          for (int i = 0; i < LW; ++i) pk[i] = pack<BF16>(fl[2 * i], fl[2 * i + 1]);
+          for (int i = 0; i < LW; ++i) {
+            if (BF16) {
+              const float2 x = __half22float2(hl[i]);
+              pk[i] = pack<true>(x.x, x.y);
+            } else {
+              pk[i] = *reinterpret_cast<const uint32_t *>(&hl[i]);
+            }
+          }
         }
         const uint32_t F = A.pe_frequencies;
         if (F) {

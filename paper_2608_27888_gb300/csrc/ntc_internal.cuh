@@ -351,6 +351,46 @@ __device__ __forceinline__ void gen_latents_t(const Assets &A, const GridDesc *g
   if (L == 2) gen_level<1, C, L * C>(A, g, lo, t, q, f);
 }
 
+// The latent features of a good query in packed fp16 pairs, h[i] = channels
+// (2i, 2i+1) of the L x C inputs: the tensor-core path's blend (hfma2 on the
+// fp16 latents; every tap load of a level is issued before any is consumed).
+template <int L, int C>
+__device__ __forceinline__ void gen_latents_h2(const Assets &A, const GridDesc *grids, const ntc_query &q,
+                                               __half2 (&h)[L * C / 2]) {
+  using Raw = typename std::conditional<C == 8, uint4, uint2>::type;
+#pragma unroll
+  for (int i = 0; i < L * C / 2; ++i) h[i] = __float2half2_rn(0.0f);
+  float t;
+  const int lo = select_mip(q.lod, A.num_mips, t);
+  const GridDesc *g = grids + (size_t)q.set_id * L * A.num_mips;
+  const bool two = t > 0.0f;
+#pragma unroll
+  for (int k = 0; k < L; ++k) {
+    unsigned long long idx[2][4];
+    float w[2][4];
+    grid_taps(g[k * A.num_mips + lo], q.u, q.v, A.address_mode, idx[0], w[0]);
+    if (two) grid_taps(g[k * A.num_mips + lo + 1], q.u, q.v, A.address_mode, idx[1], w[1]);
+    Raw raw[2][4];
+#pragma unroll
+    for (int m = 0; m < 2; ++m)
+#pragma unroll
+      for (int p = 0; p < 4; ++p)
+        if (m == 0 || two) raw[m][p] = __ldg(reinterpret_cast<const Raw *>(A.lat) + idx[m][p]);
+#pragma unroll
+    for (int m = 0; m < 2; ++m) {
+      if (m == 1 && !two) break;
+      const float s = !two ? 1.0f : (m == 0 ? __fsub_rn(1.0f, t) : t);
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const __half2 ww = __float2half2_rn(!two ? w[m][p] : w[m][p] * s);
+        const __half2 *x = reinterpret_cast<const __half2 *>(&raw[m][p]);
+#pragma unroll
+        for (int c = 0; c < C / 2; ++c) h[k * C / 2 + c] = __hfma2(ww, x[c], h[k * C / 2 + c]);
+      }
+    }
+  }
+}
+
 // The coordinates the taps see (the positional encoding's input).
 __device__ __forceinline__ void pe_coords(const Assets &A, const ntc_query &q, float &u, float &v) {
   u = A.address_mode == 0 ? __fsub_rn(q.u, floorf(q.u)) : q.u;
