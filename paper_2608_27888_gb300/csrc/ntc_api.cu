@@ -459,9 +459,14 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   // divergence to remove, so the tensor-core decode takes the queries in their
   // own order and nothing is sorted
   const bool shared = mode == NTC_MODE_BUCKETED && !fp32 && !c->general && c->D == 1;
-  // the tensor-core decodes need no stable order: single-pass bucketing
-  const bool spread = mode == NTC_MODE_BUCKETED && !fp32 && !shared && use_spread(c, n);
-  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st, spread ? ((size_t)c->D + 1) * n : n);
+  // the tensor-core decodes need no stable order: single-pass bucketing, when
+  // its per-decoder regions fit the budget and can be allocated
+  bool spread = mode == NTC_MODE_BUCKETED && !fp32 && !shared && use_spread(c, n);
+  if (spread && ensure_scratch(c, n, st, ((size_t)c->D + 1) * n) != NTC_OK) {
+    cudaGetLastError();  // an allocation failure is not sticky: fall back to the stable sort
+    spread = false;
+  }
+  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st, n);
   if (s != NTC_OK) return s;
   if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
   if (unsorted) {
