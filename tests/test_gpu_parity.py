@@ -400,3 +400,40 @@ def test_bucketing_with_the_most_decoders():
         assert np.array_equal(counts.cpu().numpy().astype(np.uint32), c)
         assert np.array_equal(tiles.cpu().numpy().astype(np.uint32), t)
     dec.close()
+
+
+@pytest.mark.parametrize("pattern", ["random", "same", "bad", "sparse"])
+def test_single_pass_bucketing_decodes_every_row(pattern):
+    """The tensor-core decode buckets in one unstable pass (per-decoder regions
+    reserved with atomics).  Every row of the output must be written exactly as
+    the oracle decodes it, over chunk boundaries and ragged tails, and the
+    reservations must be cleared for the next call (sizes vary call to call)."""
+    S, D = 40, 13
+    rng = np.random.default_rng(7)
+    m = rng.integers(0, D, S).astype(np.uint32)
+    a = tiny_assets([[(8, 8), (4, 4)]] * S, num_sets=S, num_decoders=D, set_to_decoder=m, hidden=64, out_dim=8)
+    dec = ntc().Decoder(a, "fp16")
+    for n in (1, 2047, 2048, 2049, 3 * 2048 + 77, 70001, 129):
+        if pattern == "random":
+            sets = rng.integers(0, S, n)
+        elif pattern == "same":
+            sets = np.full(n, 7)
+        elif pattern == "bad":
+            sets = rng.integers(0, S + 5, n)
+        else:
+            sets = rng.choice([1, 2], n)
+        q = np.zeros(n, dtype=W.QUERY_DTYPE)
+        q["set_id"] = sets
+        q["u"] = rng.random(n)
+        q["v"] = rng.random(n)
+        ref, nbad = oracle.decode(a, q)
+        out = torch.full((n, 8), -7.0, device="cuda")
+        dec.reset_error_count()
+        got = dec.decode(dq(q), out=out).cpu().numpy()
+        assert not (got == -7.0).any(), n
+        bad = np.isnan(ref).any(1)
+        assert np.array_equal(np.isnan(got).any(1), bad), n
+        if (~bad).any():
+            check_tc(got[~bad], ref[~bad], f"n={n}")
+        assert dec.error_count() == nbad
+    dec.close()
