@@ -221,7 +221,7 @@ struct TmSmem {
   // a valid row: n <= 2^32 - 256)
   static constexpr size_t oidx = weights + (size_t)NC * L::WIMG;
   static constexpr size_t bars = oidx + (size_t)S * 128 * 4;
-  static constexpr int nbars = 2 * S + 2 * NC;                          // full, empty, mma, weights
+  static constexpr int nbars = 2 * S + 3 * NC;                          // full, empty, mma, weights, output
   static constexpr size_t misc = bars + (size_t)nbars * 8;
   static constexpr size_t tiles = misc + 64;
   static constexpr size_t grids = tiles + 2 * kSmemTileTable * 4;
@@ -234,19 +234,23 @@ struct TmSmem {
 // then the layer-1 feature operands [128 x 16] of the NC * SC ring stages (8
 // columns each); last, one shared 8-column block holding a 1 in K column 0 and
 // zeros elsewhere: the A operand of every layer's bias K step (the decoder image
-// keeps each layer's bias as the first row of an extra 16-row K block).
+// keeps each layer's bias as the first row of an extra 16-row K block); then
+// each consumer's own 16-column accumulator for the output layer, so that the
+// next tile's layer 1 can run in the hidden accumulator meanwhile.
 template <int H, int NC, int SC>
 struct TmCols {
   static constexpr uint32_t HID = NC * H;
   static constexpr uint32_t STG = HID + NC * (H / 2);
   static constexpr uint32_t ONES = STG + NC * SC * 8;
-  static constexpr uint32_t used = ONES + 8;
+  static constexpr uint32_t OUT = (ONES + 8 + 15) / 16 * 16;
+  static constexpr uint32_t used = OUT + NC * 16;
   static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
   static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
   static __device__ __forceinline__ uint32_t acc(uint32_t c) { return c * H; }
   static __device__ __forceinline__ uint32_t hid(uint32_t c) { return HID + c * (H / 2); }
   // layer-1 A operand of stage s (= consumer * SC + st)
   static __device__ __forceinline__ uint32_t a1(uint32_t s) { return STG + 8 * s; }
+  static __device__ __forceinline__ uint32_t out(uint32_t c) { return OUT + 16 * c; }
 };
 
 // Warp-specialised gather-decode with tensor-memory operands.
@@ -436,9 +440,11 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t tD = tmem_base + TC::acc(c);  // accumulator
     const uint32_t tH = tmem_base + TC::hid(c);  // hidden A operand
     const uint32_t tOnes = tmem_base + TC::ONES; // the bias K step's A operand
+    const uint32_t tO = tmem_base + TC::out(c);  // the output layer's accumulator
     const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
     const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
-    uint32_t ph = 0, wph = 0, cur = 0xFFFFFFFFu;
+    const uint32_t obar = saddr(bars + 2 * S + 2 * NC + c);  // the output layer's completion
+    uint32_t ph = 0, wph = 0, oph = 0, cur = 0xFFFFFFFFu;
     TileWalk cwalk;
     cwalk.ident_n = B.identity_n;
     cwalk.cap = B.spread_cap;
@@ -465,9 +471,11 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       tmem_wait_st();
     };
     // Start tile k: its decoder's weights, wait for its A stage (with the
-    // rows' output indices) and issue layer 1.  Requires this
-    // consumer's previous tile to have finished all MMAs.
-    auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good) {
+    // rows' output indices) and issue layer 1.  Requires this consumer's
+    // previous tile to have read its hidden accumulator (its output layer may
+    // still run: that reads only the hidden operand and writes only tO).  The
+    // barrier also carries the decision to stop, the same for every warp.
+    auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good, bool &stop) {
       const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
       uint32_t start, len;
       cwalk.at(seg, tst, D, t, dec, start, len);
@@ -482,7 +490,9 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         wait_bar(wbar, wph);
         wph ^= 1;
       }
+      if (row == 0) stop_flag[c] = *abort_flag;
       wg_bar(wgid);
+      stop = stop_flag[c] != 0;
       oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[s * 128 + row];
       good = oi != 0xFFFFFFFFu;
       if (row == 0) {
@@ -499,10 +509,9 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       }
     };
     uint32_t k = c, dec = D, oi = 0;
-    bool good = false;
-    if (k < K) begin(k, dec, oi, good);
+    bool good = false, stop = false;
+    if (k < K) begin(k, dec, oi, good, stop);
     while (k < K) {
-      uint32_t o[16];
       if (dec < D) {
 #pragma unroll 1
         for (int layer = 0; layer < 2; ++layer) {
@@ -515,55 +524,64 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
           wg_bar(wgid);
           if (row == 0) {
             fence_after();
-            const uint64_t dW = layer == 0 ? dW2 : dW3;
-            const uint32_t id = layer == 0 ? id_hidden : id_out;
+            if (layer == 0) {
 #pragma unroll
-            for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW + 16 * kq, id, kq);
-            umma_ta(tD, tOnes, dW + 16 * (H / 16), id, 1);  // + bias
-            umma_commit(mbar);
+              for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
+              umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
+              umma_commit(mbar);
+            } else {
+#pragma unroll
+              for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, kq);
+              umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 1);  // + bias
+              umma_commit(obar);
+            }
           }
         }
-        wait_bar(mbar, ph);
-        ph ^= 1;
-        wg_bar(wgid);
-        fence_after();
-        tmem_ld16(tD + lanes, o);
-        tmem_wait_ld();
-        fence_before();
       }
-      // the next tile's layer 1 runs while this tile's outputs are written
+      // the next tile's layer 1 runs while this tile's output layer finishes
+      // and its outputs are written (the hidden accumulator has been read)
       const uint32_t kn = k + NC;
       uint32_t ndec = D, noi = 0;
-      bool ngood = false;
-      if (kn < K) begin(kn, ndec, noi, ngood);
-      if (dec < D && good) {
-        // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
-        float y[CP];
+      bool ngood = false, nstop = false;
+      if (kn < K && !stop) begin(kn, ndec, noi, ngood, nstop);
+      if (dec < D) {
+        uint32_t o[16];
+        wait_bar(obar, oph);
+        oph ^= 1;
+        wg_bar(wgid);
+        fence_after();
+        tmem_ld16(tO + lanes, o);
+        tmem_wait_ld();
+        fence_before();
+        if (good) {
+          // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
+          float y[CP];
 #pragma unroll
-        for (int cc = 0; cc < CP; ++cc) {
-          float th;
-          asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
-          y[cc] = fmaf(0.5f, th, 0.5f);
-        }
-        float *dst = out + (size_t)oi * C;
-        if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
-          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]), "f"(y[1]),
-                       "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
-                       : "memory");
-        } else {
+          for (int cc = 0; cc < CP; ++cc) {
+            float th;
+            asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
+            y[cc] = fmaf(0.5f, th, 0.5f);
+          }
+          float *dst = out + (size_t)oi * C;
+          if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
+            asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]),
+                         "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
+                         : "memory");
+          } else {
 #pragma unroll
-          for (int cc = 0; cc < CP; ++cc)
-            if (cc < (int)C) dst[cc] = y[cc];
+            for (int cc = 0; cc < CP; ++cc)
+              if (cc < (int)C) dst[cc] = y[cc];
+          }
         }
+      }
+      if (stop || nstop) {  // every warp of this warpgroup read the same flags
+        if (nstop && ndec < D) wait_bar(mbar, ph);  // the issued layer 1 ends before TMEM is released
+        break;
       }
       k = kn;
       dec = ndec;
       oi = noi;
       good = ngood;
-      // every warp of this warpgroup takes the same decision to stop
-      if (row == 0) stop_flag[c] = *abort_flag;
-      wg_bar(wgid);
-      if (stop_flag[c]) break;
     }
   }
   fence_before();
