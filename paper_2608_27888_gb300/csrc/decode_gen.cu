@@ -24,8 +24,11 @@
 namespace ntc {
 namespace {
 
+// act: 0 ReLU, 1 LeakyReLU, 2 LeakyReLU with 0 <= slope <= 1, where
+// max(x, slope * x) is the same function in two instructions
 template <bool BF16>
 __device__ __forceinline__ uint32_t pack_act(float lo, float hi, uint32_t act, float slope) {
+  if (act == 2) return pack<BF16>(fmaxf(lo, slope * lo), fmaxf(hi, slope * hi));
   if (act == 1) {
     lo = lo > 0.0f ? lo : slope * lo;
     hi = hi > 0.0f ? hi : slope * hi;
@@ -53,8 +56,10 @@ inline __host__ __device__ size_t gen_tables_off(uint32_t img_bytes) { return ((
 inline __host__ __device__ size_t gen_oidx_off(uint32_t img_bytes) {
   return gen_tables_off(img_bytes) + 2 * kGenTileTable * 4 + (size_t)kGenGrids * sizeof(GridDesc);
 }
+// two output-row slots per stage (by use parity): the producer's next use of a
+// stage writes the other slot, so no consumer warp reads a later tile's rows
 inline __host__ __device__ size_t gen_smem_bytes(uint32_t img_bytes) {
-  return gen_oidx_off(img_bytes) + (size_t)kGenStages * 128 * 4;
+  return gen_oidx_off(img_bytes) + (size_t)kGenStages * 2 * 128 * 4;
 }
 
 // Tensor memory: the accumulator (H columns), the hidden layers' A operand
@@ -78,6 +83,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
   __shared__ uint64_t bars[2 * kGenStages + 2];  // full[S], empty[S], MMA completion, weight copy
   __shared__ uint32_t tmem_slot;
   __shared__ volatile uint32_t abort_flag;
+  __shared__ volatile uint32_t stop_flag[2];  // the consumer's decision for tile j, in slot j & 1
   const uint32_t tid = threadIdx.x, row = tid & 127, wg = tid >> 7;
   const uint32_t lanes = ((row >> 5) * 32) << 16;  // this warp's TMEM lane quadrant
   constexpr int NF = L * C + 4 * kGenMaxPe;  // feature values this input layout can have
@@ -98,6 +104,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
     mbar_init(mma_bar, 1);
     mbar_init(w_bar, 1);
     abort_flag = 0;
+    stop_flag[0] = stop_flag[1] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
   if (tid < 32) {
@@ -218,7 +225,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
         }
         tmem_wait_st();
       }
-      oidx[s * 128 + row] = good ? oi : 0xFFFFFFFFu;
+      oidx[(s * 2 + (use & 1u)) * 128 + row] = good ? oi : 0xFFFFFFFFu;
       fence_before();
       __syncwarp();
       if ((row & 31) == 0) mbar_arrive(full_bar(s));
@@ -234,6 +241,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
     TileWalk cwalk;
     cwalk.cap = B.spread_cap;
     const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
+    const uint32_t act = G.activation == 1 && G.slope >= 0.0f && G.slope <= 1.0f ? 2u : G.activation;
     auto wait = [&](uint32_t bar, uint32_t parity) {
       if (!mbar_wait(bar, parity)) {
         atomicOr(status, 1u);
@@ -256,12 +264,13 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
       uint32_t dec, st, len;
       cwalk.at(seg, tst, D, blockIdx.x + j * grid, dec, st, len);
       if (row < 32) wait(full_bar(s), use & 1u);
+      // one decision to stop per tile, the same for every warp of the warpgroup
+      if (row == 0) stop_flag[j & 1] = abort_flag;
       wg_bar(1);
       fence_after();
-      const uint32_t oi = oidx[s * 128 + row];
+      if (stop_flag[j & 1]) break;
+      const uint32_t oi = oidx[(s * 2 + (use & 1u)) * 128 + row];
       const bool good = oi != 0xFFFFFFFFu;
-      wg_bar(1);  // every consumer thread has read its output row
-      if (abort_flag) break;
       if (dec >= D) {  // a tile of bad rows: nothing to multiply
         if (row == 0) mbar_arrive(empty_bar(s));
         continue;
@@ -292,16 +301,20 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
         // hidden layer l is in the accumulator: bias, activation, next A operand
         wait_mma();
         fence_after();
-        const float *bl = bias + l * H;
+        const float4 *bl = reinterpret_cast<const float4 *>(bias + l * H);  // 16-byte aligned
         if (H == 16) {
           uint32_t v[16];
           tmem_ld16(tAcc + lanes, v);
           tmem_wait_ld();
           uint32_t p[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[2 * i], __uint_as_float(v[2 * i + 1]) + bl[2 * i + 1],
-                                  G.activation, G.slope);
+          for (int i = 0; i < 4; ++i) {
+            const float4 b = bl[i];
+            p[2 * i] = pack_act<BF16>(__uint_as_float(v[4 * i]) + b.x, __uint_as_float(v[4 * i + 1]) + b.y, act,
+                                      G.slope);
+            p[2 * i + 1] = pack_act<BF16>(__uint_as_float(v[4 * i + 2]) + b.z, __uint_as_float(v[4 * i + 3]) + b.w,
+                                          act, G.slope);
+          }
           tmem_st8(tAH + lanes, p);
         } else {
           for (uint32_t c0 = 0; c0 < H; c0 += 32) {
@@ -310,16 +323,19 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
             tmem_wait_ld();
             uint32_t p[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
-              p[i] = pack_act<BF16>(__uint_as_float(v[2 * i]) + bl[c0 + 2 * i],
-                                    __uint_as_float(v[2 * i + 1]) + bl[c0 + 2 * i + 1], G.activation, G.slope);
+            for (int i = 0; i < 8; ++i) {
+              const float4 b = bl[c0 / 4 + i];
+              p[2 * i] = pack_act<BF16>(__uint_as_float(v[4 * i]) + b.x, __uint_as_float(v[4 * i + 1]) + b.y, act,
+                                        G.slope);
+              p[2 * i + 1] = pack_act<BF16>(__uint_as_float(v[4 * i + 2]) + b.z, __uint_as_float(v[4 * i + 3]) + b.w,
+                                            act, G.slope);
+            }
             tmem_st16(tAH + lanes + c0 / 2, p);
           }
         }
         tmem_wait_st();
         fence_before();
         wg_bar(1);
-        if (abort_flag) break;
         if (row == 0) {
           fence_after();
           const bool last = l + 1 == NL;
@@ -329,21 +345,29 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
           umma_commit(mma_bar);
         }
       }
-      if (abort_flag) break;
       wait_mma();
       fence_after();
       uint32_t o[16];
       tmem_ld16(tAcc + lanes, o);
       tmem_wait_ld();
       if (good) {
-        const float *bo = bias + NL * H;
+        const float4 *bo = reinterpret_cast<const float4 *>(bias + NL * H);
         float *dst = out + (size_t)oi * OC;
 #pragma unroll
-        for (int c = 0; c < 16; ++c)
-          if (c < (int)OC) dst[c] = 1.0f / (1.0f + expf(-(__uint_as_float(o[c]) + bo[c])));
+        for (int c = 0; c < 16; ++c) {
+          if (c < (int)OC) {
+            // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
+            const float4 b = bo[c / 4];
+            const float x = __uint_as_float(o[c]) + (c % 4 == 0 ? b.x : c % 4 == 1 ? b.y : c % 4 == 2 ? b.z : b.w);
+            float th;
+            asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * x));
+            dst[c] = fmaf(0.5f, th, 0.5f);
+          }
+        }
       }
+      // the next tile's barrier (after its stage is full) orders these reads of
+      // the accumulator before its layer 1 overwrites it
       fence_before();
-      wg_bar(1);  // the next tile overwrites the accumulator and the hidden operand
     }
   }
   fence_before();

@@ -217,10 +217,12 @@ struct TmSmem {
   using L = TcLayout<H>;
   static constexpr int S = NC * SC;                                     // stages in all rings
   static constexpr size_t weights = 0;                                  // per consumer
-  // per stage: 128 output rows, 0xFFFFFFFF for a row that is not good (never
-  // a valid row: n <= 2^32 - 256)
+  // per stage and use parity: 128 output rows, 0xFFFFFFFF for a row that is
+  // not good (never a valid row: n <= 2^32 - 256).  Two slots per stage: the
+  // producer's next use of a stage writes the other slot, so a consumer warp
+  // that reads late never sees the following tile's rows.
   static constexpr size_t oidx = weights + (size_t)NC * L::WIMG;
-  static constexpr size_t bars = oidx + (size_t)S * 128 * 4;
+  static constexpr size_t bars = oidx + (size_t)S * 2 * 128 * 4;
   static constexpr int nbars = 2 * S + 3 * NC;                          // full, empty, mma, weights, output
   static constexpr size_t misc = bars + (size_t)nbars * 8;
   static constexpr size_t tiles = misc + 64;
@@ -294,12 +296,13 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
   auto empty_bar = [&](uint32_t s) { return saddr(bars + S + s); };
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + M::misc);
   volatile uint32_t *abort_flag = tmem_slot + 1;
-  volatile uint32_t *stop_flag = tmem_slot + 2;  // [NC], each read only after its warpgroup's barrier
+  // [NC][2]: consumer c's decision to stop, written for its tile jc in slot jc & 1
+  volatile uint32_t *stop_flag = tmem_slot + 2;
   const uint32_t D = A.num_decoders, C = W.out_dim;
 
   // no stage has rows yet: a consumer that stops on a wait timeout reads
   // all-bad rows, never an uninitialised output index
-  for (uint32_t i = threadIdx.x; i < (uint32_t)S * 128; i += blockDim.x)
+  for (uint32_t i = threadIdx.x; i < (uint32_t)S * 2 * 128; i += blockDim.x)
     reinterpret_cast<uint32_t *>(smem + M::oidx)[i] = 0xFFFFFFFFu;
   const GridDesc *grids = A.pgrids;  // grid bases in the row-pair copy
   const uint32_t ngrids = A.num_sets * kLevels * A.num_mips;
@@ -315,7 +318,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     }
     for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), 1);
     *abort_flag = 0;
-    for (int i = 0; i < NC; ++i) stop_flag[i] = 0;
+    for (int i = 0; i < 2 * NC; ++i) stop_flag[i] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
   if (warp == 0) {
@@ -423,7 +426,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       fence_after();
       tmem_st8(tmem_base + TC::a1(s) + lanes, a);
       tmem_wait_st();
-      reinterpret_cast<uint32_t *>(smem + M::oidx)[s * 128 + row] = good ? oi : 0xFFFFFFFFu;
+      reinterpret_cast<uint32_t *>(smem + M::oidx)[(s * 2 + (n & 1)) * 128 + row] = good ? oi : 0xFFFFFFFFu;
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(full_bar(s));
@@ -490,10 +493,10 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         wait_bar(wbar, wph);
         wph ^= 1;
       }
-      if (row == 0) stop_flag[c] = *abort_flag;
+      if (row == 0) stop_flag[2 * c + (jc & 1)] = *abort_flag;
       wg_bar(wgid);
-      stop = stop_flag[c] != 0;
-      oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[s * 128 + row];
+      stop = stop_flag[2 * c + (jc & 1)] != 0;
+      oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[(s * 2 + (n & 1)) * 128 + row];
       good = oi != 0xFFFFFFFFu;
       if (row == 0) {
         fence_after();
