@@ -217,9 +217,19 @@ NTC_API ntc_status ntc_debug_bucket(ntc_ctx *ctx, const ntc_query *d_queries, si
 NTC_API size_t ntc_max_tiles(const ntc_ctx *ctx, size_t n);
 
 /* Number of bad queries decoded since creation or the last reset.  Synchronises
- * the device. */
+ * the device.  Returns NTC_ERR_CUDA (and still writes *count) when a kernel
+ * gave up one of its bounded waits since then (every mbarrier wait of the
+ * tcgen05 kernels and of the bucketing ends after 200 ms): that call's
+ * results are invalid, the context stays usable.  The reset clears both. */
 NTC_API ntc_status ntc_get_error_count(ntc_ctx *ctx, uint64_t *count);
 NTC_API ntc_status ntc_reset_error_count(ntc_ctx *ctx);
+
+/* Test of the failure path above: one thread waits, with the decode kernels'
+ * own bounded wait, for an mbarrier phase that nothing completes, gives up
+ * after the 200 ms limit and records it in the context's status word exactly
+ * as a decode kernel that gave up would.  Async on cuda_stream; nothing
+ * faults, traps or hangs. */
+NTC_API ntc_status ntc_debug_wait_timeout(ntc_ctx *ctx, void *cuda_stream);
 
 /* Stage timing.  When enabled, ntc_decode records CUDA events on its stream
  * before bucketing, between bucketing and the gather-decode, and after it.

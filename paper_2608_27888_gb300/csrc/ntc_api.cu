@@ -8,6 +8,7 @@
 #include <vector>
 
 #include "ntc_internal.cuh"
+#include "tcgen05.cuh"
 
 using namespace ntc;
 
@@ -242,6 +243,18 @@ ntc_status check_queries(const ntc_ctx *ctx, const void *q, size_t n) {
   if (n && !q) return fail(NTC_ERR_INVALID_ARG, "null query pointer");
   if (((uintptr_t)q & 15) != 0) return fail(NTC_ERR_INVALID_ARG, "query buffer is not 16-byte aligned");
   return NTC_OK;
+}
+
+// The failure path of every bounded wait, run on purpose: an mbarrier whose
+// phase 0 nothing completes (one expected arrival, none made), waited for with
+// the kernels' own mbar_wait, which returns false once kWaitLimitNs has passed;
+// the give-up sets status bit 0 as a decode kernel's would.
+__global__ void k_wait_timeout(unsigned int *status) {
+  __shared__ uint64_t bar;
+  const uint32_t b = ntc::saddr(&bar);
+  ntc::mbar_init(b, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  if (!ntc::mbar_wait(b, 0)) atomicOr(status, 1u);
 }
 
 }  // namespace
@@ -668,6 +681,16 @@ ntc_status ntc_reset_error_count(ntc_ctx *c) {
   CK(cudaDeviceSynchronize(), "synchronize");
   CK(cudaMemset(c->d_err, 0, sizeof(unsigned long long)), "error counter reset");
   CK(cudaMemset(c->d_status, 0, sizeof(unsigned int)), "status reset");
+  return NTC_OK;
+}
+
+ntc_status ntc_debug_wait_timeout(ntc_ctx *c, void *stream) {
+  if (!c) return fail(NTC_ERR_INVALID_ARG, "null context");
+  DeviceGuard g(c->device);
+  k_wait_timeout<<<1, 1, 0, (cudaStream_t)stream>>>(c->d_status);
+  c->launches += 1;
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "wait-timeout launch");
   return NTC_OK;
 }
 

@@ -28,7 +28,8 @@ MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucket
 EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps",
            "ntc_debug_features", "ntc_debug_bucket", "ntc_max_tiles", "ntc_get_error_count",
            "ntc_reset_error_count", "ntc_launch_count", "ntc_set_stage_timing", "ntc_stage_times",
-           "ntc_bucket_static", "ntc_kmeans_map", "ntc_last_error", "ntc_status_string")
+           "ntc_bucket_static", "ntc_kmeans_map", "ntc_debug_wait_timeout", "ntc_last_error",
+           "ntc_status_string")
 
 
 class ntc_desc(ctypes.Structure):
@@ -78,6 +79,7 @@ def _load():
         "ntc_max_tiles": ([P, S], S),
         "ntc_get_error_count": ([P, P], I),
         "ntc_reset_error_count": ([P], I),
+        "ntc_debug_wait_timeout": ([P, P], I),
         "ntc_launch_count": ([P], ctypes.c_uint64),
         "ntc_set_stage_timing": ([P, I], I),
         "ntc_stage_times": ([P, P], I),
@@ -145,6 +147,10 @@ def ntc_get_error_count(ctx) -> int:
 
 def ntc_reset_error_count(ctx):
     _check(_lib.ntc_reset_error_count(ctx))
+
+
+def ntc_debug_wait_timeout(ctx, stream=None):
+    _check(_lib.ntc_debug_wait_timeout(ctx, stream))
 
 
 def ntc_launch_count(ctx) -> int:
@@ -311,6 +317,11 @@ class Decoder:
 
     def reset_error_count(self):
         ntc_reset_error_count(self.ctx)
+
+    def debug_wait_timeout(self, stream=None):
+        """Make one bounded wait give up (a test of the failure path): the next
+        error_count() raises NtcError with NTC_ERR_CUDA until reset_error_count()."""
+        ntc_debug_wait_timeout(self.ctx, _stream(stream))
 
     def launches(self) -> int:
         return ntc_launch_count(self.ctx)

@@ -437,3 +437,22 @@ def test_single_pass_bucketing_decodes_every_row(pattern):
             check_tc(got[~bad], ref[~bad], f"n={n}")
         assert dec.error_count() == nbad
     dec.close()
+
+
+def test_a_wait_that_gives_up_is_reported_and_the_context_recovers():
+    """Every mbarrier wait is bounded (200 ms).  A wait that gives up records
+    it in the context's status word: error_count() then fails with
+    NTC_ERR_CUDA until the reset, and the context decodes correctly after."""
+    m = ntc()
+    w = small(2)
+    dec = decoder(2, None, "fp16")
+    dec.reset_error_count()
+    dec.debug_wait_timeout()
+    with pytest.raises(m.NtcError) as e:
+        dec.error_count()
+    assert e.value.status == m.NTC_ERR_CUDA
+    dec.reset_error_count()
+    assert dec.error_count() == 0
+    got = dec.decode(dq(w.queries)).cpu().numpy()
+    ref, _ = oracle_out(2)
+    check_tc(got, ref, "after a wait gave up")
