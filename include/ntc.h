@@ -85,9 +85,14 @@ typedef enum {
 } ntc_precision;
 
 /* Which decode path ntc_decode runs.
- * BUCKETED:     stable counting sort of the queries by decoder id, then the
- *               gather-decode over 128-query single-decoder tiles.  Tensor-core
- *               precisions run the tcgen05/TMEM kernel; FP32 runs FFMA.
+ * BUCKETED:     the queries are grouped by decoder id, then the gather-decode
+ *               runs over 128-query single-decoder tiles.  Tensor-core precisions
+ *               group in one unstable pass (see Memory above) and run the
+ *               tcgen05/TMEM kernel; FP32 groups with the stable counting sort
+ *               and runs FFMA.  With one decoder for all sets the tensor-core
+ *               decode takes the queries in their own order.  Each output row
+ *               depends only on its own query, so the grouping order never
+ *               changes an output.
  * DIVERGENT:    no sorting: each warp takes 32 consecutive queries and loops over
  *               its distinct decoders (the non-shared setting of Sec. 4.4).
  *               Tensor-core precisions only.

@@ -11,15 +11,18 @@
 //     row index, computes the bilinear taps of both latent grids (Sec. 3.1, the
 //     same fp32 operations as the reference addressing), fetches each bilinear
 //     row as one 32-byte load from the row-pair copy of the latents, blends in
-//     fp32 and stores the fp16/bf16 feature row [16] into its stage with
-//     tcgen05.st (warp q writes TMEM lanes 32q..32q+31, exactly its rows).
+//     packed fp16 (the latents' own type) and stores the fp16/bf16 feature row
+//     [16] into its stage with tcgen05.st (warp q writes TMEM lanes
+//     32q..32q+31, exactly its rows).
 //   Consumer (one elected thread issues every MMA): layer 1 reads A from the
 //     stage and B (the decoder's weights, copied by a TMA bulk copy whenever
 //     the decoder changes) from shared memory; its completion frees the stage;
 //     the ReLU/convert epilogue goes TMEM -> registers -> TMEM; layers 2 and 3
 //     read their A operand from TMEM too; each layer's bias is one more K step
-//     whose A is a shared block with a 1 in K column 0.  The sigmoid epilogue
-//     scatters rows to out[perm[i]] while the next tile's layer 1 runs.
+//     whose A is a shared block with a 1 in K column 0.  Layer 3 accumulates
+//     in the consumer's own 16 output columns, so the next tile's layer 1 is
+//     issued before it completes; the sigmoid epilogue then scatters rows to
+//     out[perm[i]].
 // Shared-memory B operands use the no-swizzle K-major canonical layout: 8-row
 // x 16-byte core matrices, K-adjacent core matrices 128 B apart (LBO), 8-row
 // groups K*16 B apart (SBO).  Every wait is bounded by time; on expiry the
@@ -265,16 +268,18 @@ struct TmCols {
 //   program order on both sides -- an mbarrier parity wait can then never be two
 //   phases ahead of its barrier.
 //   Producer: each thread computes the taps of one query row, blends them in
-//   fp32 and stores the fp16/bf16 feature row into the stage's TMEM A region
-//   (tcgen05.st; warp q of a warpgroup owns TMEM lanes 32q..32q+31, exactly its
-//   rows), with the row's output index (or 0xFFFFFFFF if the row is not good)
-//   in shared memory; four
+//   packed fp16 and stores the fp16/bf16 feature row into the stage's TMEM A
+//   region (tcgen05.st; warp q of a warpgroup owns TMEM lanes 32q..32q+31,
+//   exactly its rows), with the row's output index (or 0xFFFFFFFF if the row is
+//   not good) in shared memory, in the slot of the stage's use parity; four
 //   warp arrivals fill the stage.  The next tile's query record and output
 //   index are loaded while the current tile is gathered.
 //   Consumer: layer 1 reads A from the stage and B (weights) from shared memory;
 //   its completion empties the stage; the ReLU/convert epilogue goes TMEM ->
-//   registers -> TMEM; layers 2 and 3 read their A from TMEM too; the sigmoid
-//   epilogue scatters rows to out[perm[i]] while the next tile's layer 1 runs.
+//   registers -> TMEM; layers 2 and 3 read their A from TMEM too.  Layer 3
+//   writes the consumer's own output columns and completes on its own
+//   barrier, so the next tile's layer 1 is issued first; then the sigmoid
+//   epilogue scatters rows to out[perm[i]].
 // CTA b owns the global tiles b, b + grid, b + 2 grid, ...
 template <int H, bool BF16, bool TRI, bool WRAP, int CP, int NP, int NC, int SC>
 __global__ void __launch_bounds__((NP + NC) * 128, 1)
