@@ -146,11 +146,18 @@ def peaks():
         return 6800.0, "fallback"
 
 
-def kernel_source_hash():
-    """Hash of the decode kernels' code with comments and blank space removed,
-    so a comment edit does not detach the recorded DRAM traffic."""
+# the sources each recorded decode kernel is built from
+KERNEL_SOURCES = {
+    "bucketed-fp16": ("decode_tc.cu", "tcgen05.cuh", "ntc_internal.cuh"),
+    "bucketed-fp16-paper-decoder": ("decode_gen.cu", "tcgen05.cuh", "ntc_internal.cuh"),
+}
+
+
+def kernel_source_hash(kernel_tag):
+    """Hash of one decode kernel's sources with comments and blank space
+    removed, so a comment edit does not detach the recorded DRAM traffic."""
     h = hashlib.sha1()
-    for f in ("decode_tc.cu", "decode_gen.cu", "tcgen05.cuh", "ntc_internal.cuh"):
+    for f in KERNEL_SOURCES[kernel_tag]:
         with open(os.path.join(ROOT, "paper_2608_27888_gb300", "csrc", f)) as fh:
             src = fh.read()
         src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
@@ -167,7 +174,7 @@ def recorded_traffic(kernel_tag):
         with open(path) as f:
             rec = json.load(f)
         r = rec.get(kernel_tag)
-        if r and r.get("source_hash") == kernel_source_hash():
+        if r and kernel_tag in KERNEL_SOURCES and r.get("source_hash") == kernel_source_hash(kernel_tag):
             return float(r["dram_bytes_per_launch"])
     except Exception:
         pass

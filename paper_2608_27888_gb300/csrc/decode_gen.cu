@@ -192,10 +192,13 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
         }
         const uint32_t F = A.pe_frequencies;
         if (F) {
+          // sin/cos(2 pi u) from the hardware approximation, after reducing u
+          // to [-1/2, 1/2] (exact), where its absolute error is about 2^-21:
+          // far below the fp16/bf16 rounding the features then go through
           float u, v, su, cu, sv, cv;
           pe_coords(A, q, u, v);
-          sincospif(2.0f * u, &su, &cu);
-          sincospif(2.0f * v, &sv, &cv);
+          __sincosf(6.28318530718f * __fsub_rn(u, rintf(u)), &su, &cu);
+          __sincosf(6.28318530718f * __fsub_rn(v, rintf(v)), &sv, &cv);
 #pragma unroll
           for (int k = 0; k < kGenMaxPe; ++k) {
             if (LW + 2 * k + 1 >= NW) break;
