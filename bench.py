@@ -43,7 +43,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "decoded queries/sec on 1 GB300 vs distinct decoders per warp; % of roofline"
 UNIT = "queries/s"
-WORKLOAD = ("config2: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16), 16 decoders "
+WORKLOAD = ("uniform-4m: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16), 16 decoders "
             "16->64->64->8 (one per set), 4,194,304 queries: uniform set id, uniform UV, lod 0")
 L2_FLUSH_BYTES = 256 << 20
 KERNEL_NAMES = {("bucketed", False): "k_decode_tc (tcgen05/TMEM gather-decode)",
@@ -69,10 +69,10 @@ def parse():
                    help="also decode a 586-set workload under the five groupings of Table 2")
     p.add_argument("--variants", action="store_true",
                    help="also time Sec. 4's decoder and the A x B sizes of its MLP ablation")
-    p.add_argument("--configs", action="store_true",
-                   help="also time every full-size workload (1-5 and their maps); adds about two minutes")
+    p.add_argument("--workloads", action="store_true",
+                   help="also time every full-size named workload and its groupings; adds about two minutes")
     p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
-    p.add_argument("--workload", default="config2", choices=["config2", "paper-decoder"],
+    p.add_argument("--workload", default="uniform-4m", choices=["uniform-4m", "paper-decoder"],
                    help="the timed batch: the 4M-query 16-decoder workload (default), or Sec. 4's "
                         "decoder (256^2x4 grid, positional encoding, LeakyReLU, 64x3) on a 1080p G-buffer")
     return p.parse_args()
@@ -200,7 +200,7 @@ def shape_costs(a, q):
     return bpq, flops, w_bytes
 
 
-def workload(small: bool, rank: int, name: str = "config2"):
+def workload(small: bool, rank: int, name: str = "uniform-4m"):
     """The benchmark batch of one rank: the same assets on every rank, a
     rank-specific query stream (queries are sharded, assets replicated)."""
     from paper_2608_27888_gb300 import workloads as W
@@ -210,7 +210,7 @@ def workload(small: bool, rank: int, name: str = "config2"):
     S, T, n = (16, 128, 40_077) if small else (16, 1024, 4_194_304)
     a = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
     q = W.queries_uniform(seed + 1000 * rank, n, S)
-    return W.Workload("config2-small" if small else "config2-full", a, q, {})
+    return W.Workload("uniform-4m-small" if small else "uniform-4m-full", a, q, {})
 
 
 def aggregate(n_per_rank: int, ms_local: float, dist=None):
@@ -259,7 +259,7 @@ def run_reference(args, ws, rank):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD if args.workload == "config2" else w.name, "sample_queries": sample},
+        "config": {"workload": WORKLOAD if args.workload == "uniform-4m" else w.name, "sample_queries": sample},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
@@ -341,10 +341,10 @@ def main():
     bpq, flops_q, w_bytes = shape_costs(w.assets, w.queries)
     alg_bytes = n * bpq + w_bytes
     achieved = alg_bytes / (decode_ms / 1e3) / 1e9
-    kernel_tag = f"{args.mode}-{args.precision}" + ("" if args.workload == "config2" else f"-{args.workload}")
+    kernel_tag = f"{args.mode}-{args.precision}" + ("" if args.workload == "uniform-4m" else f"-{args.workload}")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": recorded_traffic(kernel_tag),
-                "kernel": KERNEL_NAMES[(args.mode, args.precision == "fp32")] if args.workload == "config2"
+                "kernel": KERNEL_NAMES[(args.mode, args.precision == "fp32")] if args.workload == "uniform-4m"
                 else "k_decode_gen_tc (general-shape tcgen05 gather-decode)",
                 "kernel_ms": decode_ms, "bucketing_ms": bucket_ms,
                 "peak_kind": f"{peak_kind} HBM copy bandwidth",
@@ -368,7 +368,7 @@ def main():
     # the in-run comparison: the unsorted divergent kernel on the same batch
     extra = {}
     for other in ("divergent", "divergent_fma"):
-        if args.mode == other or (other == "divergent" and (args.precision == "fp32" or args.workload != "config2")):
+        if args.mode == other or (other == "divergent" and (args.precision == "fp32" or args.workload != "uniform-4m")):
             continue
         dms, _, _ = timed_steps(other, max(5, args.steps // 2), 2)
         extra[other] = {"value": n * ws / (statistics.mean(dms) / 1e3), "unit": UNIT,
@@ -382,7 +382,7 @@ def main():
         "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f16" if args.precision == "fp16" else args.precision.replace("fp", "f"),
         "data": "synthetic",
-        "config": {"workload": (WORKLOAD if args.workload == "config2" else w.name) if not args.small else w.name,
+        "config": {"workload": (WORKLOAD if args.workload == "uniform-4m" else w.name) if not args.small else w.name,
                    "queries_per_gpu": n,
                    "decoders": w.assets.num_decoders, "mode": args.mode, "precision": args.precision,
                    "mean_distinct_decoders_per_warp": dd,
@@ -397,8 +397,8 @@ def main():
         result["sweep"] = sweep(ntc, torch, args.precision)
     if not args.no_mirror and not args.small and rank == 0 and args.precision != "fp32":
         result["paper_mirror"] = paper_mirror(ntc, torch, args.precision)
-    if args.configs and rank == 0:
-        result["configs"] = per_config(ntc, torch, args.precision)
+    if args.workloads and rank == 0:
+        result["workloads"] = per_workload(ntc, torch, args.precision)
     if args.maps and rank == 0:
         result["maps"] = map_sources(ntc, torch, args.precision)
     if args.variants and rank == 0:
@@ -552,7 +552,7 @@ def map_sources(ntc, torch, precision):
             "what": "586 sets of 1024^2, 1920x1080 G-buffer, 600 regions; Gq/s of the whole ntc_decode"}
 
 
-def per_config(ntc, torch, precision):
+def per_workload(ntc, torch, precision):
     """Every full-size workload: queries/s of the whole ntc_decode (bucketed),
     the bucketing / gather-decode split, the unsorted kernels, and the whole
     step against the roofline rate of that workload's algorithmic bytes."""
@@ -561,9 +561,11 @@ def per_config(ntc, torch, precision):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     rows = []
-    for k, variant in ((1, None), (2, None), (3, "identity"), (3, "clustered4"), (3, "shared"),
-                       (4, "128"), (4, "16"), (4, "8"), (4, "1"), (5, None)):
-        w = W.config(k, "full", variant)
+    for name, variant in (("raster-256", None), ("uniform-4m", None), ("gbuffer-1080p", "identity"),
+                          ("gbuffer-1080p", "clustered4"), ("gbuffer-1080p", "shared"), ("gbuffer-2160p", "128"),
+                          ("gbuffer-2160p", "16"), ("gbuffer-2160p", "8"), ("gbuffer-2160p", "1"),
+                          ("gbuffer-2160p-x4-trilinear", None)):
+        w = W.named(name, "full", variant)
         a, q = w.assets, w.queries
         n, C = len(q), a.out_dim
         dec = ntc.Decoder(a, precision)

@@ -270,27 +270,42 @@ def make_assets(seed, num_sets, T, num_mips, num_decoders, set_to_decoder, hidde
 
 # --------------------------------------------------------------- named workloads
 #
-# full  = the sizes of the five workload configurations (1: one 256^2 set; 2: 16
-#         sets of 1024^2, 4M uniform queries; 3: 1080p G-buffer over 32 sets;
-#         4: 2160p G-buffer over 128 sets of 2048^2; 5: 512 sets of 2048^2,
-#         4 frames of 2160p with trilinear mips);
+# full  = the sizes of the five workloads:
+#   raster-256                  one 256^2 set, one decoder, a texel-centre raster;
+#   uniform-4m                  16 sets of 1024^2, a decoder per set, 4,194,304
+#                               queries with uniform set id and UV;
+#   gbuffer-1080p               a 1920x1080 G-buffer over 32 sets of 1024^2 (4 mips);
+#   gbuffer-2160p               a 3840x2160 G-buffer over 128 sets of 2048^2;
+#   gbuffer-2160p-x4-trilinear  4 frames of 3840x2160 over 512 sets of 2048^2,
+#                               16->128->128->9 decoders, continuous lods;
 # small = the same recipes shrunk so the oracle finishes in seconds, still
 #         spanning many 128-query tiles and a ragged tail.
 
-def config(k: int, size: str = "full", variant: str | None = None) -> Workload:
-    seed = BASE_SEED + k
+# seed offset of each named workload (the generated inputs depend on it)
+_SEED = {"raster-256": 1, "uniform-4m": 2, "gbuffer-1080p": 3, "gbuffer-2160p": 4,
+         "gbuffer-2160p-x4-trilinear": 5}
+WORKLOADS = tuple(_SEED)
+
+
+def named(name: str, size: str = "full", variant: str | None = None) -> Workload:
+    """One of WORKLOADS.  variant: the set->decoder grouping of gbuffer-1080p
+    ("identity", "clustered4", "shared") or the decoder count of gbuffer-2160p
+    ("128", "16", "8", "1")."""
+    if name not in _SEED:
+        raise ValueError(f"unknown workload {name}")
+    seed = BASE_SEED + _SEED[name]
     full = size == "full"
-    if k == 1:
+    if name == "raster-256":
         T = 256 if full else 64
         a = make_assets(seed, 1, T, 1, 1, map_shared(1))
         q = queries_texel_centres(T, 0)
-        return Workload(f"config1-{size}", a, q, {"T": T, "maps": "shared"})
-    if k == 2:
+        return Workload(f"{name}-{size}", a, q, {"T": T, "maps": "shared"})
+    if name == "uniform-4m":
         S, T, n = (16, 1024, 4_194_304) if full else (16, 128, 40_000 + 77)
         a = make_assets(seed, S, T, 1, S, map_identity(S))
         q = queries_uniform(seed, n, S)
-        return Workload(f"config2-{size}", a, q, {"T": T, "maps": "identity"})
-    if k == 3:
+        return Workload(f"{name}-{size}", a, q, {"T": T, "maps": "identity"})
+    if name == "gbuffer-1080p":
         S, T = 32, (1024 if full else 128)
         W, H, R = (1920, 1080, 200) if full else (240, 136, 40)
         variant = variant or "identity"
@@ -299,23 +314,21 @@ def config(k: int, size: str = "full", variant: str | None = None) -> Workload:
         D = {"identity": S, "clustered4": 4, "shared": 1}[variant]
         a = make_assets(seed, S, T, 4, D, m)
         q = queries_gbuffer(seed, W, H, R, S, T, lod_mode=0)
-        return Workload(f"config3-{size}-{variant}", a, q, {"T": T, "maps": variant})
-    if k == 4:
+        return Workload(f"{name}-{size}-{variant}", a, q, {"T": T, "maps": variant})
+    if name == "gbuffer-2160p":
         S, T = (128, 2048) if full else (128, 64)
         W, H, R = (3840, 2160, 800) if full else (320, 180, 120)
         D = int(variant or 128)
         m = map_identity(S) if D == S else map_random_partition(seed, S, D)
         a = make_assets(seed, S, T, 4, D, m, out_dim=9)
         q = queries_gbuffer(seed, W, H, R, S, T, lod_mode=0)
-        return Workload(f"config4-{size}-{D}", a, q, {"T": T, "maps": f"random{D}"})
-    if k == 5:
-        S, T = (512, 2048) if full else (24, 128)
-        W, H, R, F = (3840, 2160, 2000, 4) if full else (256, 128, 60, 2)
-        D = 8
-        a = make_assets(seed, S, T, 4, D, map_random_partition(seed, S, D), hidden=128, out_dim=9)
-        q = queries_gbuffer(seed, W, H, R, S, T, lod_mode=1, lod_max=3.0, frames=F)
-        return Workload(f"config5-{size}", a, q, {"T": T, "maps": "random8", "frames": F})
-    raise ValueError(f"unknown workload {k}")
+        return Workload(f"{name}-{size}-{D}", a, q, {"T": T, "maps": f"random{D}"})
+    S, T = (512, 2048) if full else (24, 128)
+    W, H, R, F = (3840, 2160, 2000, 4) if full else (256, 128, 60, 2)
+    D = 8
+    a = make_assets(seed, S, T, 4, D, map_random_partition(seed, S, D), hidden=128, out_dim=9)
+    q = queries_gbuffer(seed, W, H, R, S, T, lod_mode=1, lod_max=3.0, frames=F)
+    return Workload(f"{name}-{size}", a, q, {"T": T, "maps": "random8", "frames": F})
 
 
 def paper_decoder(size: str = "full", hidden=64, layers=2, levels=1, channels=4, pe=4, activation=1,

@@ -20,8 +20,10 @@ pytestmark = pytest.mark.gpu
 
 FP32_TOL = 1e-5
 TC_MAX, TC_MEAN = 2e-2, 2e-3
-SMALL = [(1, None), (2, None), (3, "identity"), (3, "clustered4"), (3, "shared"), (4, "128"), (4, "16"),
-         (4, "8"), (4, "1"), (5, None)]
+SMALL = [("raster-256", None), ("uniform-4m", None), ("gbuffer-1080p", "identity"),
+         ("gbuffer-1080p", "clustered4"), ("gbuffer-1080p", "shared"), ("gbuffer-2160p", "128"),
+         ("gbuffer-2160p", "16"), ("gbuffer-2160p", "8"), ("gbuffer-2160p", "1"),
+         ("gbuffer-2160p-x4-trilinear", None)]
 
 
 def ntc():
@@ -30,19 +32,19 @@ def ntc():
 
 
 @functools.lru_cache(maxsize=None)
-def small(k, variant=None):
-    return W.config(k, "small", variant)
+def small(name, variant=None):
+    return W.named(name, "small", variant)
 
 
 @functools.lru_cache(maxsize=None)
-def oracle_out(k, variant=None):
-    w = small(k, variant)
+def oracle_out(name, variant=None):
+    w = small(name, variant)
     return oracle.decode(w.assets, w.queries)
 
 
 @functools.lru_cache(maxsize=4)
-def decoder(k, variant, precision):
-    return ntc().Decoder(small(k, variant).assets, precision)
+def decoder(name, variant, precision):
+    return ntc().Decoder(small(name, variant).assets, precision)
 
 
 def dq(q):
@@ -58,10 +60,10 @@ def check_tc(got, ref, what):
 
 # --------------------------------------------------------------- bucketing
 
-@pytest.mark.parametrize("k,variant", SMALL)
-def test_bucketing_bit_exact(k, variant):
-    w = small(k, variant)
-    dec = decoder(k, variant, "fp16")
+@pytest.mark.parametrize("name,variant", SMALL)
+def test_bucketing_bit_exact(name, variant):
+    w = small(name, variant)
+    dec = decoder(name, variant, "fp16")
     perm, counts, tiles = dec.bucket(dq(w.queries))
     p, c, o, t = oracle.bucket(w.queries["set_id"], w.assets.set_to_decoder, w.assets.num_decoders)
     assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
@@ -110,10 +112,11 @@ def _taps_equal(dec, a, q):
     assert np.array_equal(t.cpu().numpy().view(np.uint32), rt.view(np.uint32))
 
 
-@pytest.mark.parametrize("k,variant", [(1, None), (2, None), (3, "identity"), (4, "128"), (5, None)])
-def test_taps_bit_exact(k, variant):
-    w = small(k, variant)
-    _taps_equal(decoder(k, variant, "fp16"), w.assets, w.queries)
+@pytest.mark.parametrize("name,variant", [("raster-256", None), ("uniform-4m", None), ("gbuffer-1080p", "identity"),
+                                          ("gbuffer-2160p", "128"), ("gbuffer-2160p-x4-trilinear", None)])
+def test_taps_bit_exact(name, variant):
+    w = small(name, variant)
+    _taps_equal(decoder(name, variant, "fp16"), w.assets, w.queries)
 
 
 @pytest.mark.parametrize("mode", [0, 1])
@@ -156,10 +159,10 @@ def test_decode_tc_tiny_grids_edges(mode, dims, mips):
         dec.close()
 
 
-@pytest.mark.parametrize("k,variant", [(2, None), (5, None)])
-def test_features_match_oracle(k, variant):
-    w = small(k, variant)
-    f = decoder(k, variant, "fp16").features(dq(w.queries)).cpu().numpy()
+@pytest.mark.parametrize("name,variant", [("uniform-4m", None), ("gbuffer-2160p-x4-trilinear", None)])
+def test_features_match_oracle(name, variant):
+    w = small(name, variant)
+    f = decoder(name, variant, "fp16").features(dq(w.queries)).cpu().numpy()
     ref = oracle.features(w.assets, w.queries)
     assert np.abs(f - ref).max() <= 1e-5 * max(1.0, np.abs(ref).max())
 
@@ -167,31 +170,31 @@ def test_features_match_oracle(k, variant):
 # --------------------------------------------------------------- decode
 
 @pytest.mark.parametrize("mode", ["bucketed", "divergent_fma"])
-@pytest.mark.parametrize("k,variant", SMALL)
-def test_decode_fp32_mode(k, variant, mode):
-    w = small(k, variant)
-    ref, _ = oracle_out(k, variant)
-    got = decoder(k, variant, "fp32").decode(dq(w.queries), mode=mode).cpu().numpy()
+@pytest.mark.parametrize("name,variant", SMALL)
+def test_decode_fp32_mode(name, variant, mode):
+    w = small(name, variant)
+    ref, _ = oracle_out(name, variant)
+    got = decoder(name, variant, "fp32").decode(dq(w.queries), mode=mode).cpu().numpy()
     assert np.abs(got - ref).max() <= FP32_TOL
 
 
 @pytest.mark.parametrize("precision", ["fp16", "bf16"])
 @pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent", "divergent_fma"])
-@pytest.mark.parametrize("k,variant", SMALL)
-def test_decode_tensor_core_modes(k, variant, mode, precision):
-    w = small(k, variant)
-    ref, _ = oracle_out(k, variant)
-    got = decoder(k, variant, precision).decode(dq(w.queries), mode=mode).cpu().numpy()
-    check_tc(got, ref, f"config {k}/{variant} {mode} {precision}")
+@pytest.mark.parametrize("name,variant", SMALL)
+def test_decode_tensor_core_modes(name, variant, mode, precision):
+    w = small(name, variant)
+    ref, _ = oracle_out(name, variant)
+    got = decoder(name, variant, precision).decode(dq(w.queries), mode=mode).cpu().numpy()
+    check_tc(got, ref, f"{name}/{variant} {mode} {precision}")
 
 
 def test_hidden_128_and_9_channels_on_all_paths():
-    w = small(5)
-    ref, _ = oracle_out(5)
+    w = small("gbuffer-2160p-x4-trilinear")
+    ref, _ = oracle_out("gbuffer-2160p-x4-trilinear")
     for prec, modes in (("fp32", ["bucketed", "divergent_fma"]),
                         ("fp16", ["bucketed", "bucketed_mma", "divergent", "divergent_fma"]),
                         ("bf16", ["divergent_fma"])):
-        dec = decoder(5, None, prec)
+        dec = decoder("gbuffer-2160p-x4-trilinear", None, prec)
         for m in modes:
             got = dec.decode(dq(w.queries), mode=m).cpu().numpy()
             if prec == "fp32":
@@ -202,8 +205,8 @@ def test_hidden_128_and_9_channels_on_all_paths():
 
 @pytest.mark.parametrize("mode", ["bucketed", "bucketed_mma", "divergent", "divergent_fma"])
 def test_order_invariance_is_bitwise(mode):
-    w = small(3, "clustered4")
-    dec = decoder(3, "clustered4", "fp16")
+    w = small("gbuffer-1080p", "clustered4")
+    dec = decoder("gbuffer-1080p", "clustered4", "fp16")
     out = dec.decode(dq(w.queries), mode=mode).cpu().numpy()
     p = np.random.default_rng(1).permutation(len(w.queries))
     out2 = dec.decode(dq(w.queries[p]), mode=mode).cpu().numpy()
@@ -213,7 +216,7 @@ def test_order_invariance_is_bitwise(mode):
 
 
 def test_bad_queries_nan_and_counted():
-    w = small(2)
+    w = small("uniform-4m")
     q = w.queries[:5000].copy()
     q["set_id"][::97] = 999
     q["u"][5::101] = np.nan
@@ -233,8 +236,8 @@ def test_bad_queries_nan_and_counted():
 
 
 def test_decode_host_equals_device_decode():
-    w = small(3, "identity")
-    dec = decoder(3, "identity", "fp16")
+    w = small("gbuffer-1080p", "identity")
+    dec = decoder("gbuffer-1080p", "identity", "fp16")
     dev = dec.decode(dq(w.queries)).cpu().numpy()
     hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
     host = dec.decode_host(hq).numpy()
@@ -243,27 +246,28 @@ def test_decode_host_equals_device_decode():
 
 def test_empty_and_invalid_calls():
     m = ntc()
-    dec = decoder(1, None, "fp16")
+    dec = decoder("raster-256", None, "fp16")
     empty = torch.empty((0, 4), dtype=torch.int32, device="cuda")
     out = dec.decode(empty)
     assert out.shape == (0, 8)
     with pytest.raises(m.NtcError):
         m.ntc_decode(dec.ctx, 0, 10, 0, 0, m.NTC_MODE_BUCKETED)
     with pytest.raises(m.NtcError):
-        fp32 = decoder(1, None, "fp32")
-        fp32.decode(dq(small(1).queries[:64]), mode="divergent")
+        fp32 = decoder("raster-256", None, "fp32")
+        fp32.decode(dq(small("raster-256").queries[:64]), mode="divergent")
 
 
 # ------------------------------------------------- full sizes, sampled check
 
-FULL = [(1, None), (2, None), (3, "identity"), (4, "128"), (5, None)]
+FULL = [("raster-256", None), ("uniform-4m", None), ("gbuffer-1080p", "identity"), ("gbuffer-2160p", "128"),
+        ("gbuffer-2160p-x4-trilinear", None)]
 
 
-@pytest.mark.parametrize("k,variant", FULL)
-def test_full_size_sampled(k, variant):
-    w = W.config(k, "full", variant)
+@pytest.mark.parametrize("name,variant", FULL)
+def test_full_size_sampled(name, variant):
+    w = W.named(name, "full", variant)
     n = len(w.queries)
-    rng = np.random.default_rng(k)
+    rng = np.random.default_rng(W.WORKLOADS.index(name) + 1)
     sample = np.unique(np.concatenate([rng.integers(0, n, 20000), np.arange(min(n, 4096)),
                                        np.arange(max(0, n - 300), n)]))
     ref, _ = oracle.decode(w.assets, w.queries[sample])
@@ -271,10 +275,10 @@ def test_full_size_sampled(k, variant):
     dec = ntc().Decoder(w.assets, "fp16")
     out = dec.decode(qd, mode="bucketed")
     got = out[torch.from_numpy(sample).cuda()].cpu().numpy()
-    check_tc(got, ref, f"config {k} full bucketed")
+    check_tc(got, ref, f"{w.name} bucketed")
     for mode in ("divergent", "divergent_fma"):
         div = dec.decode(qd, mode=mode)[torch.from_numpy(sample).cuda()].cpu().numpy()
-        check_tc(div, ref, f"config {k} full {mode}")
+        check_tc(div, ref, f"{w.name} {mode}")
     perm, counts, tiles = dec.bucket(qd)
     p, c, _, t = oracle.bucket(w.queries["set_id"], w.assets.set_to_decoder, w.assets.num_decoders)
     assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
@@ -323,13 +327,13 @@ def _coherent_case(kind, n, rng, assets, base):
 def test_single_decoder_and_mixed_warps(kind, n, variant):
     """With one shared decoder ("shared") the tensor-core path sorts nothing and
     decodes the queries in their own order; with four it buckets them."""
-    base_w = small(3, variant)
+    base_w = small("gbuffer-1080p", variant)
     a = base_w.assets
     rng = np.random.default_rng(n * 7 + len(kind))
     base = np.resize(base_w.queries, max(n, 1))
     q = _coherent_case(kind, n, rng, a, base)
     ref, nbad = oracle.decode(a, q)
-    dec = decoder(3, variant, "fp16")
+    dec = decoder("gbuffer-1080p", variant, "fp16")
     dec.reset_error_count()
     got = dec.decode(dq(q), mode="bucketed").cpu().numpy()
     assert np.array_equal(np.isnan(got), np.isnan(ref))
@@ -444,8 +448,8 @@ def test_a_wait_that_gives_up_is_reported_and_the_context_recovers():
     it in the context's status word: error_count() then fails with
     NTC_ERR_CUDA until the reset, and the context decodes correctly after."""
     m = ntc()
-    w = small(2)
-    dec = decoder(2, None, "fp16")
+    w = small("uniform-4m")
+    dec = decoder("uniform-4m", None, "fp16")
     dec.reset_error_count()
     dec.debug_wait_timeout()
     with pytest.raises(m.NtcError) as e:
@@ -454,5 +458,5 @@ def test_a_wait_that_gives_up_is_reported_and_the_context_recovers():
     dec.reset_error_count()
     assert dec.error_count() == 0
     got = dec.decode(dq(w.queries)).cpu().numpy()
-    ref, _ = oracle_out(2)
+    ref, _ = oracle_out("uniform-4m")
     check_tc(got, ref, "after a wait gave up")

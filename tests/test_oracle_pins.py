@@ -151,7 +151,7 @@ def test_trilinear_blend_of_constant_mips():
 def test_fractional_lod_blends_the_two_integral_lods():
     # with t = 0 only mip lo is read; with t > 0 the feature is the linear blend
     # of the features the same UV gets at lod = lo and lod = lo + 1.
-    w = W.config(5, "small")
+    w = W.named("gbuffer-2160p-x4-trilinear", "small")
     q = w.queries[:3000].copy()
     lo = np.floor(q["lod"])
     t = (q["lod"] - lo).astype(np.float64)
@@ -236,7 +236,7 @@ def test_each_query_uses_its_sets_decoder():
 
 
 def test_shared_decoder_equals_one_dense_batch():
-    w = W.config(1, "small")
+    w = W.named("raster-256", "small")
     a = w.assets
     out, _ = oracle.decode(a, w.queries)
     x = torch.from_numpy(oracle.features(a, w.queries))
@@ -258,7 +258,7 @@ def test_bad_queries_are_nan_and_counted():
 
 
 def test_decode_is_invariant_to_query_order():
-    w = W.config(3, "small")
+    w = W.named("gbuffer-1080p", "small")
     out, _ = oracle.decode(w.assets, w.queries)
     p = np.random.default_rng(0).permutation(len(w.queries))
     out2, _ = oracle.decode(w.assets, w.queries[p])
@@ -266,7 +266,7 @@ def test_decode_is_invariant_to_query_order():
 
 
 def test_thread_count_does_not_change_results():
-    w = W.config(2, "small")
+    w = W.named("uniform-4m", "small")
     o1, _ = oracle.decode(w.assets, w.queries[:5000], nthreads=1)
     o2, _ = oracle.decode(w.assets, w.queries[:5000], nthreads=7)
     assert np.array_equal(o1, o2)

@@ -27,7 +27,8 @@ def _static_bucket(ntc, a, qd):
 
 def test_static_bucketing_matches_context_bucketing_on_consecutive_calls():
     from paper_2608_27888_gb300 import ntc
-    cases = [W.config(3, "small", "clustered4"), W.config(2, "small"), W.config(3, "small", "clustered4")]
+    cases = [W.named("gbuffer-1080p", "small", "clustered4"), W.named("uniform-4m", "small"),
+             W.named("gbuffer-1080p", "small", "clustered4")]
     for w in cases:  # three calls in a row, different sizes and decoder counts
         qd = ntc.queries_to_device(w.queries)
         perm, srt = _static_bucket(ntc, w.assets, qd)
@@ -41,7 +42,7 @@ def test_static_bucketing_matches_context_bucketing_on_consecutive_calls():
 
 def test_static_bucketing_rejects_sizes_beyond_its_scratch():
     from paper_2608_27888_gb300 import ntc
-    w = W.config(1, "small")
+    w = W.named("raster-256", "small")
     qd = ntc.queries_to_device(w.queries)
     m = np.zeros(1, dtype=np.uint32)
     n_too_many = 262144 // 4096 * 4096 * 2  # (4095 + 1) * ceil(n / 2048) > 262144
