@@ -329,6 +329,14 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
   }
   if (reg_base && threadIdx.x < D1) gbase[threadIdx.x] = my_base;
   __syncthreads();
+  // SPREAD: every reservation of this chunk has been made (their results are in
+  // gbase), so the chunk takes its ticket now, before thread 0 has any global
+  // store in flight; the atomic's round trip overlaps the copy-out
+  uint32_t ticket_no = 0;
+  if (SPREAD && threadIdx.x == 0) {
+    __threadfence();  // this CTA's reservations before its ticket
+    ticket_no = atomicAdd(cursor + D1, 1u);
+  }
   // coalesced copy-out: consecutive slots of one decoder go to consecutive
   // positions of that decoder's segment
   for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
@@ -340,11 +348,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
   if (SPREAD) {
     __shared__ bool last;
     uint32_t *ticket = cursor + D1;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      __threadfence();  // this CTA's reservations before its ticket
-      last = atomicAdd(ticket, 1u) == gridDim.x - 1;
-    }
+    if (threadIdx.x == 0) last = ticket_no == gridDim.x - 1;
     __syncthreads();
     if (!last) return;
     __threadfence();
