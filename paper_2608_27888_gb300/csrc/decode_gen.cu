@@ -25,10 +25,19 @@ namespace ntc {
 namespace {
 
 // act: 0 ReLU, 1 LeakyReLU, 2 LeakyReLU with 0 <= slope <= 1, where
-// max(x, slope * x) is the same function in two instructions
+// max(h, slope * h) is the same function: evaluated on the packed fp16/bf16
+// pair (slope2 = the slope in both halves), two instructions per pair
 template <bool BF16>
-__device__ __forceinline__ uint32_t pack_act(float lo, float hi, uint32_t act, float slope) {
-  if (act == 2) return pack<BF16>(fmaxf(lo, slope * lo), fmaxf(hi, slope * hi));
+__device__ __forceinline__ uint32_t pack_act(float lo, float hi, uint32_t act, float slope, uint32_t slope2) {
+  if (act == 2) {
+    const uint32_t h = pack<BF16>(lo, hi);
+    uint32_t r;
+    if (BF16)
+      asm("{\n.reg .b32 t;\nmul.rn.bf16x2 t, %1, %2;\nmax.bf16x2 %0, %1, t;\n}" : "=r"(r) : "r"(h), "r"(slope2));
+    else
+      asm("{\n.reg .b32 t;\nmul.rn.f16x2 t, %1, %2;\nmax.f16x2 %0, %1, t;\n}" : "=r"(r) : "r"(h), "r"(slope2));
+    return r;
+  }
   if (act == 1) {
     lo = lo > 0.0f ? lo : slope * lo;
     hi = hi > 0.0f ? hi : slope * hi;
@@ -245,6 +254,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
     cwalk.cap = B.spread_cap;
     const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
     const uint32_t act = G.activation == 1 && G.slope >= 0.0f && G.slope <= 1.0f ? 2u : G.activation;
+    const uint32_t slope2 = pack<BF16>(G.slope, G.slope);
     auto wait = [&](uint32_t bar, uint32_t parity) {
       if (!mbar_wait(bar, parity)) {
         atomicOr(status, 1u);
@@ -314,9 +324,9 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
           for (int i = 0; i < 4; ++i) {
             const float4 b = bl[i];
             p[2 * i] = pack_act<BF16>(__uint_as_float(v[4 * i]) + b.x, __uint_as_float(v[4 * i + 1]) + b.y, act,
-                                      G.slope);
+                                      G.slope, slope2);
             p[2 * i + 1] = pack_act<BF16>(__uint_as_float(v[4 * i + 2]) + b.z, __uint_as_float(v[4 * i + 3]) + b.w,
-                                          act, G.slope);
+                                          act, G.slope, slope2);
           }
           tmem_st8(tAH + lanes, p);
         } else {
@@ -329,9 +339,9 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
             for (int i = 0; i < 8; ++i) {
               const float4 b = bl[c0 / 4 + i];
               p[2 * i] = pack_act<BF16>(__uint_as_float(v[4 * i]) + b.x, __uint_as_float(v[4 * i + 1]) + b.y, act,
-                                        G.slope);
+                                        G.slope, slope2);
               p[2 * i + 1] = pack_act<BF16>(__uint_as_float(v[4 * i + 2]) + b.z, __uint_as_float(v[4 * i + 3]) + b.w,
-                                            act, G.slope);
+                                            act, G.slope, slope2);
             }
             tmem_st16(tAH + lanes + c0 / 2, p);
           }
