@@ -78,7 +78,10 @@ __host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) {
 }
 
 // Warp-specialised: warpgroup 0 produces, warpgroup 1 consumes.  The CTA's
-// tiles are t_j = blockIdx.x + j * gridDim.x; tile j goes through ring stage
+// tiles are a contiguous range t_j = t0 + j of the tile list (the latents of
+// these decoders are small enough to stay in L2, so there is no locality to
+// gain from neighbouring CTAs sharing tiles; consecutive tiles share their
+// decoder instead); tile j goes through ring stage
 // j mod kGenStages.  Producer thread r gathers row r of tile j into the stage's
 // A operand (TMEM lane r) and its output row into oidx; each producer warp
 // arrives on full[s].  The consumer's thread 0 issues layer 1 from the stage
@@ -148,7 +151,11 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
   const uint32_t tA1 = tmem_slot + H + H / 2;  // ring stages, K1 / 2 columns each
   const uint32_t T = __ldg(B.meta);
   const uint32_t grid = gridDim.x;
-  const uint32_t K = blockIdx.x < T ? (T - blockIdx.x + grid - 1) / grid : 0;  // this CTA's tiles
+  // this CTA's tiles: a contiguous range t0 .. t0 + K - 1 of the tile list, so
+  // consecutive tiles share their decoder and the weights are copied rarely
+  const uint32_t per = T / grid, rem = T % grid;
+  const uint32_t t0 = blockIdx.x * per + min(blockIdx.x, rem);
+  const uint32_t K = per + (blockIdx.x < rem ? 1u : 0u);
   if (wg == 0) {
     // ------------------------------------------------------------- producer
     TileWalk walk;
@@ -157,7 +164,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
     // tile j is gathered
     auto load_row = [&](uint32_t jj, uint32_t &d_, uint32_t &len_, ntc_query &q_, uint32_t &oi_) {
       uint32_t st_;
-      walk.at(seg, tst, D, blockIdx.x + jj * grid, d_, st_, len_);
+      walk.at(seg, tst, D, t0 + jj, d_, st_, len_);
       oi_ = 0;
       if (row < len_) {
         q_ = load_query(B.sorted + st_ + row);
@@ -275,7 +282,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
     for (uint32_t j = 0; j < K; ++j) {
       const uint32_t s = j % kGenStages, use = j / kGenStages;
       uint32_t dec, st, len;
-      cwalk.at(seg, tst, D, blockIdx.x + j * grid, dec, st, len);
+      cwalk.at(seg, tst, D, t0 + j, dec, st, len);
       if (row < 32) wait(full_bar(s), use & 1u);
       // one decision to stop per tile, the same for every warp of the warpgroup
       if (row == 0) stop_flag[j & 1] = abort_flag;
