@@ -46,6 +46,15 @@ __device__ __forceinline__ uint32_t pack_act(float lo, float hi, uint32_t act, f
   return pack_relu<BF16>(__float_as_uint(lo), __float_as_uint(hi));
 }
 
+// LeakyReLU (0 <= slope <= 1) of the fp16 pair h + b: max(t, slope * t)
+__device__ __forceinline__ uint32_t act_h2(uint32_t h, uint32_t b, uint32_t slope2) {
+  uint32_t r;
+  asm("{\n.reg .b32 t, u;\nadd.rn.f16x2 t, %1, %2;\nmul.rn.f16x2 u, t, %3;\nmax.f16x2 %0, t, u;\n}"
+      : "=r"(r)
+      : "r"(h), "r"(b), "r"(slope2));
+  return r;
+}
+
 __device__ __forceinline__ void count_bad_warp(bool bad, unsigned long long *err) {
   const unsigned m = __ballot_sync(0xFFFFFFFFu, bad);
   if (m && (threadIdx.x & 31) == __ffs(m) - 1) atomicAdd(err, (unsigned long long)__popc(m));
@@ -322,7 +331,28 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
         wait_mma();
         fence_after();
         const float4 *bl = reinterpret_cast<const float4 *>(bias + l * H);  // 16-byte aligned
-        if (H == 16) {
+        // fp16 with LeakyReLU: bias and activation on the packed pair
+        const uint4 *bh = reinterpret_cast<const uint4 *>(bias + NL * H + 16) + l * H / 8;
+        if (!BF16 && act == 2) {
+          for (uint32_t c0 = 0; c0 < H; c0 += 16) {
+            uint32_t v[16];
+            tmem_ld16(tAcc + lanes + c0, v);
+            tmem_wait_ld();
+            uint32_t p[8];
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+              const uint4 b = bh[c0 / 8 + i];
+              p[4 * i] = act_h2(pack<false>(__uint_as_float(v[8 * i]), __uint_as_float(v[8 * i + 1])), b.x, slope2);
+              p[4 * i + 1] =
+                  act_h2(pack<false>(__uint_as_float(v[8 * i + 2]), __uint_as_float(v[8 * i + 3])), b.y, slope2);
+              p[4 * i + 2] =
+                  act_h2(pack<false>(__uint_as_float(v[8 * i + 4]), __uint_as_float(v[8 * i + 5])), b.z, slope2);
+              p[4 * i + 3] =
+                  act_h2(pack<false>(__uint_as_float(v[8 * i + 6]), __uint_as_float(v[8 * i + 7])), b.w, slope2);
+            }
+            tmem_st8(tAH + lanes + c0 / 2, p);
+          }
+        } else if (H == 16) {
           uint32_t v[16];
           tmem_ld16(tAcc + lanes, v);
           tmem_wait_ld();
@@ -520,6 +550,8 @@ __global__ void k_pack_gen(const float *w32, GenWeights G, uint8_t *tc, uint8_t 
       const uint32_t l = e / H;
       b[e] = l < NL ? bsrc(l)[e % H] : (e - NL * H < C ? bsrc(NL)[e - NL * H] : 0.0f);
     }
+    __half *bh = reinterpret_cast<__half *>(b + NL * H + 16);
+    for (uint32_t e = threadIdx.x; e < NL * H; e += blockDim.x) bh[e] = __float2half_rn(bsrc(e / H)[e % H]);
   }
   T *o = reinterpret_cast<T *>(fma + (size_t)d * G.fma_stride);
   for (uint32_t e = threadIdx.x; e < H * I; e += blockDim.x) o[e] = E::cvt(Wsrc(0)[e]);

@@ -91,7 +91,8 @@ constexpr int kGenMaxPe = 8;       // encoding frequencies
 //  tc image (fp16/bf16 tcgen05 B operands, no-swizzle K-major core matrices):
 //    W1 [H][K1] (K1 = in_dim rounded up to 16, zero padded), W_l [H][H] for
 //    each further hidden layer, Wout [16][H] (rows >= C zero), then fp32 b1[H],
-//    b_l[H]..., bout[16].
+//    b_l[H]..., bout[16], then the hidden biases again as fp16 (the fp16
+//    epilogue adds them to the packed pair).
 //  fma image (the precision's type T, row-major): W1 [H][in], W_l [H][H]...,
 //    Wout^T [H][CP], then fp32 biases as above (bout padded to CP).
 struct GenWeights {
@@ -111,7 +112,7 @@ inline __host__ __device__ size_t gen_bias_floats(uint32_t H, uint32_t layers) {
   return (size_t)layers * H + 16;
 }
 inline __host__ __device__ size_t gen_tc_image_bytes(uint32_t in_dim, uint32_t H, uint32_t layers) {
-  return gen_tc_weight_bytes(in_dim, H, layers) + gen_bias_floats(H, layers) * 4;
+  return gen_tc_weight_bytes(in_dim, H, layers) + gen_bias_floats(H, layers) * 4 + (size_t)layers * H * 2;
 }
 inline __host__ __device__ size_t gen_fma_image_bytes(uint32_t in_dim, uint32_t H, uint32_t layers, uint32_t C,
                                                       uint32_t elem) {
