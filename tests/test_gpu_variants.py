@@ -136,3 +136,21 @@ def test_modes_without_a_general_kernel_are_refused():
         with pytest.raises(m.NtcError, match="decoder shape"):
             dec.decode(dq(w.queries[:64]), mode=mode)
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("slope", [1.25, -0.1])
+def test_leaky_slopes_outside_the_unit_interval(slope):
+    """A LeakyReLU slope outside [0, 1] takes the kernels' general activation
+    (a select, not max(x, slope * x)); every precision and mode agrees with the
+    oracle."""
+    w = W.paper_decoder("small", leaky_slope=slope)
+    r, _ = oracle.decode(w.assets, w.queries)
+    for precision in ("fp16", "bf16", "fp32"):
+        dec = ntc().Decoder(w.assets, precision)
+        for mode in ("bucketed", "divergent_fma"):
+            got = dec.decode(dq(w.queries), mode=mode).cpu().numpy()
+            if precision == "fp32":
+                assert np.abs(got - r).max() <= FP32_TOL, (precision, mode)
+            else:
+                check_tc(got, r, f"slope {slope} {mode} {precision}")
+        dec.close()
