@@ -466,12 +466,16 @@ def test_four_channel_grid_returns_texel_values_at_centres():
     assert np.array_equal(f, grid[ij[:, 1], ij[:, 0]])
 
 
-def test_leaky_relu_identity_weights_closed_form():
+@pytest.mark.parametrize("slope", [0.2, 1.25, -0.1])
+def test_leaky_relu_identity_weights_closed_form(slope):
+    """Identity weights and zero biases reduce the decoder to the activation
+    applied once per hidden layer: x -> x for x > 0, slope * x otherwise.  With
+    a negative slope the second layer sees a positive value and leaves it."""
     rng = np.random.default_rng(4)
     dims = [[(8, 8), (4, 4)]]
     _, _, total = W.pyramid_layout(1, dims, 1)
     a = tiny_assets(dims, latents=rng.standard_normal(total * 8).astype(np.float32), hidden=16,
-                    out_dim=8, activation=1, leaky_slope=0.2)
+                    out_dim=8, activation=1, leaky_slope=slope)
     a.weights[:] = 0
     W1, b1, W2, b2, W3, b3 = split_weights(a)
     W1[:] = np.eye(16)
@@ -480,10 +484,13 @@ def test_leaky_relu_identity_weights_closed_form():
     q = queries([(0, float(u), float(v), 0.0) for u, v in rng.uniform(-2, 2, (300, 2))])
     out, _ = oracle.decode(a, q)
     f = oracle.features(a, q)[:, :8]
-    slope = float(np.float32(0.2))
-    leaky = np.where(f > 0, f, slope * slope * f)  # two hidden layers
+    s = float(np.float32(slope))
+    once = np.where(f > 0, f, s * f)
+    twice = np.where(once > 0, once, s * once)  # two hidden layers
     assert (f < 0).any()
-    assert np.allclose(out, sigmoid(leaky), atol=1e-15)
+    expected = np.where(f > 0, f, s * s * f) if s > 0 else np.where(f > 0, f, s * f)
+    assert np.allclose(twice, expected, rtol=1e-14, atol=0.0)
+    assert np.allclose(out, sigmoid(twice), atol=1e-15)
 
 
 @pytest.mark.parametrize("hidden,layers", [(16, 1), (32, 2), (64, 2), (64, 3), (128, 4), (32, 4)])
