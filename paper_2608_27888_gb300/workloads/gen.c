@@ -141,7 +141,8 @@ static void *lat_worker(void *arg) {
 void gen_latents(uint64_t seed, uint32_t S, uint32_t L, uint32_t M, uint32_t C,
                  const uint32_t *dims, const uint64_t *offs, double sigma, uint16_t *out,
                  int nthreads) {
-  lat_job J = {seed, S, L, M, C, dims, offs, out, sigma, 0};
+  lat_job J = {.seed = seed, .S = S, .L = L, .M = M, .C = C, .dims = dims, .offs = offs,
+               .out = out, .sigma = sigma, .next = 0};
   pthread_mutex_init(&J.mu, NULL);
   if (nthreads < 1) nthreads = 1;
   pthread_t *th = (pthread_t *)malloc(sizeof(pthread_t) * nthreads);
