@@ -29,13 +29,12 @@
  *
  * Memory: the context owns device copies of latents, weights and map.  Query
  * and output buffers of ntc_decode are DEVICE pointers owned by the caller.
- * Scratch (bucket counts, permutation, sorted queries) is owned by the context
- * and grows on demand with cudaMallocAsync on the call's stream.  The
- * tensor-core BUCKETED decode sorts in one pass when (num_decoders + 1) * n
- * rows of 20 bytes fit in 24 GiB, giving every decoder a region of n rows
- * (e.g. 1.4 GB for 16 decoders and 4M queries); otherwise it runs the stable
- * three-kernel sort, which needs n rows.  One context must not run two
- * decodes concurrently (on different streams or threads).
+ * Scratch (the permutation and the queries in bucket order, 20 bytes per
+ * query, the tile table, and 8 bytes per decoder and 2048 queries of
+ * look-back records) is owned by the context and grows on demand with
+ * cudaMallocAsync on the call's stream.  Every bucketed decode sorts with the
+ * same stable counting sort that ntc_debug_bucket exports.  One context must
+ * not run two decodes concurrently (on different streams or threads).
  *
  * Errors: host-detectable problems return a status and enqueue nothing; the
  * message is available from ntc_last_error().  A query whose set id is out of
@@ -85,14 +84,13 @@ typedef enum {
 } ntc_precision;
 
 /* Which decode path ntc_decode runs.
- * BUCKETED:     the queries are grouped by decoder id, then the gather-decode
- *               runs over 128-query single-decoder tiles.  Tensor-core precisions
- *               group in one unstable pass (see Memory above) and run the
- *               tcgen05/TMEM kernel; FP32 groups with the stable counting sort
- *               and runs FFMA.  With one decoder for all sets the tensor-core
- *               decode takes the queries in their own order.  Each output row
- *               depends only on its own query, so the grouping order never
- *               changes an output.
+ * BUCKETED:     the queries are sorted stably by decoder id (the permutation
+ *               ntc_debug_bucket returns), then the gather-decode runs over
+ *               128-query single-decoder tiles: the tcgen05/TMEM kernel for
+ *               the tensor-core precisions, FFMA for FP32.  With one decoder
+ *               for all sets the tensor-core decode takes the queries in their
+ *               own order.  Each output row depends only on its own query, so
+ *               the grouping never changes an output.
  * DIVERGENT:    no sorting: each warp takes 32 consecutive queries and loops over
  *               its distinct decoders (the non-shared setting of Sec. 4.4).
  *               Tensor-core precisions only.
@@ -208,15 +206,51 @@ NTC_API ntc_status ntc_debug_taps(ntc_ctx *ctx, const ntc_query *d_queries, size
 NTC_API ntc_status ntc_debug_features(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_feat,
                               void *cuda_stream);
 
-/* The bucketing stage alone.  d_perm[n]: query indices in (decoder, original
- * index) order, where a query with an out-of-range set id counts as decoder
- * num_decoders.  d_counts (may be NULL): [num_decoders+1] queries per decoder.
+/* The bucketing stage alone (Sec. 2: the queries of one block that need
+ * different decoders are what diverges; sorting by decoder leaves tiles of one
+ * decoder), by the same kernels and the same scratch as ntc_decode's BUCKETED
+ * mode.  d_perm[n]: query indices in (decoder, original index) order, where a
+ * query with an out-of-range set id counts as decoder num_decoders.  d_counts (may be NULL): [num_decoders+1] queries per decoder.
  * d_tiles (may be NULL): [ntc_max_tiles(ctx, n)][3] = (decoder, first position
  * in perm, length) of every 128-query tile, in decoder order; d_num_tiles (may
  * be NULL): [1] the number of tiles written.  Device pointers; async. */
 NTC_API ntc_status ntc_debug_bucket(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, uint32_t *d_perm,
                             uint32_t *d_counts, uint32_t *d_tiles, uint32_t *d_num_tiles,
                             void *cuda_stream);
+
+/* One query row as the default tensor-core decode (BUCKETED, TC_FP16/TC_BF16,
+ * the standard shape) built it -- the bilinear fetch of Sec. 1's latent grids
+ * that feeds x^_i = D_c(i)(z_i) of Sec. 3.3 -- recorded by
+ * ntc_debug_decode_rows.  Level k, mip slot m (0: mip lo; 1: mip lo + 1,
+ * written only when t > 0) and tap p in the order 00, 10, 01, 11:
+ *   idx  texel index into `latents` (the ntc_desc array) of the tap, from the
+ *        kernel's own texel coordinates;
+ *   raw  the 16 bytes (8 fp16 channels) the kernel blended for the tap;
+ *   w    the fp32 weight it blended them with: the bilinear weight times
+ *        1 - t (slot 0 of a blend) or t (slot 1).  In clamp mode a row whose
+ *        two texels coincide (an edge) carries the row's whole weight on tap
+ *        0 (or 2) and weight 0 on tap 1 (or 3), whose raw is then unused;
+ *   t, lo the mip pick;
+ *   feat the MLP input as stored in tensor memory: 16 fp16 (TC_FP16) or bf16
+ *        (TC_BF16) values, feat[i] holding inputs 2i (low half) and 2i + 1. */
+typedef struct {
+  uint64_t idx[2][2][4];
+  uint32_t raw[2][2][4][4];
+  float w[2][2][4];
+  float t;
+  uint32_t lo;
+  uint32_t feat[8];
+  uint32_t pad[6];
+} ntc_debug_row; /* 512 bytes */
+
+/* ntc_decode in BUCKETED mode through a debug instantiation of its tcgen05
+ * kernel: the same bucketing, kernel template, launch configuration and
+ * outputs (d_out as ntc_decode), and every good query's row recorded in
+ * d_rows[i] (device array of n records; rows of bad queries are not
+ * written).  TC_FP16/TC_BF16 contexts of the standard shape only
+ * (NTC_ERR_UNSUPPORTED otherwise).  Device pointers; async. */
+NTC_API ntc_status ntc_debug_decode_rows(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_out,
+                                         ntc_debug_row *d_rows, void *cuda_stream);
 
 /* Upper bound on the number of 128-query tiles of n queries. */
 NTC_API size_t ntc_max_tiles(const ntc_ctx *ctx, size_t n);
@@ -260,8 +294,13 @@ NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
  * num_decoders) and d_sorted[n] the query records in that order.  h_set_to_decoder
  * is a HOST array of num_sets entries (each < num_decoders); d_queries,
  * d_perm and d_sorted are caller-owned device buffers (the query buffers
- * 16-byte aligned).  Its scratch is one file-scope device array of 1,360,896
- * bytes that every GPU loading the library holds until the process exits, so:
+ * 16-byte aligned).  d_status (may be NULL) is a caller-owned device word: the
+ * kernels OR a nonzero value into it when one of their bounded waits (200 ms)
+ * gave up, and the result of that call is then invalid; the library never
+ * clears it, so zero it before the calls it should watch and read it after
+ * they have completed.  Its scratch is one file-scope device array of
+ * 2,409,472 bytes that every GPU loading the library holds until the process
+ * exits, so:
  *   - num_sets <= 65536, num_decoders <= 4095 and
  *     (num_decoders + 1) * ceil(n / 2048) <= 262144 (larger calls return
  *     NTC_ERR_UNSUPPORTED and enqueue nothing);
@@ -276,7 +315,8 @@ NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
  * cudaFree or allocating library routine. */
 NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder, uint32_t num_sets,
                                      uint32_t num_decoders, const ntc_query *d_queries, size_t n,
-                                     uint32_t *d_perm, ntc_query *d_sorted, void *cuda_stream);
+                                     uint32_t *d_perm, ntc_query *d_sorted, uint32_t *d_status,
+                                     void *cuda_stream);
 
 /* ---------------------------------------------------------- map sources
  *

@@ -3,16 +3,23 @@
 // Sec. 2 of the paper defines divergence as several decoders being needed by
 // the queries of one block; sorting the queries by decoder (stable, so each
 // bucket keeps the original order) turns the interleaved stream into runs of
-// single-decoder 128-query tiles.  Three kernels, no inter-CTA waiting:
-//   k_hist    per-chunk histogram; each warp of a chunk owns a contiguous range
-//             and counts it with __match_any_sync (one leader per decoder run)
-//   k_scan    one CTA per decoder scans that decoder's per-chunk counts; the last
-//             CTA to finish (atomic ticket) scans the decoder totals into the
-//             segment starts and the tile starts
-//   k_scatter recomputes each warp's counts, sorts its chunk stably by decoder
-//             in shared memory, then copies each decoder's run out to its
-//             segment with coalesced stores (perm[] and the sorted records)
-// A query whose set id is out of range goes to the extra bucket D.
+// single-decoder 128-query tiles.  Two kernels:
+//   k_count  the decoder histogram of all queries: per-warp counters in shared
+//            memory (one __match_any_sync leader per run of equal decoders),
+//            one atomicAdd per decoder and CTA into the global totals
+//   k_place  one CTA per 2048-query chunk, chunks taken in ticket order.  It
+//            ranks its queries stably within the chunk, publishes its
+//            per-decoder counts, and finds how many queries of each decoder
+//            the earlier chunks hold by a decoupled look-back over their
+//            published counts and inclusive prefixes (it waits only on CTAs
+//            that took an earlier ticket, which are already running).  With
+//            the segment starts (the scan of the totals) that fixes every
+//            query's place; the chunk is sorted in shared memory and copied
+//            out with coalesced stores (perm[] and the sorted records).  The
+//            CTA with chunk 0 writes the tile table; the last CTA to finish
+//            clears the totals and tickets for the next call.
+// The permutation is exactly std::stable_sort of the indices by decoder.  A
+// query whose set id is out of range goes to the extra bucket D.
 #include "ntc_internal.cuh"
 
 namespace ntc {
@@ -46,6 +53,13 @@ struct MapLookup {
 
 __device__ __forceinline__ uint32_t saddr_b(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+constexpr uint64_t kWaitNs = 200ull * 1000ull * 1000ull;  // every wait gives up after 200 ms
+
 // Stream `bytes` (a multiple of 16) from global memory into shared memory with
 // one bulk copy (TMA): bulk_issue (every thread; thread 0 issues), then
 // bulk_wait, which is false if the copy has not landed after 200 ms.
@@ -74,136 +88,66 @@ __device__ bool bulk_wait(uint64_t *bar) {
         : "r"(b)
         : "memory");
     if (ok) return true;
-    uint64_t now;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(now));
+    const uint64_t now = globaltimer();
     if (spin == 0) t0 = now;
-    else if (now - t0 > 200ull * 1000ull * 1000ull) return false;
+    else if (now - t0 > kWaitNs) return false;
   }
 }
 
-__global__ void __launch_bounds__(kBucketThreads) k_hist(Assets A, const ntc_query *q, size_t n,
-                                                         uint32_t *counts, uint32_t chunks,
-                                                         unsigned int *status) {
-  // shared memory: the chunk's records [kBucketChunk], then [kWarps][D+1] counters
-  extern __shared__ uint4 srec[];
-  __shared__ uint64_t bar;
-  uint32_t *cnt = reinterpret_cast<uint32_t *>(srec + kBucketChunk);
+// Look-back descriptors, one 64-bit word per (chunk, decoder): the low half is
+// a count, the high half (epoch << 2) | state with state 1 = the chunk's own
+// count, 2 = the inclusive prefix over chunks 0..c.  A word of another epoch
+// (an earlier call) is "not ready", so nothing has to be cleared between calls.
+__device__ __forceinline__ unsigned long long ld_desc(const unsigned long long *p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_desc(unsigned long long *p, unsigned long long v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long make_desc(uint32_t epoch, uint32_t state, uint32_t count) {
+  return ((unsigned long long)((epoch << 2) | state) << 32) | count;
+}
+
+// ------------------------------------------------------------------ k_count
+
+__global__ void __launch_bounds__(kBucketThreads) k_count(Assets A, const ntc_query *q, size_t n,
+                                                          uint32_t chunks, uint32_t *totals) {
+  extern __shared__ uint32_t cnt[];  // [kWarps][D+1]
+  pdl_trigger();                     // k_place may start its own work at once
   const uint32_t D1 = A.num_decoders + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const MapLookup lookup(A);
-  const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
-  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
-  bulk_issue(srec, q + cbase, valid * 16u, &bar);
-  pdl_trigger();  // k_scan may launch (it waits for this grid before reading)
-  if (!bulk_wait(&bar)) atomicOr(status, 2u);
-  const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);
+  __syncthreads();
+  const MapLookup lookup(A);
   uint32_t *my = cnt + warp * D1;
+  const uint32_t *sid = reinterpret_cast<const uint32_t *>(q);
+  for (uint32_t c = blockIdx.x; c < chunks; c += gridDim.x) {
+    const size_t wbase = (size_t)c * kBucketChunk + (size_t)warp * (kBucketItems * 32);
+    uint32_t s[kBucketItems];
 #pragma unroll
-  for (int it = 0; it < kBucketItems; ++it) {
-    const uint32_t j = wbase + it * 32 + lane;
-    const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
-    const uint32_t d = j < valid ? dl : 0xFFFFFFFFu;
-    const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
-    if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
-    __syncwarp();
+    for (int it = 0; it < kBucketItems; ++it) {  // every load in flight before any is used
+      const size_t j = wbase + it * 32 + lane;
+      s[it] = j < n ? __ldg(sid + 4 * j) : 0u;
+    }
+#pragma unroll
+    for (int it = 0; it < kBucketItems; ++it) {
+      const size_t j = wbase + it * 32 + lane;
+      const uint32_t dl = lookup(A, s[it]);  // every lane: the lookup shuffles
+      const uint32_t d = j < n ? dl : 0xFFFFFFFFu;
+      const uint32_t m = __match_any_sync(0xFFFFFFFFu, d);
+      if (d != 0xFFFFFFFFu && lane == __ffs(m) - 1) my[d] += __popc(m);
+      __syncwarp();
+    }
   }
   __syncthreads();
   for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
     uint32_t s = 0;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) s += cnt[w * D1 + d];
-    counts[(size_t)d * chunks + blockIdx.x] = s;
+    if (s) atomicAdd(totals + d, s);
   }
-}
-
-// Exclusive scan of one value per thread over a 1024-thread block.
-__device__ __forceinline__ uint32_t block_scan_1024(uint32_t v, uint32_t &total, uint32_t *ws) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t x = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) ws[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    uint32_t s = ws[lane];
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      uint32_t y = __shfl_up_sync(0xFFFFFFFFu, s, o);
-      if (lane >= o) s += y;
-    }
-    ws[lane] = s;
-  }
-  __syncthreads();
-  uint32_t excl = x - v + (warp > 0 ? ws[warp - 1] : 0u);
-  total = ws[31];
-  __syncthreads();
-  return excl;
-}
-
-// Scan `len` values in place (exclusive) with 1024 threads, 4 per thread per
-// round; returns the total.
-__device__ uint32_t block_scan_inplace(uint32_t *a, uint32_t len, uint32_t *ws) {
-  uint32_t carry = 0;
-  for (uint32_t b = 0; b < len; b += 4096) {
-    uint32_t v[4], s = 0;
-    const uint32_t i0 = b + threadIdx.x * 4;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      v[j] = i0 + j < len ? a[i0 + j] : 0u;
-      s += v[j];
-    }
-    uint32_t tot;
-    uint32_t e = block_scan_1024(s, tot, ws) + carry;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (i0 + j < len) a[i0 + j] = e;
-      e += v[j];
-    }
-    carry += tot;
-  }
-  return carry;
-}
-
-// meta layout: [0] num_tiles, [1 .. D+2] seg_start, [D+3 .. 2D+4] tile_start;
-// ticket: one word, zero between calls.
-__global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks, uint32_t D,
-                                               uint32_t n, uint32_t *totals, uint32_t *meta,
-                                               uint32_t *ticket) {
-  __shared__ uint32_t ws[32];
-  __shared__ bool last;
-  const uint32_t d = blockIdx.x;
-  pdl_wait();  // the per-chunk counts of k_hist
-  uint32_t tot = block_scan_inplace(counts + (size_t)d * chunks, chunks, ws);
-  if (threadIdx.x == 0) {
-    totals[d] = tot;
-    __threadfence();
-    last = atomicAdd(ticket, 1u) == D;  // gridDim.x == D + 1
-  }
-  __syncthreads();
-  if (!last) return;
-  __threadfence();
-  uint32_t *seg = meta + 1, *tst = meta + 1 + (D + 2);
-  // segment starts and tile starts over the D+1 buckets
-  for (uint32_t i = threadIdx.x; i < D + 1; i += blockDim.x) {
-    uint32_t c = ((volatile uint32_t *)totals)[i];
-    seg[i] = c;
-    tst[i] = (c + kTile - 1) / kTile;
-  }
-  __syncthreads();
-  uint32_t ns = block_scan_inplace(seg, D + 1, ws);
-  __syncthreads();
-  uint32_t nt = block_scan_inplace(tst, D + 1, ws);
-  if (threadIdx.x == 0) {
-    seg[D + 1] = ns;  // == n
-    tst[D + 1] = nt;
-    meta[0] = nt;
-    *ticket = 0;
-  }
-  (void)n;
 }
 
 // In-place exclusive scan of len values (in shared memory) by the 256 threads of
@@ -234,41 +178,41 @@ __device__ void block_scan_256(uint32_t *a, uint32_t len) {
   __syncthreads();
 }
 
-// SPREAD (the single-pass bucketing of the tensor-core decode): no k_hist or
-// k_scan runs first.  Decoder d owns region [d * cap, d * cap + cap) of perm
-// and sorted (cap = n); each chunk reserves room for its run of decoder d with
-// one atomicAdd on cursor[d], so runs of one decoder keep chunk order only as
-// far as the atomics happen to, and the permutation is not the stable one
-// (every decoded row is independent of the others in its tile, so outputs do
-// not change).  The last CTA to finish (atomic ticket, no waiting) writes meta
-// with seg[d] = the decoder's count and the tile starts, and clears cursor and
-// ticket for the next call.
-template <bool SPREAD>
-__global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_query *q, size_t n,
-                                                            const uint32_t *counts, uint32_t chunks,
-                                                            uint32_t *meta, uint32_t *perm,
-                                                            ntc_query *sorted, unsigned int *status,
-                                                            uint32_t *cursor, uint32_t cap) {
+// ------------------------------------------------------------------ k_place
+
+// meta layout: [0] num_tiles, [1 .. D+2] seg_start, [D+3 .. 2D+4] tile_start;
+// then totals [D+1], the start ticket and the done ticket (zero between calls).
+__global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_query *q, size_t n,
+                                                          uint32_t chunks, uint32_t *meta,
+                                                          unsigned long long *desc, uint32_t epoch,
+                                                          uint32_t *perm, ntc_query *sorted,
+                                                          unsigned int *status) {
   // shared memory: the chunk's records [chunk] (16 B), the chunk-local index
   // [chunk] (u16) and decoder [chunk] (u16) of every sorted slot, then per-warp
-  // counters [kWarps][D+1] and the chunk's per-decoder local offsets and global
-  // bases [D+1] each
+  // counters [kWarps][D+1] (reused for the segment starts once the chunk is
+  // sorted), and per decoder the chunk-local run start and the global base
   extern __shared__ uint4 srec[];
   __shared__ uint64_t bar;
+  __shared__ uint32_t s_chunk;
+  __shared__ bool s_last;
   uint16_t *sidx = reinterpret_cast<uint16_t *>(srec + kBucketChunk);
   uint16_t *sdec = sidx + kBucketChunk;
   uint32_t *cnt = reinterpret_cast<uint32_t *>(sdec + kBucketChunk);
-  const uint32_t D1 = A.num_decoders + 1;
+  const uint32_t D = A.num_decoders, D1 = D + 1;
   uint32_t *loff = cnt + kWarps * D1;  // chunk-local start of each decoder's run
   uint32_t *gbase = loff + D1;         // global position of that run's first element
+  uint32_t *totals = meta + meta_words(D);
+  uint32_t *start_ticket = totals + D1, *done_ticket = start_ticket + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const MapLookup lookup(A);
-  const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
-  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+  if (threadIdx.x == 0) s_chunk = atomicAdd(start_ticket, 1u);  // chunks in the order CTAs start
   for (uint32_t i = threadIdx.x; i < kWarps * D1; i += blockDim.x) cnt[i] = 0;
-  bulk_issue(srec, q + cbase, valid * 16u, &bar);  // the queries do not depend on k_scan
-  if (!SPREAD) pdl_wait();                           // the scanned counts and segment starts
-  pdl_trigger();                                     // the decode may launch (it waits for this grid)
+  __syncthreads();
+  const uint32_t c = s_chunk;
+  const size_t cbase = (size_t)c * kBucketChunk;
+  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+  bulk_issue(srec, q + cbase, valid * 16u, &bar);
+  pdl_trigger();  // the decode may launch (it waits for this grid before reading)
+  const MapLookup lookup(A);
   if (!bulk_wait(&bar)) atomicOr(status, 2u);
   const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
   uint32_t dec[kBucketItems];
@@ -292,32 +236,22 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
     __syncwarp();
   }
   __syncthreads();
-  // per decoder: warp prefix (in place), chunk total and global base.  SPREAD
-  // with D + 1 <= blockDim.x: thread d keeps its reservation in a register
-  // until the copy-out, so the atomic's round trip overlaps the scan and the
-  // local sort
-  const uint32_t *seg = meta + 1;
-  const bool reg_base = SPREAD && D1 <= blockDim.x;
-  uint32_t my_base = 0;
+  // per decoder: warp prefix (in place) and the chunk's count, published at
+  // once so later chunks can look back past this one
   for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
     uint32_t run = 0;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) {
-      const uint32_t c = cnt[w * D1 + d];
+      const uint32_t x = cnt[w * D1 + d];
       cnt[w * D1 + d] = run;
-      run += c;
+      run += x;
     }
     loff[d] = run;
-    if (SPREAD) {
-      const uint32_t b = run ? d * cap + atomicAdd(cursor + d, run) : 0u;
-      if (reg_base) my_base = b;
-      else gbase[d] = b;
-    } else {
-      gbase[d] = __ldg(seg + d) + counts[(size_t)d * chunks + blockIdx.x];
-    }
+    gbase[d] = run;  // the count, until the look-back replaces it
+    st_desc(desc + (size_t)c * D1 + d, make_desc(epoch, c == 0 ? 2u : 1u, run));
   }
   __syncthreads();
-  block_scan_256(loff, D1);  // exclusive scan of the chunk totals over decoders
+  block_scan_256(loff, D1);  // exclusive scan of the chunk's counts over decoders
   // stable local sort of (local index, decoder) pairs
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
@@ -327,16 +261,62 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
     sidx[lp] = (uint16_t)(wbase + it * 32 + lane);
     sdec[lp] = (uint16_t)d;
   }
-  if (reg_base && threadIdx.x < D1) gbase[threadIdx.x] = my_base;
-  __syncthreads();
-  // SPREAD: every reservation of this chunk has been made (their results are in
-  // gbase), so the chunk takes its ticket now, before thread 0 has any global
-  // store in flight; the atomic's round trip overlaps the copy-out
-  uint32_t ticket_no = 0;
-  if (SPREAD && threadIdx.x == 0) {
-    __threadfence();  // this CTA's reservations before its ticket
-    ticket_no = atomicAdd(cursor + D1, 1u);
+  // decoupled look-back: the queries of decoder d in chunks 0..c-1
+  bool gave_up = false;
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
+    const uint32_t own = gbase[d];
+    uint32_t before = 0;
+    if (c > 0) {
+      uint32_t p = c - 1;
+      uint64_t t0 = 0;
+      for (uint32_t spin = 0;;) {
+        const unsigned long long v = ld_desc(desc + (size_t)p * D1 + d);
+        const uint32_t hi = (uint32_t)(v >> 32);
+        if ((hi >> 2) == epoch && (hi & 3u) != 0u) {
+          before += (uint32_t)v;
+          if ((hi & 3u) == 2u || p == 0) break;
+          --p;
+          continue;
+        }
+        const uint64_t now = globaltimer();  // chunk p has not published yet
+        if (spin++ == 0) t0 = now;
+        else if (now - t0 > kWaitNs) {
+          gave_up = true;
+          break;
+        }
+      }
+      st_desc(desc + (size_t)c * D1 + d, make_desc(epoch, 2u, before + own));
+    }
+    gbase[d] = before;
   }
+  if (gave_up) atomicOr(status, 4u);
+  // the totals of k_count give the segment starts (into cnt, free now)
+  pdl_wait();
+  __syncthreads();
+  uint32_t *seg = cnt;
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) seg[d] = __ldcg(totals + d);
+  __syncthreads();
+  block_scan_256(seg, D1);
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) gbase[d] += seg[d];
+  if (c == 0) {  // the tile table: segment starts and tile starts over the D+1 buckets
+    uint32_t *mseg = meta + 1, *tst = meta + 1 + (D + 2);
+    uint32_t *tiles = seg + D1;  // cnt has kWarps * D1 words
+    for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
+      mseg[d] = seg[d];
+      tiles[d] = (__ldcg(totals + d) + kTile - 1) / kTile;
+    }
+    __syncthreads();
+    const uint32_t last_tiles = tiles[D];
+    __syncthreads();
+    block_scan_256(tiles, D1);
+    for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) tst[d] = tiles[d];
+    if (threadIdx.x == 0) {
+      mseg[D1] = (uint32_t)n;
+      tst[D1] = tiles[D] + last_tiles;
+      meta[0] = tiles[D] + last_tiles;
+    }
+  }
+  __syncthreads();
   // coalesced copy-out: consecutive slots of one decoder go to consecutive
   // positions of that decoder's segment
   for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
@@ -345,33 +325,20 @@ __global__ void __launch_bounds__(kBucketThreads) k_scatter(Assets A, const ntc_
     perm[pos] = (uint32_t)(cbase + j);
     reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
   }
-  if (SPREAD) {
-    __shared__ bool last;
-    uint32_t *ticket = cursor + D1;
-    if (threadIdx.x == 0) last = ticket_no == gridDim.x - 1;
-    __syncthreads();
-    if (!last) return;
+  // the last CTA to finish clears the totals and tickets for the next call
+  // (every CTA has read the totals before it takes its done ticket)
+  __syncthreads();
+  if (threadIdx.x == 0) {
     __threadfence();
-    // every chunk has reserved its runs: counts per decoder and tile starts
-    uint32_t *segc = meta + 1, *tst = meta + 1 + (D1 + 1);
-    for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) {
-      const uint32_t c = ((volatile uint32_t *)cursor)[d];
-      segc[d] = c;
-      loff[d] = (c + kTile - 1) / kTile;
-      cursor[d] = 0;
-    }
-    __syncthreads();
-    const uint32_t last_tiles = loff[D1 - 1];
-    __syncthreads();
-    block_scan_256(loff, D1);
-    for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) tst[d] = loff[d];
-    if (threadIdx.x == 0) {
-      const uint32_t T = loff[D1 - 1] + last_tiles;
-      tst[D1] = T;
-      segc[D1] = 0;
-      meta[0] = T;
-      *ticket = 0;
-    }
+    s_last = atomicAdd(done_ticket, 1u) == chunks - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (uint32_t d = threadIdx.x; d < D1; d += blockDim.x) totals[d] = 0;
+  if (threadIdx.x == 0) {
+    *start_ticket = 0;
+    *done_ticket = 0;
   }
 }
 
@@ -394,42 +361,42 @@ __global__ void k_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles
 
 }  // namespace
 
-size_t bucket_scratch_counts(uint32_t D, size_t n) {
-  size_t chunks = (n + kBucketChunk - 1) / kBucketChunk;
-  return (size_t)(D + 1) * chunks;
-}
+size_t bucket_chunks(size_t n) { return (n + kBucketChunk - 1) / kBucketChunk; }
+size_t bucket_desc_words(uint32_t D, size_t n) { return ((size_t)D + 1) * bucket_chunks(n); }
+size_t bucket_meta_words(uint32_t D) { return meta_words(D) + ((size_t)D + 1) + 2; }
 
 cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
                           cudaStream_t st, int *launches, unsigned int *status) {
-  const uint32_t chunks = (uint32_t)((n + kBucketChunk - 1) / kBucketChunk);
-  const uint32_t D = A.num_decoders;
-  const size_t cnt_bytes = (size_t)kWarps * (D + 1) * sizeof(uint32_t);
-  const size_t smem = (size_t)kBucketChunk * 16 + cnt_bytes;
-  const size_t smem_scatter = (size_t)kBucketChunk * (16 + 2 + 2) + cnt_bytes + 2 * (D + 1) * sizeof(uint32_t);
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaFuncSetAttribute(k_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    cudaFuncSetAttribute(k_scatter<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    attr_done = true;
-  }
-  // totals[D+1] and the ticket live after meta
-  uint32_t *totals = s.meta + meta_words(D);
-  uint32_t *ticket = totals + (D + 1);
-  if (s.cursor) {  // single pass: reserve runs in per-decoder regions
-    cudaFuncSetAttribute(k_scatter<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    k_scatter<true><<<chunks, kBucketThreads, smem_scatter, st>>>(A, q, n, nullptr, chunks, s.meta, s.perm,
-                                                                   s.sorted, status, s.cursor, s.cap);
-    *launches += 1;
-    return cudaGetLastError();
-  }
-  k_hist<<<chunks, kBucketThreads, smem, st>>>(A, q, n, s.counts, chunks, status);
-  cudaError_t e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, (uint32_t)n, totals,
-                             s.meta, ticket);
-  if (e == cudaSuccess)
-    e = launch_pdl(k_scatter<false>, dim3(chunks), dim3(kBucketThreads), smem_scatter, st, A, q, n,
-                   (const uint32_t *)s.counts, chunks, s.meta, s.perm, s.sorted, status, (uint32_t *)nullptr,
-                   0u);
-  *launches += 3;
+  const uint32_t chunks = (uint32_t)bucket_chunks(n);
+  const uint32_t D1 = A.num_decoders + 1;
+  const size_t smem_count = (size_t)kWarps * D1 * sizeof(uint32_t);
+  const size_t smem_place = (size_t)kBucketChunk * (16 + 2 + 2) + (size_t)(kWarps + 2) * D1 * sizeof(uint32_t);
+  static PerDevice attrs;
+  cudaError_t e = attrs.once([]() {
+    cudaError_t r = cudaFuncSetAttribute(k_count, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    if (r == cudaSuccess)
+      r = cudaFuncSetAttribute(k_place, cudaFuncAttributeMaxDynamicSharedMemorySize, 210 * 1024);
+    return r;
+  });
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 1, smem_sm = 233472, thr_sm = 2048;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+  cudaDeviceGetAttribute(&thr_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev);
+  // k_count: a grid that is resident at once (by threads and by its shared
+  // memory, which grows with the decoder count), each CTA striding over chunks
+  size_t occ = (size_t)thr_sm / kBucketThreads;
+  const size_t by_smem = (size_t)smem_sm / (smem_count + 1024);
+  if (by_smem < occ) occ = by_smem;
+  if (occ < 1) occ = 1;
+  size_t grid = (size_t)sms * occ;
+  if (grid > chunks) grid = chunks;
+  uint32_t *totals = s.meta + meta_words(A.num_decoders);
+  k_count<<<(unsigned)grid, kBucketThreads, smem_count, st>>>(A, q, n, chunks, totals);
+  e = launch_pdl(k_place, dim3(chunks), dim3(kBucketThreads), smem_place, st, A, q, n, chunks, s.meta, s.desc,
+                 s.epoch, s.perm, s.sorted, status);
+  *launches += 2;
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

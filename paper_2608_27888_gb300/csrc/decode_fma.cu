@@ -172,11 +172,11 @@ __global__ void k_pack_fma(const float *w32, uint32_t H, uint32_t C, uint8_t *im
 template <int H, int CP, typename T>
 cudaError_t launch_fma_t(const Assets &A, const WeightImages &W, const ntc_query *q, size_t n, float *out,
                          unsigned long long *err, int num_sms, cudaStream_t st) {
-  static int occ = -1;
-  if (occ < 0) {
-    occ = resident_ctas(k_decode_divergent_fma<H, CP, T>, 128, 0);
-    if (occ < 1) occ = 1;
-  }
+  static PerDevice occ_of;
+  const int occ = occ_of.value([&]() {
+    const int o = resident_ctas(k_decode_divergent_fma<H, CP, T>, 128, 0);
+    return o < 1 ? 1 : o;
+  });
   const size_t blocks = (n + 127) / 128;
   size_t grid = (size_t)num_sms * occ * 8;
   if (grid > blocks) grid = blocks;

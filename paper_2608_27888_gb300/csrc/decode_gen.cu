@@ -168,7 +168,6 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
   if (wg == 0) {
     // ------------------------------------------------------------- producer
     TileWalk walk;
-    walk.cap = B.spread_cap;
     // tile j's query record and output row; the next tile's are loaded while
     // tile j is gathered
     auto load_row = [&](uint32_t jj, uint32_t &d_, uint32_t &len_, ntc_query &q_, uint32_t &oi_) {
@@ -267,7 +266,6 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
     uint32_t cur = 0xFFFFFFFFu, mph = 0, wph = 0;
     const uint32_t sW = saddr(smem);
     TileWalk cwalk;
-    cwalk.cap = B.spread_cap;
     const uint32_t id_h = instr_desc<BF16>(H), id_o = instr_desc<BF16>(16);
     const uint32_t act = G.activation == 1 && G.slope >= 0.0f && G.slope <= 1.0f ? 2u : G.activation;
     const uint32_t slope2 = pack<BF16>(G.slope, G.slope);

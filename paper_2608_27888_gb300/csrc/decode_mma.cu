@@ -392,12 +392,12 @@ cudaError_t launch_mma_t(const Assets &A, const WeightImages &W, const Buckets &
                          float *out, unsigned long long *err, int num_sms, cudaStream_t st) {
   using I = MmaImage<H>;
   const size_t smem = ((I::bytes + 15) & ~(size_t)15) + (size_t)4 * 32 * kFeatStride * 2;
-  static int occ = -1;
-  if (occ < 0) {
+  static PerDevice occ_of;
+  const int occ = occ_of.value([&]() {
     cudaFuncSetAttribute(k_decode_mma<H, NT3, BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    occ = resident_ctas(k_decode_mma<H, NT3, BF16>, kTile, smem);
-    if (occ < 1) occ = 1;
-  }
+    const int o = resident_ctas(k_decode_mma<H, NT3, BF16>, kTile, smem);
+    return o < 1 ? 1 : o;
+  });
   size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms * occ;
   if (grid > max_tiles) grid = max_tiles;
@@ -408,11 +408,11 @@ cudaError_t launch_mma_t(const Assets &A, const WeightImages &W, const Buckets &
 template <int H, int NT3, bool BF16>
 cudaError_t launch_div_t(const Assets &A, const WeightImages &W, const ntc_query *q, size_t n,
                          float *out, unsigned long long *err, int num_sms, cudaStream_t st) {
-  static int occ = -1;
-  if (occ < 0) {
-    occ = resident_ctas(k_decode_divergent<H, NT3, BF16>, 128, 0);
-    if (occ < 1) occ = 1;
-  }
+  static PerDevice occ_of;
+  const int occ = occ_of.value([&]() {
+    const int o = resident_ctas(k_decode_divergent<H, NT3, BF16>, 128, 0);
+    return o < 1 ? 1 : o;
+  });
   size_t blocks = (n + 127) / 128;
   size_t grid = (size_t)num_sms * occ * 4;
   if (grid > blocks) grid = blocks;

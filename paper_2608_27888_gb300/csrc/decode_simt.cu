@@ -227,12 +227,12 @@ template <int H, int CP>
 cudaError_t launch_fp32_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
                           float *out, unsigned long long *err, int num_sms, cudaStream_t st) {
   const size_t smem = f32_image_floats(H, W.out_dim) * sizeof(float);
-  static int occ = -1;
-  if (occ < 0) {
+  static PerDevice occ_of;
+  const int occ = occ_of.value([&]() {
     cudaFuncSetAttribute(k_decode_fp32<H, CP>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    occ = resident_ctas(k_decode_fp32<H, CP>, kTile, smem);
-    if (occ < 1) occ = 1;
-  }
+    const int o = resident_ctas(k_decode_fp32<H, CP>, kTile, smem);
+    return o < 1 ? 1 : o;
+  });
   size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms * occ;
   if (grid > max_tiles) grid = max_tiles;

@@ -1,652 +1,13 @@
-// tcgen05 / TMEM gather-decode (sm_103a), warp-specialised.
-//
-// One persistent CTA per SM runs NP producer and NC consumer warpgroups.
-// Tiles (128 queries of one decoder, from the bucketing) are dealt out
-// round-robin over the CTAs, so at any moment the whole GPU works on
-// neighbouring tiles -- one decoder and, in set-major bucket order, one set's
-// latents, which keeps them in L2.  Inside a CTA, consumer c takes the CTA's
-// tiles c, c + NC, ... and is fed by its own producers through a private ring
-// of SC tensor-memory stages.
-//   Producer (one thread per tile row): loads the query record and its output
-//     row index, computes the bilinear taps of both latent grids (Sec. 3.1, the
-//     same fp32 operations as the reference addressing), fetches each bilinear
-//     row as one 32-byte load from the row-pair copy of the latents, blends in
-//     packed fp16 (the latents' own type) and stores the fp16/bf16 feature row
-//     [16] into its stage with tcgen05.st (warp q writes TMEM lanes
-//     32q..32q+31, exactly its rows).
-//   Consumer (one elected thread issues every MMA): layer 1 reads A from the
-//     stage and B (the decoder's weights, copied by a TMA bulk copy whenever
-//     the decoder changes) from shared memory; its completion frees the stage;
-//     the ReLU/convert epilogue goes TMEM -> registers -> TMEM; layers 2 and 3
-//     read their A operand from TMEM too; each layer's bias is one more K step
-//     whose A is a shared block with a 1 in K column 0.  Layer 3 accumulates
-//     in the consumer's own 16 output columns, so the next tile's layer 1 is
-//     issued before it completes; the sigmoid epilogue then scatters rows to
-//     out[perm[i]].
-// Shared-memory B operands use the no-swizzle K-major canonical layout: 8-row
-// x 16-byte core matrices, K-adjacent core matrices 128 B apart (LBO), 8-row
-// groups K*16 B apart (SBO).  Every wait is bounded by time; on expiry the
-// kernel records an error and stops cleanly (TMEM is always released).
-#include "tcgen05.cuh"
+// tcgen05 / TMEM gather-decode (sm_103a): the production instantiations of
+// the kernel in decode_tc.cuh, and the weight-image packing.
+#include "decode_tc.cuh"
 
 namespace ntc {
 
-constexpr int kTcKA = 32;  // K of layer 1's weight image: 16 features + the bias K step
 size_t tc_image_bytes(uint32_t H) {
   const size_t KH = H + 16;
   return (size_t)H * kTcKA * 2 + (size_t)H * KH * 2 + (size_t)16 * KH * 2;
 }
-
-namespace {
-
-template <int H>
-struct TcLayout {
-  static constexpr uint32_t KH = H + 16;
-  static constexpr uint32_t W1 = H * kTcKA * 2;
-  static constexpr uint32_t W2 = H * KH * 2;
-  static constexpr uint32_t W3 = 16 * KH * 2;
-  static constexpr uint32_t WIMG = W1 + W2 + W3;
-};
-
-// Latent taps of one query from one mip, loaded ahead of use: 2 levels x 4
-// taps; a mip blend factor is folded into the weights.
-struct Taps {
-  static constexpr int N = 8;
-  uint4 raw[N];
-  float w[N];
-};
-
-// Mip selection of one query row, kept between the two fetch phases of a
-// kernel that may blend mips.
-struct MipPick {
-  int lo = 0;
-  float t = 0.0f;
-};
-
-// One axis of the tap addressing, fp32 round-to-nearest with no contraction
-// (the same operations, in the same order, as the reference addressing).
-// WRAP: c is finite and the texel pair wraps at the edge; clamp: both texels
-// are clamped into [0, n-1].
-template <bool WRAP>
-__device__ __forceinline__ void axis_pair(float c, uint32_t n, uint32_t &i0, uint32_t &i1, float &frac) {
-  const float x = WRAP ? __fsub_rn(__fmul_rn(__fsub_rn(c, floorf(c)), (float)n), 0.5f)
-                       : __fsub_rn(__fmul_rn(c, (float)n), 0.5f);
-  const float x0f = floorf(x);
-  frac = __fsub_rn(x, x0f);
-  if (WRAP) {
-    const int x0 = (int)x0f;  // in [-1, n-1]
-    i0 = x0 < 0 ? n - 1 : (uint32_t)x0;
-    const uint32_t a1 = (uint32_t)(x0 + 1);
-    i1 = a1 == n ? 0u : a1;
-  } else {
-    const int x0 = (int)fminf(fmaxf(x0f, -1.0f), (float)n);
-    i0 = (uint32_t)min(max(x0, 0), (int)n - 1);
-    i1 = (uint32_t)min(x0 + 1, (int)n - 1);
-  }
-}
-
-// Both texels of one bilinear row from the row-pair copy: one 32-byte load.
-struct alignas(32) TexelPair {
-  uint4 a, b;
-};
-__device__ __forceinline__ void ld_pair(const TexelPair *p, uint4 &a, uint4 &b) {
-  asm volatile("ld.global.nc.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-               : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
-               : "l"(p));
-}
-
-// Issue the tap loads of one grid (taps 00, 10 from row j0; 01, 11 from row
-// j1) and compute their bilinear weights, scaled by sc.  In-grid offsets are
-// 32-bit (a grid holds fewer than 2^32 texels).  Clamp mode at an edge has
-// x0 = x1, while the pair at x0 holds x0 and its right neighbour: the whole
-// row weight then goes to the first texel.
-template <bool WRAP>
-__device__ __forceinline__ void grid_fetch(const uint4 *pair, const GridDesc &g, float u, float v, float sc,
-                                           uint4 *raw, float *w) {
-  uint32_t i0, i1, j0, j1;
-  float fx, fy;
-  axis_pair<WRAP>(u, g.W, i0, i1, fx);
-  axis_pair<WRAP>(v, g.H, j0, j1, fy);
-  const TexelPair *p = reinterpret_cast<const TexelPair *>(pair) + g.base;
-  ld_pair(p + (j0 * g.W + i0), raw[0], raw[1]);
-  ld_pair(p + (j1 * g.W + i0), raw[2], raw[3]);
-  const float ax = __fsub_rn(1.0f, fx), ay = __fsub_rn(1.0f, fy);
-  float w00 = __fmul_rn(ax, ay), w10 = __fmul_rn(fx, ay), w01 = __fmul_rn(ax, fy), w11 = __fmul_rn(fx, fy);
-  if (!WRAP && i1 == i0) {
-    w00 = __fadd_rn(w00, w10);
-    w01 = __fadd_rn(w01, w11);
-    w10 = w11 = 0.0f;
-  }
-  w[0] = w00 * sc;
-  w[1] = w10 * sc;
-  w[2] = w01 * sc;
-  w[3] = w11 * sc;
-}
-
-// All tap loads of one query from mip lo, issued before any is consumed.  A
-// row that is not good (padding, bad set id or UV, bad bucket) fetches texel
-// (0, 0) of set 0 instead: no branch and no out-of-range address; its flag
-// marks it.  TRI: the kernel may blend mips, so the mip is selected per row
-// and mip lo is weighted by 1 - t; otherwise every grid has one mip.
-template <bool TRI, bool WRAP>
-__device__ __forceinline__ void issue_taps(const Assets &A, const GridDesc *grids, const ntc_query &q,
-                                           bool good, Taps &tp, MipPick &mp) {
-  const uint32_t sid = good ? q.set_id : 0u;
-  const float u = good ? q.u : 0.0f, v = good ? q.v : 0.0f;
-  if (TRI) mp.lo = select_mip(good ? q.lod : 0.0f, A.num_mips, mp.t);
-  const uint32_t M = TRI ? A.num_mips : 1u;
-  const GridDesc *g = grids + (size_t)sid * kLevels * M;
-  const float s = TRI ? __fsub_rn(1.0f, mp.t) : 1.0f;
-#pragma unroll
-  for (int k = 0; k < kLevels; ++k) grid_fetch<WRAP>(A.pair, g[k * M + mp.lo], u, v, s, tp.raw + 4 * k, tp.w + 4 * k);
-}
-
-// The second phase of a mip blend, one level at a time (fewer registers live
-// than a whole query's taps): the taps of level k at mip lo + 1, weighted by
-// t, for the rows with t > 0 (the others load nothing and get zero weights, so
-// their accumulation is unchanged).
-template <bool WRAP>
-__device__ __forceinline__ void issue_level_hi(const Assets &A, const GridDesc *grids, const ntc_query &q,
-                                               bool good, const MipPick &mp, int k, uint4 (&raw)[4],
-                                               float (&w)[4]) {
-  if (good && mp.t > 0.0f) {
-    const uint32_t M = A.num_mips;
-    grid_fetch<WRAP>(A.pair, grids[((size_t)q.set_id * kLevels + k) * M + mp.lo + 1], q.u, q.v, mp.t, raw, w);
-  } else {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      w[i] = 0.0f;
-      raw[i] = make_uint4(0, 0, 0, 0);
-    }
-  }
-}
-
-// acc[c/2] += w * tap[c] over the 8 channels of one tap, in packed fp16 pairs
-// (the latents' own type; hfma2, the first tap multiplies): the feature row
-// becomes the fp16/bf16 A operand, so the blend needs no fp32 conversions.
-template <bool FIRST>
-__device__ __forceinline__ void accum_tap_x2(__half2 (&acc)[4], uint4 raw, float w) {
-  const __half2 ww = __float2half2_rn(w);
-  const __half2 *h = reinterpret_cast<const __half2 *>(&raw);
-#pragma unroll
-  for (int p = 0; p < 4; ++p) acc[p] = FIRST ? __hmul2(ww, h[p]) : __hfma2(ww, h[p], acc[p]);
-}
-
-// Feature accumulation: acc[k][c/2] over the 8 channels of level k, all taps
-// of mip lo first (FIRST: the first tap multiplies), then those of mip lo + 1.
-template <bool FIRST>
-__device__ __forceinline__ void accum_taps(const Taps &tp, __half2 (&acc)[kLevels][4]) {
-#pragma unroll
-  for (int k = 0; k < kLevels; ++k) {
-    accum_tap_x2<FIRST>(acc[k], tp.raw[k * 4], tp.w[k * 4]);
-#pragma unroll
-    for (int p = 1; p < 4; ++p) accum_tap_x2<false>(acc[k], tp.raw[k * 4 + p], tp.w[k * 4 + p]);
-  }
-}
-
-template <bool BF16>
-__device__ __forceinline__ void pack_row(const __half2 (&acc)[kLevels][4], uint32_t (&packed)[8]) {
-#pragma unroll
-  for (int k = 0; k < kLevels; ++k)
-#pragma unroll
-    for (int p = 0; p < 4; ++p) {
-      if (BF16) {
-        const float2 x = __half22float2(acc[k][p]);
-        packed[k * 4 + p] = pack<true>(x.x, x.y);
-      } else {
-        packed[k * 4 + p] = *reinterpret_cast<const uint32_t *>(&acc[k][p]);
-      }
-    }
-}
-
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
-      "l"(src), "r"(bytes), "r"(bar)
-      : "memory");
-}
-
-constexpr uint32_t kSmemTileTable = 1024;  // staged when D + 2 <= this
-constexpr uint32_t kSmemGrids = 1024;      // staged when S * 2 * M <= this
-
-
-// Shared-memory plan of the warp-specialised kernel: only the decoders' weights
-// (the B operands) and bookkeeping live in shared memory; every A operand and
-// accumulator lives in tensor memory, so most of the SM's L1/shared array stays
-// L1, which holds the in-flight latent gathers.
-template <int H, int NC, int SC>
-struct TmSmem {
-  using L = TcLayout<H>;
-  static constexpr int S = NC * SC;                                     // stages in all rings
-  static constexpr size_t weights = 0;                                  // per consumer
-  // per stage and use parity: 128 output rows, 0xFFFFFFFF for a row that is
-  // not good (never a valid row: n <= 2^32 - 256).  Two slots per stage: the
-  // producer's next use of a stage writes the other slot, so a consumer warp
-  // that reads late never sees the following tile's rows.
-  static constexpr size_t oidx = weights + (size_t)NC * L::WIMG;
-  static constexpr size_t bars = oidx + (size_t)S * 2 * 128 * 4;
-  static constexpr int nbars = 2 * S + 3 * NC;                          // full, empty, mma, weights, output
-  static constexpr size_t misc = bars + (size_t)nbars * 8;
-  static constexpr size_t tiles = misc + 64;
-  static constexpr size_t grids = tiles + 2 * kSmemTileTable * 4;
-  static constexpr size_t total = grids + kSmemGrids * sizeof(GridDesc);
-};
-
-// Tensor-memory plan (columns).  The NC fp32 accumulators (H columns each)
-// come first, so every accumulator starts on a multiple of H; then each
-// consumer's hidden A operand (H/2 columns: two 16-bit K elements per column);
-// then the layer-1 feature operands [128 x 16] of the NC * SC ring stages (8
-// columns each); last, one shared 8-column block holding a 1 in K column 0 and
-// zeros elsewhere: the A operand of every layer's bias K step (the decoder image
-// keeps each layer's bias as the first row of an extra 16-row K block); then
-// each consumer's own 16-column accumulator for the output layer, so that the
-// next tile's layer 1 can run in the hidden accumulator meanwhile.
-template <int H, int NC, int SC>
-struct TmCols {
-  static constexpr uint32_t HID = NC * H;
-  static constexpr uint32_t STG = HID + NC * (H / 2);
-  static constexpr uint32_t ONES = STG + NC * SC * 8;
-  static constexpr uint32_t OUT = (ONES + 8 + 15) / 16 * 16;
-  static constexpr uint32_t used = OUT + NC * 16;
-  static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
-  static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
-  static __device__ __forceinline__ uint32_t acc(uint32_t c) { return c * H; }
-  static __device__ __forceinline__ uint32_t hid(uint32_t c) { return HID + c * (H / 2); }
-  // layer-1 A operand of stage s (= consumer * SC + st)
-  static __device__ __forceinline__ uint32_t a1(uint32_t s) { return STG + 8 * s; }
-  static __device__ __forceinline__ uint32_t out(uint32_t c) { return OUT + 16 * c; }
-};
-
-// Warp-specialised gather-decode with tensor-memory operands.
-//   Consumer warpgroups (the last NC) each decode the CTA's local tiles
-//   k = c, c + NC, ... (j = k / NC counts a consumer's tiles).  Each consumer has
-//   a private ring of SC stages in tensor memory, filled by its own R = NP / NC
-//   producer warpgroups: tile j of consumer c is gathered by producer c + NC *
-//   (j mod R) into stage j mod SC.  SC is a multiple of R, so every stage has one
-//   producer and one consumer and successive uses of a stage are ordered by
-//   program order on both sides -- an mbarrier parity wait can then never be two
-//   phases ahead of its barrier.
-//   Producer: each thread computes the taps of one query row, blends them in
-//   packed fp16 and stores the fp16/bf16 feature row into the stage's TMEM A
-//   region (tcgen05.st; warp q of a warpgroup owns TMEM lanes 32q..32q+31,
-//   exactly its rows), with the row's output index (or 0xFFFFFFFF if the row is
-//   not good) in shared memory, in the slot of the stage's use parity; four
-//   warp arrivals fill the stage.  The next tile's query record and output
-//   index are loaded while the current tile is gathered.
-//   Consumer: layer 1 reads A from the stage and B (weights) from shared memory;
-//   its completion empties the stage; the ReLU/convert epilogue goes TMEM ->
-//   registers -> TMEM; layers 2 and 3 read their A from TMEM too.  Layer 3
-//   writes the consumer's own output columns and completes on its own
-//   barrier, so the next tile's layer 1 is issued first; then the sigmoid
-//   epilogue scatters rows to out[perm[i]].
-// CTA b owns the global tiles b, b + grid, b + 2 grid, ...
-template <int H, bool BF16, bool TRI, bool WRAP, int CP, int NP, int NC, int SC>
-__global__ void __launch_bounds__((NP + NC) * 128, 1)
-    k_decode_tm(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
-                unsigned int *status, int vec_out) {
-  static_assert(NP % NC == 0 && SC % (NP / NC) == 0, "each ring stage needs one producer");
-  constexpr int R = NP / NC;  // producers per consumer
-  constexpr int S = NC * SC;
-  using L = TcLayout<H>;
-  using M = TmSmem<H, NC, SC>;
-  using TC = TmCols<H, NC, SC>;
-  extern __shared__ __align__(128) uint8_t smem[];
-  const int role = threadIdx.x >> 7, row = threadIdx.x & 127, warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const uint32_t lanes = (uint32_t)((warp & 3) * 32) << 16;  // this warp's TMEM lane quadrant
-  const uint32_t sbase = saddr(smem);
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + M::bars);
-  auto full_bar = [&](uint32_t s) { return saddr(bars + s); };
-  auto empty_bar = [&](uint32_t s) { return saddr(bars + S + s); };
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + M::misc);
-  volatile uint32_t *abort_flag = tmem_slot + 1;
-  // [NC][2]: consumer c's decision to stop, written for its tile jc in slot jc & 1
-  volatile uint32_t *stop_flag = tmem_slot + 2;
-  const uint32_t D = A.num_decoders, C = W.out_dim;
-
-  // no stage has rows yet: a consumer that stops on a wait timeout reads
-  // all-bad rows, never an uninitialised output index
-  for (uint32_t i = threadIdx.x; i < (uint32_t)S * 2 * 128; i += blockDim.x)
-    reinterpret_cast<uint32_t *>(smem + M::oidx)[i] = 0xFFFFFFFFu;
-  const GridDesc *grids = A.pgrids;  // grid bases in the row-pair copy
-  const uint32_t ngrids = A.num_sets * kLevels * A.num_mips;
-  if (ngrids <= kSmemGrids) {
-    GridDesc *s_grids = reinterpret_cast<GridDesc *>(smem + M::grids);
-    for (uint32_t i = threadIdx.x; i < ngrids; i += blockDim.x) s_grids[i] = A.pgrids[i];
-    grids = s_grids;
-  }
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < S; ++i) {
-      mbar_init(full_bar(i), 4);   // one arrival per producer warp
-      mbar_init(empty_bar(i), 1);  // the consumer's layer-1 commit
-    }
-    for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), 1);
-    *abort_flag = 0;
-    for (int i = 0; i < 2 * NC; ++i) stop_flag[i] = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
-  }
-  if (warp == 0) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
-                     saddr(tmem_slot)),
-                 "r"(TC::alloc)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
-  }
-  fence_before();
-  __syncthreads();
-  fence_after();
-  const uint32_t tmem_base = *tmem_slot;
-  const uint32_t one = BF16 ? 0x3F80u : 0x3C00u;  // 1.0 in the low half, 0 in the high half
-  if (warp < 4) {  // the shared bias operand: K column 0 is 1, the rest 0
-    const uint32_t z[8] = {one, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-    tmem_st8(tmem_base + TC::ONES + lanes, z);
-    tmem_wait_st();
-  }
-  // everything above is independent of the bucketing; the tile table is not
-  pdl_wait();
-  const uint32_t *seg = B.meta + 1, *tst = B.meta + 1 + (D + 2);
-  if (!B.identity_n && D + 2 <= kSmemTileTable) {
-    uint32_t *s_seg = reinterpret_cast<uint32_t *>(smem + M::tiles);
-    uint32_t *s_tst = s_seg + kSmemTileTable;
-    for (uint32_t i = threadIdx.x; i < D + 2; i += blockDim.x) {
-      s_seg[i] = __ldg(seg + i);
-      s_tst[i] = __ldg(tst + i);
-    }
-    seg = s_seg;
-    tst = s_tst;
-  }
-  fence_before();
-  __syncthreads();
-  fence_after();
-  const uint32_t T = B.identity_n ? (B.identity_n + kTile - 1) / kTile : __ldg(B.meta);
-  const uint32_t grid = gridDim.x;
-  const uint32_t K = blockIdx.x < T ? (T - blockIdx.x + grid - 1) / grid : 0;  // local tiles
-
-  if (role < NP) {
-    // ------------------------------------------------------------ producer
-    const uint32_t pc = role % NC, pq = role / NC;  // serves consumer pc, tiles j = pq mod R
-    auto tile_of = [&](uint32_t j) { return pc + NC * j; };
-    uint32_t j = pq;
-    uint32_t dec = D, start = 0, len = 0, oi = 0;
-    ntc_query q;
-    TileWalk walk;
-    walk.ident_n = B.identity_n;
-    walk.cap = B.spread_cap;
-    if (tile_of(j) < K) {
-      walk.at(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
-      if ((uint32_t)row < len) {
-        q = load_query(B.sorted + start + row);
-        oi = B.identity_n ? start + row : __ldg(B.perm + start + row);
-      }
-    }
-    for (; tile_of(j) < K; j += R) {
-      if (*abort_flag) break;
-      // the next tile's query record and output row go in flight early: before
-      // the taps, or (TRI, where registers are scarcer) once the first mip's
-      // taps are consumed
-      uint32_t ndec = D, nstart = 0, nlen = 0, noi = 0;
-      ntc_query nq;
-      auto prefetch = [&]() {
-        if (tile_of(j + R) < K) {
-          walk.at(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
-          if ((uint32_t)row < nlen) {
-            nq = load_query(B.sorted + nstart + row);
-            noi = B.identity_n ? nstart + row : __ldg(B.perm + nstart + row);
-          }
-        }
-      };
-      if (!TRI) prefetch();
-      const bool valid = (uint32_t)row < len;
-      const bool good = valid && dec < D && !query_bad(A, q);
-      Taps taps;
-      MipPick mp;
-      issue_taps<TRI, WRAP>(A, grids, q, good, taps, mp);
-      // bad rows (set id out of range, non-finite UV, or the bad bucket) decode to NaN
-      const bool bad = valid && !good;
-      const uint32_t badm = __ballot_sync(0xFFFFFFFFu, bad);
-      if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
-      if (bad)
-        for (uint32_t cc = 0; cc < C; ++cc) out[(size_t)oi * C + cc] = __int_as_float(0x7fc00000);
-      __half2 acc[kLevels][4];
-      accum_taps<true>(taps, acc);
-      if (TRI) prefetch();
-      if (TRI && __any_sync(0xFFFFFFFFu, good && mp.t > 0.0f)) {  // some row blends two mips
-#pragma unroll
-        for (int k = 0; k < kLevels; ++k) {
-          uint4 raw[4];
-          float w[4];
-          issue_level_hi<WRAP>(A, grids, q, good, mp, k, raw, w);
-#pragma unroll
-          for (int p = 0; p < 4; ++p) accum_tap_x2<false>(acc[k], raw[p], w[p]);
-        }
-      }
-      uint32_t a[8];
-      pack_row<BF16>(acc, a);
-      const uint32_t s = pc * SC + j % SC, n = j / SC;
-      if (!mbar_wait(empty_bar(s), (n & 1) ^ 1)) {  // the stage's previous tile has left layer 1
-        atomicOr(status, 1u);
-        *abort_flag = 1;
-      }
-      fence_after();
-      tmem_st8(tmem_base + TC::a1(s) + lanes, a);
-      tmem_wait_st();
-      reinterpret_cast<uint32_t *>(smem + M::oidx)[(s * 2 + (n & 1)) * 128 + row] = good ? oi : 0xFFFFFFFFu;
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(full_bar(s));
-      dec = ndec;
-      len = nlen;
-      q = nq;
-      oi = noi;
-    }
-  } else {
-    // ------------------------------------------------------------ consumer
-    const int c = role - NP;
-    const int wgid = role;  // named barrier id role + 1
-    const bool poller = (row >> 5) == (c & 3);  // one waiting warp per consumer, spread over the sub-partitions
-    const uint32_t tD = tmem_base + TC::acc(c);  // accumulator
-    const uint32_t tH = tmem_base + TC::hid(c);  // hidden A operand
-    const uint32_t tOnes = tmem_base + TC::ONES; // the bias K step's A operand
-    const uint32_t tO = tmem_base + TC::out(c);  // the output layer's accumulator
-    const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
-    const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
-    const uint32_t obar = saddr(bars + 2 * S + 2 * NC + c);  // the output layer's completion
-    uint32_t ph = 0, wph = 0, oph = 0, cur = 0xFFFFFFFFu;
-    TileWalk cwalk;
-    cwalk.ident_n = B.identity_n;
-    cwalk.cap = B.spread_cap;
-    constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
-    const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
-    auto wait_bar = [&](uint32_t b, uint32_t parity) {
-      if (poller && !mbar_wait(b, parity)) {
-        atomicOr(status, 1u);
-        *abort_flag = 1;
-      }
-    };
-    // TMEM accumulator -> ReLU -> fp16/bf16 pairs -> hidden A operand
-    auto hidden = [&]() {
-#pragma unroll 1
-      for (int c0 = 0; c0 < H; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(tD + lanes + c0, v);
-        tmem_wait_ld();
-        uint32_t p[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) p[i] = pack_relu<BF16>(v[2 * i], v[2 * i + 1]);
-        tmem_st16(tH + lanes + c0 / 2, p);
-      }
-      tmem_wait_st();
-    };
-    // Start tile k: its decoder's weights, wait for its A stage (with the
-    // rows' output indices) and issue layer 1.  Requires this consumer's
-    // previous tile to have read its hidden accumulator (its output layer may
-    // still run: that reads only the hidden operand and writes only tO).  The
-    // barrier also carries the decision to stop, the same for every warp.
-    auto begin = [&](uint32_t k, uint32_t &dec, uint32_t &oi, bool &good, bool &stop) {
-      const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
-      uint32_t start, len;
-      cwalk.at(seg, tst, D, t, dec, start, len);
-      bool wpend = false;
-      if (dec < D && dec != cur) {
-        if (row == 0) bulk_g2s(sW1, W.tc + (size_t)dec * W.tc_stride, L::WIMG, wbar);
-        wpend = true;
-        cur = dec;
-      }
-      wait_bar(full_bar(s), n & 1);
-      if (wpend) {
-        wait_bar(wbar, wph);
-        wph ^= 1;
-      }
-      if (row == 0) stop_flag[2 * c + (jc & 1)] = *abort_flag;
-      wg_bar(wgid);
-      stop = stop_flag[2 * c + (jc & 1)] != 0;
-      oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[(s * 2 + (n & 1)) * 128 + row];
-      good = oi != 0xFFFFFFFFu;
-      if (row == 0) {
-        fence_after();
-        if (dec < D) {
-          const uint32_t tA = tmem_base + TC::a1(s);
-          umma_ta(tD, tA, dW1, id_hidden, 0);
-          umma_ta(tD, tOnes, dW1 + 16, id_hidden, 1);  // + bias
-          umma_commit(mbar);
-          umma_commit(empty_bar(s));
-        } else {
-          mbar_arrive(empty_bar(s));  // a tile of bad queries: nothing to multiply
-        }
-      }
-    };
-    uint32_t k = c, dec = D, oi = 0;
-    bool good = false, stop = false;
-    if (k < K) begin(k, dec, oi, good, stop);
-    while (k < K) {
-      if (dec < D) {
-#pragma unroll 1
-        for (int layer = 0; layer < 2; ++layer) {
-          wait_bar(mbar, ph);
-          ph ^= 1;
-          wg_bar(wgid);
-          fence_after();
-          hidden();
-          fence_before();
-          wg_bar(wgid);
-          if (row == 0) {
-            fence_after();
-            if (layer == 0) {
-#pragma unroll
-              for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
-              umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
-              umma_commit(mbar);
-            } else {
-#pragma unroll
-              for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, kq);
-              umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 1);  // + bias
-              umma_commit(obar);
-            }
-          }
-        }
-      }
-      // the next tile's layer 1 runs while this tile's output layer finishes
-      // and its outputs are written (the hidden accumulator has been read)
-      const uint32_t kn = k + NC;
-      uint32_t ndec = D, noi = 0;
-      bool ngood = false, nstop = false;
-      if (kn < K && !stop) begin(kn, ndec, noi, ngood, nstop);
-      if (dec < D) {
-        uint32_t o[16];
-        wait_bar(obar, oph);
-        oph ^= 1;
-        wg_bar(wgid);
-        fence_after();
-        tmem_ld16(tO + lanes, o);
-        tmem_wait_ld();
-        fence_before();
-        if (good) {
-          // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
-          float y[CP];
-#pragma unroll
-          for (int cc = 0; cc < CP; ++cc) {
-            float th;
-            asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
-            y[cc] = fmaf(0.5f, th, 0.5f);
-          }
-          float *dst = out + (size_t)oi * C;
-          if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
-            asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]),
-                         "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
-                         : "memory");
-          } else {
-#pragma unroll
-            for (int cc = 0; cc < CP; ++cc)
-              if (cc < (int)C) dst[cc] = y[cc];
-          }
-        }
-      }
-      if (stop || nstop) {  // every warp of this warpgroup read the same flags
-        if (nstop && ndec < D) wait_bar(mbar, ph);  // the issued layer 1 ends before TMEM is released
-        break;
-      }
-      k = kn;
-      dec = ndec;
-      oi = noi;
-      good = ngood;
-    }
-  }
-  fence_before();
-  __syncthreads();
-  if (warp == 0) {
-    fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(TC::alloc)
-                 : "memory");
-  }
-}
-
-template <int H, bool BF16, bool TRI, bool WRAP, int NP, int NC, int SC>
-cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, float *out,
-                        unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
-  using M = TmSmem<H, NC, SC>;
-  const size_t smem = M::total;
-  const bool c8 = W.out_dim <= 8;
-  static bool attr[2] = {false, false};
-  if (!attr[c8]) {
-    // as little shared memory as the kernel needs: the rest of the array is L1
-    const int carve = (int)((smem * 100 + 232448 - 1) / 232448);
-    cudaError_t e;
-    if (c8) {
-      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC>,
-                                 cudaFuncAttributePreferredSharedMemoryCarveout, carve);
-    } else {
-      e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC>,
-                                 cudaFuncAttributePreferredSharedMemoryCarveout, carve);
-    }
-    if (e != cudaSuccess) return e;
-    attr[c8] = true;
-  }
-  const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
-  size_t grid = (size_t)num_sms;
-  if (grid > max_tiles) grid = max_tiles;
-  const int vec_out = ((uintptr_t)out & 31) == 0;  // 32-byte rows need a 32-byte aligned base
-  const unsigned threads = (NP + NC) * 128;
-  // launched as a programmatic dependent of the bucketing: its prologue overlaps
-  // the end of k_scatter
-  cudaError_t e;
-  if (c8)
-    e = launch_pdl(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC>, dim3((unsigned)grid), dim3(threads), smem, st,
-                   A, W, B, out, err, status, vec_out);
-  else
-    e = launch_pdl(k_decode_tm<H, BF16, TRI, WRAP, 16, NP, NC, SC>, dim3((unsigned)grid), dim3(threads), smem, st,
-                   A, W, B, out, err, status, vec_out);
-  if (e != cudaSuccess) return e;
-  return cudaGetLastError();
-}
-
-}  // namespace
 
 // One CTA per decoder: fp32 weights -> the shared-memory image of the tcgen05
 // kernel (bias folded in as column `in` of each layer's B operand).
@@ -691,23 +52,7 @@ cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Bucke
                              float *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches) {
   *launches += 1;
-  const bool tri = A.num_mips > 1, wrap = A.address_mode == 0;
-#define NTC_WS2(H, TRI, WRAP, NP, NC, SC)                                                                  \
-  return bf16 ? launch_tm_t<H, true, TRI, WRAP, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st) \
-              : launch_tm_t<H, false, TRI, WRAP, NP, NC, SC>(A, W, B, n, out, err, status, num_sms, st)
-#define NTC_WS(H, TRI, NP, NC, SC)              \
-  do {                                          \
-    if (wrap) NTC_WS2(H, TRI, true, NP, NC, SC); \
-    NTC_WS2(H, TRI, false, NP, NC, SC);          \
-  } while (0)
-  if (W.hidden == 64) {
-    if (tri) NTC_WS(64, true, 4, 4, 1);
-    NTC_WS(64, false, 4, 4, 1);
-  }
-  if (tri) NTC_WS(128, true, 4, 2, 2);
-  NTC_WS(128, false, 4, 2, 2);
-#undef NTC_WS
-#undef NTC_WS2
+  return dispatch_tm<false>(A, W, B, n, out, err, status, bf16, num_sms, st, nullptr);
 }
 
 }  // namespace ntc

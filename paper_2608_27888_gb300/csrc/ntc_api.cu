@@ -43,10 +43,11 @@ struct ntc_ctx {
   unsigned long long *d_err = nullptr;
   unsigned int *d_status = nullptr;  // nonzero: a decode kernel gave up a bounded wait
   // bucketing scratch (grows on demand, stream-ordered)
-  size_t cap_n = 0, cap_counts = 0;
-  uint32_t *d_counts = nullptr, *d_perm = nullptr, *d_meta = nullptr;
+  size_t cap_n = 0, cap_desc = 0;
+  uint32_t *d_perm = nullptr, *d_meta = nullptr;
   ntc_query *d_sorted = nullptr;
-  uint32_t *d_cursor = nullptr;  // single-pass bucketing: [D+1] cursors + ticket, zero between calls
+  unsigned long long *d_desc = nullptr;  // look-back descriptors of the bucketing
+  uint32_t epoch = 0;                    // the last bucketing call's descriptor epoch
   // staging for ntc_decode_host, and its copy streams and chunk events
   size_t cap_host = 0;
   ntc_query *d_hq = nullptr;
@@ -173,68 +174,60 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_gfma);
   cudaFree(c->d_err);
   cudaFree(c->d_status);
-  cudaFree(c->d_counts);
   cudaFree(c->d_perm);
   cudaFree(c->d_sorted);
   cudaFree(c->d_meta);
-  cudaFree(c->d_cursor);
+  cudaFree(c->d_desc);
   cudaFree(c->d_hq);
   cudaFree(c->d_hout);
 }
 
 size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
 
-// Single-pass bucketing gives every decoder a region of n rows: used when
-// that fits this budget (the stable three-kernel sort needs n rows in all).
-constexpr size_t kSpreadBudgetBytes = 24ull << 30;
-
-bool use_spread(const ntc_ctx *c, size_t n) {
-  const size_t rows = ((size_t)c->D + 1) * n;
-  return rows * (sizeof(ntc_query) + 4) <= kSpreadBudgetBytes && rows < 0xFFFFFF00ull;
-}
-
-// Make sure the bucketing scratch holds n queries (stream-ordered allocation);
-// `rows` entries of perm and sorted (n, or (D+1) * n for the single pass).
-ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st, size_t rows = 0) {
-  if (rows < n) rows = n;
-  const size_t chunks = (n + kBucketChunk - 1) / kBucketChunk;
-  const size_t counts = (size_t)(c->D + 1) * (chunks ? chunks : 1);
+// Make sure the bucketing scratch holds n queries (stream-ordered
+// allocation): perm and sorted records [n], the tile table with the totals and
+// tickets (zeroed once), and the look-back descriptors (zeroed whenever they
+// are allocated, so no stale word can carry a live epoch).
+ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
+  const size_t desc = bucket_desc_words(c->D, n);
   if (!c->d_meta) {
-    const size_t words = meta_words(c->D) + (c->D + 1) + 1;
+    const size_t words = bucket_meta_words(c->D);
     CK(cudaMallocAsync((void **)&c->d_meta, words * 4, st), "scratch allocation");
     CK(cudaMemsetAsync(c->d_meta, 0, words * 4, st), "scratch clear");
   }
-  if (counts > c->cap_counts) {
-    if (c->d_counts) CK(cudaFreeAsync(c->d_counts, st), "scratch free");
-    c->d_counts = nullptr;
-    c->cap_counts = 0;
-    CK(cudaMallocAsync((void **)&c->d_counts, counts * 4, st), "scratch allocation");
-    c->cap_counts = counts;
+  if (desc > c->cap_desc) {
+    if (c->d_desc) CK(cudaFreeAsync(c->d_desc, st), "scratch free");
+    c->d_desc = nullptr;
+    c->cap_desc = 0;
+    CK(cudaMallocAsync((void **)&c->d_desc, desc * 8, st), "scratch allocation");
+    CK(cudaMemsetAsync(c->d_desc, 0, desc * 8, st), "scratch clear");
+    c->cap_desc = desc;
   }
-  if (rows > c->cap_n) {
+  if (n > c->cap_n) {
     if (c->d_perm) CK(cudaFreeAsync(c->d_perm, st), "scratch free");
     if (c->d_sorted) CK(cudaFreeAsync(c->d_sorted, st), "scratch free");
     c->d_perm = nullptr;
     c->d_sorted = nullptr;
     c->cap_n = 0;
-    CK(cudaMallocAsync((void **)&c->d_perm, rows * 4, st), "scratch allocation");
-    CK(cudaMallocAsync((void **)&c->d_sorted, rows * sizeof(ntc_query), st), "scratch allocation");
-    c->cap_n = rows;
-  }
-  if (!c->d_cursor) {
-    CK(cudaMallocAsync((void **)&c->d_cursor, ((size_t)c->D + 2) * 4, st), "scratch allocation");
-    CK(cudaMemsetAsync(c->d_cursor, 0, ((size_t)c->D + 2) * 4, st), "scratch clear");
+    CK(cudaMallocAsync((void **)&c->d_perm, n * 4, st), "scratch allocation");
+    CK(cudaMallocAsync((void **)&c->d_sorted, n * sizeof(ntc_query), st), "scratch allocation");
+    c->cap_n = n;
   }
   return NTC_OK;
 }
 
-Scratch scratch_of(const ntc_ctx *c) {
-  Scratch s;
-  s.counts = c->d_counts;
+// The scratch of the next bucketing call, with a fresh descriptor epoch.
+ntc_status next_scratch(ntc_ctx *c, cudaStream_t st, Scratch &s) {
+  if (++c->epoch >= kBucketEpochs) {  // wrapped: no old word may match a reused epoch
+    CK(cudaMemsetAsync(c->d_desc, 0, c->cap_desc * 8, st), "scratch clear");
+    c->epoch = 1;
+  }
   s.perm = c->d_perm;
   s.sorted = c->d_sorted;
   s.meta = c->d_meta;
-  return s;
+  s.desc = c->d_desc;
+  s.epoch = c->epoch;
+  return NTC_OK;
 }
 
 ntc_status check_queries(const ntc_ctx *ctx, const void *q, size_t n) {
@@ -444,8 +437,32 @@ ntc_status ntc_destroy(ntc_ctx *c) {
   return NTC_OK;
 }
 
+namespace {
+ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream, ntc_mode mode,
+                       ntc_debug_row *rows);
+}
+
 ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream,
                       ntc_mode mode) {
+  return decode_impl(c, q, n, out, stream, mode, nullptr);
+}
+
+ntc_status ntc_debug_decode_rows(ntc_ctx *c, const ntc_query *q, size_t n, float *out, ntc_debug_row *rows,
+                                 void *stream) {
+  if (!c) return fail(NTC_ERR_INVALID_ARG, "null context");
+  if (c->general || c->prec == NTC_PREC_FP32)
+    return fail(NTC_ERR_UNSUPPORTED, "rows are recorded by the standard-shape tensor-core decode only");
+  if (n && !rows) return fail(NTC_ERR_INVALID_ARG, "null rows pointer");
+  return decode_impl(c, q, n, out, stream, NTC_MODE_BUCKETED, rows);
+}
+
+}  // extern "C"
+
+namespace {
+// ntc_decode; with rows != nullptr the tensor-core kernel is the debug
+// instantiation that also records every row it builds.
+ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream, ntc_mode mode,
+                       ntc_debug_row *rows) {
   ntc_status s = check_queries(c, q, n);
   if (s != NTC_OK) return s;
   if (n && !out) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
@@ -472,14 +489,7 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   // divergence to remove, so the tensor-core decode takes the queries in their
   // own order and nothing is sorted
   const bool shared = mode == NTC_MODE_BUCKETED && !fp32 && !c->general && c->D == 1;
-  // the tensor-core decodes need no stable order: single-pass bucketing, when
-  // its per-decoder regions fit the budget and can be allocated
-  bool spread = mode == NTC_MODE_BUCKETED && !fp32 && !shared && use_spread(c, n);
-  if (spread && ensure_scratch(c, n, st, ((size_t)c->D + 1) * n) != NTC_OK) {
-    cudaGetLastError();  // an allocation failure is not sticky: fall back to the stable sort
-    spread = false;
-  }
-  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st, n);
+  s = unsorted || shared ? NTC_OK : ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
   if (c->timing) CK(cudaEventRecord(c->ev[0], st), "event record");
   if (unsorted) {
@@ -505,11 +515,9 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     B.meta = nullptr;
     B.identity_n = (uint32_t)n;
   } else {
-    Scratch sc = scratch_of(c);
-    if (spread) {
-      sc.cursor = c->d_cursor;
-      sc.cap = (uint32_t)n;
-    }
+    Scratch sc;
+    s = next_scratch(c, st, sc);
+    if (s != NTC_OK) return s;
     e = launch_bucket(A, q, n, sc, st, &launches, c->d_status);
     if (e != cudaSuccess) {
       c->launches += launches;
@@ -518,7 +526,6 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     B.sorted = c->d_sorted;
     B.perm = c->d_perm;
     B.meta = c->d_meta;
-    B.spread_cap = spread ? (uint32_t)n : 0u;
   }
   if (c->timing) CK(cudaEventRecord(c->ev[1], st), "event record");
   if (c->general && fp32)
@@ -529,6 +536,8 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
     e = launch_decode_fp32(A, W, B, n, out, c->d_err, c->num_sms, st, &launches);
   else if (mode == NTC_MODE_BUCKETED_MMA)
     e = launch_decode_mma(A, W, B, n, out, c->d_err, bf16, c->num_sms, st, &launches);
+  else if (rows)
+    e = launch_decode_tc_debug(A, W, B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches, rows);
   else
     e = launch_decode_tc(A, W, B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
   c->launches += launches;
@@ -539,6 +548,9 @@ ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void
   }
   return NTC_OK;
 }
+}  // namespace
+
+extern "C" {
 
 ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hout, void *stream,
                            ntc_mode mode) {
@@ -653,7 +665,10 @@ ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *
   }
   s = ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
-  cudaError_t e = launch_bucket(assets_of(c), q, n, scratch_of(c), st, &launches, c->d_status);
+  Scratch sc;
+  s = next_scratch(c, st, sc);
+  if (s != NTC_OK) return s;
+  cudaError_t e = launch_bucket(assets_of(c), q, n, sc, st, &launches, c->d_status);
   if (e == cudaSuccess) e = cudaMemcpyAsync(perm, c->d_perm, n * 4, cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && (counts || tiles || num_tiles))
     e = launch_tiles_export(c->d_meta, c->D, tiles, num_tiles, counts, ntc_max_tiles(c, n), st, &launches);

@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <climits>
 #include <type_traits>
 
 #include "../../include/ntc.h"
@@ -129,9 +131,6 @@ struct Buckets {
   const uint32_t *perm;     // original index of each sorted query
   const uint32_t *meta;     // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
   uint32_t identity_n = 0;
-  // spread_cap != 0: single-pass bucketing; decoder d's sorted rows are at
-  // d * spread_cap .. and meta's seg[d] holds the decoder's count
-  uint32_t spread_cap = 0;
 };
 inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2); }
 
@@ -440,12 +439,10 @@ __device__ __forceinline__ void tile_info(const uint32_t *meta, uint32_t D, uint
 // The tiles of one role in increasing order: the decoder index only moves
 // forward, so a lookup is a few compares instead of a binary search.  With
 // ident_n != 0 (one decoder, nothing sorted) tile t is queries 128t .. of the
-// caller's array; with cap != 0 (single-pass bucketing) decoder d's rows start
-// at d * cap and seg[d] is their count.
+// caller's array.
 struct TileWalk {
   uint32_t d = 0;
   uint32_t ident_n = 0;
-  uint32_t cap = 0;
   __device__ __forceinline__ void at(const uint32_t *seg, const uint32_t *tst, uint32_t D, uint32_t t,
                                      uint32_t &dec, uint32_t &start, uint32_t &len) {
     if (ident_n) {
@@ -456,33 +453,31 @@ struct TileWalk {
     }
     while (d < D && tst[d + 1] <= t) ++d;
     dec = d;
-    const uint32_t off = (t - tst[d]) * kTile;
-    if (cap) {
-      start = d * cap + off;
-      len = min((uint32_t)kTile, seg[d] - off);
-    } else {
-      start = seg[d] + off;
-      len = min((uint32_t)kTile, seg[d + 1] - start);
-    }
+    start = seg[d] + (t - tst[d]) * kTile;
+    len = min((uint32_t)kTile, seg[d + 1] - start);
   }
 };
 
 // ---------------------------------------------------------------- launchers
 
+// Device scratch of one bucketing call.
 struct Scratch {
-  uint32_t *counts;   // [(D+1) * chunks]
-  uint32_t *perm;     // [n], or [(D+1) * cap] with cursor
-  ntc_query *sorted;  // [n], or [(D+1) * cap] with cursor
-  uint32_t *meta;     // meta_words(D)
-  // single-pass bucketing (see k_scatter<true>): decoder d's runs go to
-  // [d * cap, d * cap + cap); cursor [D+1] + ticket [1], zero between calls
-  uint32_t *cursor = nullptr;
-  uint32_t cap = 0;
+  uint32_t *perm;             // [n]
+  ntc_query *sorted;          // [n]
+  uint32_t *meta;             // bucket_meta_words(D): the tile table, then the
+                              // totals [D+1] and two tickets, zero between calls
+  unsigned long long *desc;   // [bucket_desc_words(D, n)] look-back descriptors
+  uint32_t epoch;             // 1 .. kBucketEpochs - 1, different from the
+                              // previous call's on the same descriptors
 };
+constexpr uint32_t kBucketEpochs = 1u << 30;  // descriptors are cleared when the epoch wraps
 
 constexpr int kBucketThreads = 256;
 constexpr int kBucketItems = 8;  // queries per thread
 constexpr int kBucketChunk = kBucketThreads * kBucketItems;
+size_t bucket_chunks(size_t n);
+size_t bucket_desc_words(uint32_t D, size_t n);
+size_t bucket_meta_words(uint32_t D);
 
 cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
                           cudaStream_t st, int *launches, unsigned int *status);
@@ -516,6 +511,9 @@ cudaError_t launch_pack_gen(const float *w32, uint32_t D, const GenWeights &G, n
 cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
                              float *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches);
+cudaError_t launch_decode_tc_debug(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
+                                   float *out, unsigned long long *err, unsigned int *status, bool bf16,
+                                   int num_sms, cudaStream_t st, int *launches, ntc_debug_row *rows);
 cudaError_t launch_pack_tc(const float *w32, uint32_t D, uint32_t H, uint32_t C, bool bf16,
                            uint8_t *tc, size_t tc_stride, cudaStream_t st);
 cudaError_t launch_debug_taps(const Assets &A, const ntc_query *q, size_t n, unsigned long long *idx,
@@ -544,6 +542,47 @@ inline int resident_ctas(Kernel kernel, int threads, size_t dyn_smem) {
   occ = occ < cta_sm ? occ : cta_sm;
   return occ < 1 ? 1 : occ;
 }
+
+// Per-device one-time set-up.  Kernel attributes (the dynamic shared-memory
+// limit, the carveout) belong to a device, so every device a process uses
+// needs its own; once() runs f on the current device the first time that
+// device asks and remembers success, value() caches an int result (an
+// occupancy) per device.  Threads racing on a first use may both run f, which
+// must therefore be idempotent.
+class PerDevice {
+ public:
+  PerDevice() {
+    for (auto &v : val_) v.store(INT_MIN, std::memory_order_relaxed);
+  }
+  template <typename F>
+  cudaError_t once(F f) {
+    std::atomic<int> *slot = slot_of();
+    if (slot && slot->load(std::memory_order_acquire) == 0) return cudaSuccess;
+    const cudaError_t e = f();
+    if (e == cudaSuccess && slot) slot->store(0, std::memory_order_release);
+    return e;
+  }
+  template <typename F>
+  int value(F f) {
+    std::atomic<int> *slot = slot_of();
+    if (slot) {
+      const int v = slot->load(std::memory_order_acquire);
+      if (v != INT_MIN) return v;
+    }
+    const int v = f();
+    if (slot) slot->store(v, std::memory_order_release);
+    return v;
+  }
+
+ private:
+  static constexpr int kMaxDevices = 64;
+  std::atomic<int> val_[kMaxDevices];
+  std::atomic<int> *slot_of() {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    return &val_[dev];
+  }
+};
 
 // Launch with programmatic stream serialisation (see pdl_wait).
 template <typename... KArgs, typename... Args>

@@ -83,7 +83,7 @@ def _load():
         "ntc_launch_count": ([P], ctypes.c_uint64),
         "ntc_set_stage_timing": ([P, I], I),
         "ntc_stage_times": ([P, P], I),
-        "ntc_bucket_static": ([P, ctypes.c_uint32, ctypes.c_uint32, P, S, P, P, P], I),
+        "ntc_bucket_static": ([P, ctypes.c_uint32, ctypes.c_uint32, P, S, P, P, P, P], I),
         "ntc_kmeans_map": ([P, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, P, ctypes.c_uint32, P, P, P], I),
         "ntc_last_error": ([], ctypes.c_char_p),
         "ntc_status_string": ([I], ctypes.c_char_p),
@@ -167,10 +167,11 @@ def ntc_stage_times(ctx):
     return float(t[0]), float(t[1])
 
 
-def ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm, d_sorted, stream):
+def ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm, d_sorted, d_status,
+                      stream):
     """Allocation-free bucketing (no context): see include/ntc.h."""
     _check(_lib.ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm,
-                                  d_sorted, stream))
+                                  d_sorted, d_status, stream))
 
 
 def ntc_kmeans_map(h_features, n, dim, m, h_init, max_iters, h_map, h_centroids, iters_run):

@@ -407,11 +407,11 @@ def test_bucketing_with_the_most_decoders():
 
 
 @pytest.mark.parametrize("pattern", ["random", "same", "bad", "sparse"])
-def test_single_pass_bucketing_decodes_every_row(pattern):
-    """The tensor-core decode buckets in one unstable pass (per-decoder regions
-    reserved with atomics).  Every row of the output must be written exactly as
-    the oracle decodes it, over chunk boundaries and ragged tails, and the
-    reservations must be cleared for the next call (sizes vary call to call)."""
+def test_bucketed_decode_writes_every_row(pattern):
+    """The tensor-core decode sorts with the look-back counting sort (chunks in
+    ticket order, totals and tickets cleared by the last CTA).  Every row of
+    the output must be written exactly as the oracle decodes it, over chunk
+    boundaries and ragged tails, on consecutive calls of varying sizes."""
     S, D = 40, 13
     rng = np.random.default_rng(7)
     m = rng.integers(0, D, S).astype(np.uint32)
@@ -460,3 +460,32 @@ def test_a_wait_that_gives_up_is_reported_and_the_context_recovers():
     got = dec.decode(dq(w.queries)).cpu().numpy()
     ref, _ = oracle_out("uniform-4m")
     check_tc(got, ref, "after a wait gave up")
+
+
+@pytest.mark.parametrize("hidden,out_dim,mips", [(64, 8, 1), (128, 9, 2)])
+def test_every_tile_switches_decoder(hidden, out_dim, mips):
+    """The most decoder changes the tensor-core decode can meet: 4095 decoders
+    of exactly 8 tiles (1024 queries) each, so the next tile of every consumer
+    (4 x 152 tiles later at H = 64, 2 x 152 at H = 128) belongs to another
+    decoder and the weight image is reloaded before every tile.  The reload must
+    wait for the previous tile's output layer, which still reads W3 of the
+    image (Sec. 3.3: every row is decoded by its own decoder D_c(i)).  Every row
+    is compared with the oracle."""
+    D, per = 4095, 1024
+    seed = W.BASE_SEED + 900 + hidden
+    a = W.make_assets(seed, D, 16, mips, D, W.map_identity(D), hidden=hidden, out_dim=out_dim)
+    n = D * per
+    rng = np.random.default_rng(seed)
+    q = np.zeros(n, dtype=W.QUERY_DTYPE)
+    q["set_id"] = rng.permutation(np.repeat(np.arange(D, dtype=np.uint32), per))
+    q["u"] = rng.random(n, dtype=np.float32)
+    q["v"] = rng.random(n, dtype=np.float32)
+    q["lod"] = rng.random(n, dtype=np.float32) if mips > 1 else 0.0
+    ref, _ = oracle.decode(a, q)
+    dec = ntc().Decoder(a, "fp16")
+    for _ in range(2):
+        got = dec.decode(dq(q)).cpu().numpy()
+        check_tc(got, ref, f"H={hidden} every tile a new decoder")
+    assert dec.error_count() == 0
+    dec.close()
+    torch.cuda.empty_cache()
