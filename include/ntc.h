@@ -29,12 +29,12 @@
  *
  * Memory: the context owns device copies of latents, weights and map.  Query
  * and output buffers of ntc_decode are DEVICE pointers owned by the caller.
- * Scratch (the permutation and the queries in bucket order, 20 bytes per
- * query, the tile table, and 8 bytes per decoder and 2048 queries of
- * look-back records) is owned by the context and grows on demand with
- * cudaMallocAsync on the call's stream.  Every bucketed decode sorts with the
- * same stable counting sort that ntc_debug_bucket exports.  One context must
- * not run two decodes concurrently (on different streams or threads).
+ * Scratch (the permutation and a decoder id per query, 5 or 6 bytes per
+ * query, 4 bytes per decoder and 2048 queries of chunk counts, and the tile
+ * table) is owned by the context and grows on demand with cudaMallocAsync on
+ * the call's stream.  Every bucketed decode sorts with the same stable
+ * counting sort that ntc_debug_bucket exports.  One context must not run two
+ * decodes concurrently (on different streams or threads).
  *
  * Errors: host-detectable problems return a status and enqueue nothing; the
  * message is available from ntc_last_error().  A query whose set id is out of
@@ -258,8 +258,9 @@ NTC_API size_t ntc_max_tiles(const ntc_ctx *ctx, size_t n);
 /* Number of bad queries decoded since creation or the last reset.  Synchronises
  * the device.  Returns NTC_ERR_CUDA (and still writes *count) when a kernel
  * gave up one of its bounded waits since then (every mbarrier wait of the
- * tcgen05 kernels and of the bucketing ends after 200 ms): that call's
- * results are invalid, the context stays usable.  The reset clears both. */
+ * tcgen05 kernels ends after 200 ms; the bucketing waits on nothing): that
+ * call's results are invalid, the context stays usable.  The reset clears
+ * both. */
 NTC_API ntc_status ntc_get_error_count(ntc_ctx *ctx, uint64_t *count);
 NTC_API ntc_status ntc_reset_error_count(ntc_ctx *ctx);
 
@@ -294,13 +295,10 @@ NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
  * num_decoders) and d_sorted[n] the query records in that order.  h_set_to_decoder
  * is a HOST array of num_sets entries (each < num_decoders); d_queries,
  * d_perm and d_sorted are caller-owned device buffers (the query buffers
- * 16-byte aligned).  d_status (may be NULL) is a caller-owned device word: the
- * kernels OR a nonzero value into it when one of their bounded waits (200 ms)
- * gave up, and the result of that call is then invalid; the library never
- * clears it, so zero it before the calls it should watch and read it after
- * they have completed.  Its scratch is one file-scope device array of
- * 2,409,472 bytes that every GPU loading the library holds until the process
- * exits, so:
+ * 16-byte aligned).  Its kernels wait on nothing (no barrier, flag or
+ * timeout), so a call that was enqueued completes.  Its scratch is one
+ * file-scope device array of 1,360,896 bytes that every GPU loading the
+ * library holds until the process exits, so:
  *   - num_sets <= 65536, num_decoders <= 4095 and
  *     (num_decoders + 1) * ceil(n / 2048) <= 262144 (larger calls return
  *     NTC_ERR_UNSUPPORTED and enqueue nothing);
@@ -315,8 +313,7 @@ NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
  * cudaFree or allocating library routine. */
 NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder, uint32_t num_sets,
                                      uint32_t num_decoders, const ntc_query *d_queries, size_t n,
-                                     uint32_t *d_perm, ntc_query *d_sorted, uint32_t *d_status,
-                                     void *cuda_stream);
+                                     uint32_t *d_perm, ntc_query *d_sorted, void *cuda_stream);
 
 /* ---------------------------------------------------------- map sources
  *

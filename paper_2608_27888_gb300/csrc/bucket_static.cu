@@ -7,8 +7,8 @@
 // or fail half-way through it.  ntc_bucket_static gives them the stable
 // counting sort by decoder id (the same kernels as ntc_decode and
 // ntc_debug_bucket) without a context and without allocating: a copy of the
-// set->decoder map, the tile table with the totals and tickets, and the
-// look-back descriptors live in one file-scope device array of fixed size that
+// set->decoder map, the tile table with the totals and the ticket, and the
+// per-chunk counts live in one file-scope device array of fixed size that
 // every GPU loading this library keeps until the process exits.
 #include <mutex>
 
@@ -23,9 +23,9 @@ using namespace ntc;
 namespace {
 
 constexpr size_t kMapWords = 65536;    // set->decoder map copy
-constexpr size_t kMetaWords = 12544;   // tile table, totals, tickets (<= 12293 for D <= 4095), status
-constexpr size_t kDescs = 262144;      // (D+1) * ceil(n / 2048) look-back descriptors of 8 bytes
-constexpr size_t kStaticWords = kMapWords + kMetaWords + 2 * kDescs;  // 2,409,472 bytes
+constexpr size_t kMetaWords = 12544;   // tile table, totals, ticket (<= 12292 words for D <= 4095)
+constexpr size_t kCountWords = 262144; // (D+1) * ceil(n / 2048) per-chunk counts
+constexpr size_t kStaticWords = kMapWords + kMetaWords + kCountWords;  // 1,360,896 bytes
 
 // The scratch.  In host code this name is only a host-side stand-in: kernels
 // receive the device address looked up with cudaGetSymbolAddress below.
@@ -34,7 +34,6 @@ static __device__ __align__(256) uint32_t g_bucket_scratch[kStaticWords];
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 uint32_t *g_addr[kMaxDevices] = {};
-uint32_t g_epoch[kMaxDevices] = {};  // the last call's descriptor epoch on each device
 
 ntc_status failed(ntc_status s, const char *m) {
   set_last_error(m);
@@ -46,7 +45,7 @@ ntc_status failed(ntc_status s, const char *m) {
 extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder, uint32_t num_sets,
                                                 uint32_t num_decoders, const ntc_query *d_queries,
                                                 size_t n, uint32_t *d_perm, ntc_query *d_sorted,
-                                                uint32_t *d_status, void *cuda_stream) {
+                                                void *cuda_stream) {
   if (!h_set_to_decoder) return failed(NTC_ERR_INVALID_ARG, "null set_to_decoder");
   if (num_sets < 1 || num_sets > kMapWords)
     return failed(NTC_ERR_INVALID_ARG, "num_sets must be in 1..65536");
@@ -57,23 +56,18 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
   if (!d_queries || !d_perm || !d_sorted) return failed(NTC_ERR_INVALID_ARG, "null device pointer");
   if (((uintptr_t)d_queries & 15) || ((uintptr_t)d_sorted & 15))
     return failed(NTC_ERR_INVALID_ARG, "query buffers must be 16-byte aligned");
-  if (((uintptr_t)d_status & 3)) return failed(NTC_ERR_INVALID_ARG, "status word is not 4-byte aligned");
-  if (bucket_desc_words(num_decoders, n) > kDescs)
+  if (bucket_count_words(num_decoders, n) > kCountWords)
     return failed(NTC_ERR_UNSUPPORTED,
-                  "(num_decoders + 1) * ceil(n / 2048) exceeds the static scratch (262144 descriptors)");
+                  "(num_decoders + 1) * ceil(n / 2048) exceeds the static scratch (262144 counts)");
   for (uint32_t s = 0; s < num_sets; ++s)
     if (h_set_to_decoder[s] >= num_decoders)
       return failed(NTC_ERR_INVALID_ARG, "set_to_decoder entry is not a decoder");
 
-  cudaStream_t st = (cudaStream_t)cuda_stream;
-  // set-up, once per device, with that device current: the array's device
-  // address, and its descriptors cleared (no stale word may carry an epoch)
+  // set-up, once per device, with that device current
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
     return failed(NTC_ERR_CUDA, "no usable current CUDA device");
   uint32_t *base = nullptr;
-  uint32_t epoch = 0;
-  bool clear_desc = false;
   {
     std::lock_guard<std::mutex> lk(g_mu);
     if (!g_addr[dev]) {
@@ -81,25 +75,17 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
       cudaError_t e = cudaGetSymbolAddress(&p, g_bucket_scratch);
       if (e != cudaSuccess) return failed(NTC_ERR_CUDA, cudaGetErrorString(e));
       g_addr[dev] = static_cast<uint32_t *>(p);
-      clear_desc = true;
     }
     base = g_addr[dev];
-    if (++g_epoch[dev] >= kBucketEpochs) {  // wrapped: clear before an epoch repeats
-      g_epoch[dev] = 1;
-      clear_desc = true;
-    }
-    epoch = g_epoch[dev];
   }
+  cudaStream_t st = (cudaStream_t)cuda_stream;
   uint32_t *map = base;
   uint32_t *meta = base + kMapWords;
-  unsigned long long *desc = reinterpret_cast<unsigned long long *>(meta + kMetaWords);
-  unsigned int *status = d_status ? reinterpret_cast<unsigned int *>(d_status)
-                                  : reinterpret_cast<unsigned int *>(meta + kMetaWords - 1);
-  // the map copy, and the tile table, totals and tickets cleared (the totals
-  // and tickets must start at 0)
+  uint32_t *counts = meta + kMetaWords;
+  // the map copy, and the tile table, totals and ticket cleared (the ticket
+  // must start at 0)
   cudaError_t e = cudaMemcpyAsync(map, h_set_to_decoder, (size_t)num_sets * 4, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(meta, 0, bucket_meta_words(num_decoders) * 4, st);
-  if (e == cudaSuccess && clear_desc) e = cudaMemsetAsync(desc, 0, kDescs * 8, st);
   if (e != cudaSuccess) return failed(NTC_ERR_CUDA, cudaGetErrorString(e));
   Assets A{};
   A.map = map;
@@ -107,12 +93,11 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
   A.num_decoders = num_decoders;
   Scratch s;
   s.perm = d_perm;
-  s.sorted = d_sorted;
   s.meta = meta;
-  s.desc = desc;
-  s.epoch = epoch;
+  s.counts = counts;
+  s.sorted = d_sorted;
   int launches = 0;
-  e = launch_bucket(A, d_queries, n, s, st, &launches, status);
+  e = launch_bucket(A, d_queries, n, s, st, &launches);
   if (e != cudaSuccess) return failed(NTC_ERR_CUDA, cudaGetErrorString(e));
   return NTC_OK;
 }

@@ -168,28 +168,28 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
   if (wg == 0) {
     // ------------------------------------------------------------- producer
     TileWalk walk;
-    // tile j's query record and output row; the next tile's are loaded while
-    // tile j is gathered
-    auto load_row = [&](uint32_t jj, uint32_t &d_, uint32_t &len_, ntc_query &q_, uint32_t &oi_) {
-      uint32_t st_;
+    // this thread's row of tile jj: its output row (kNoRow past the tile's
+    // end) and query record; the bad bucket (set id out of range) is rejected
+    // by query_bad().  The next tile's are loaded while tile j is gathered.
+    constexpr uint32_t kNoRow = 0xFFFFFFFFu;  // never a row: n <= 2^32 - 256
+    auto fetch_row = [&](uint32_t jj, uint32_t &oi_, ntc_query &q_) {
+      oi_ = kNoRow;
+      if (jj >= K) return;
+      uint32_t d_, st_, len_;
       walk.at(seg, tst, D, t0 + jj, d_, st_, len_);
-      oi_ = 0;
-      if (row < len_) {
-        q_ = load_query(B.sorted + st_ + row);
-        oi_ = __ldg(B.perm + st_ + row);
-      }
+      if (row < len_) bucket_row(B, st_ + row, oi_, q_);
     };
-    uint32_t dec = D, len = 0, oi = 0;
+    uint32_t oi;
     ntc_query q;
-    if (K) load_row(0, dec, len, q, oi);
+    fetch_row(0, oi, q);
     for (uint32_t j = 0; j < K; ++j) {
       if (abort_flag) break;
       const uint32_t s = j % kGenStages, use = j / kGenStages;
-      uint32_t ndec = D, nlen = 0, noi = 0;
+      uint32_t noi;
       ntc_query nq;
-      if (j + 1 < K) load_row(j + 1, ndec, nlen, nq, noi);
-      const bool valid = row < len;
-      const bool good = valid && dec < D && !query_bad(A, q);
+      fetch_row(j + 1, noi, nq);
+      const bool valid = oi != kNoRow;
+      const bool good = valid && !query_bad(A, q);
       const bool bad = valid && !good;
       count_bad_warp(bad, err);
       if (bad)
@@ -241,23 +241,21 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
         abort_flag = 1;
       }
       fence_after();
-      if (dec < D) {
+      // (a tile of the bad bucket is stored too: its rows are zeros and the
+      // consumer multiplies nothing)
 #pragma unroll
-        for (int kc = 0; kc < NP / 16; ++kc) {
-          if ((uint32_t)kc * 16 >= K1) break;
-          uint32_t p[8];
+      for (int kc = 0; kc < NP / 16; ++kc) {
+        if ((uint32_t)kc * 16 >= K1) break;
+        uint32_t p[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) p[i] = pk[8 * kc + i];
-          tmem_st8(tA1 + s * (K1 / 2) + lanes + 8 * kc, p);
-        }
-        tmem_wait_st();
+        for (int i = 0; i < 8; ++i) p[i] = pk[8 * kc + i];
+        tmem_st8(tA1 + s * (K1 / 2) + lanes + 8 * kc, p);
       }
+      tmem_wait_st();
       oidx[(s * 2 + (use & 1u)) * 128 + row] = good ? oi : 0xFFFFFFFFu;
       fence_before();
       __syncwarp();
       if ((row & 31) == 0) mbar_arrive(full_bar(s));
-      dec = ndec;
-      len = nlen;
       q = nq;
       oi = noi;
     }
@@ -452,7 +450,7 @@ __device__ __forceinline__ float act_f(float x, uint32_t act, float slope) {
   return x > 0.0f ? x : (act == 1 ? slope * x : 0.0f);
 }
 
-// Per-lane decode of a general shape; row i is sorted[i] written to out[perm[i]]
+// Per-lane decode of a general shape; row i is qs[i] written to out[perm[i]]
 // (or query i itself when perm is null).
 template <typename T>
 __global__ void __launch_bounds__(128) k_decode_gen_fma(Assets A, GenWeights G, const ntc_query *qs,

@@ -308,8 +308,7 @@ __global__ void __launch_bounds__(kTile) k_decode_mma(Assets A, WeightImages W, 
     bool bad = false;
     uint32_t oi = 0;
     if (valid) {
-      q = load_query(B.sorted + start + r);
-      oi = __ldg(B.perm + start + r);
+      bucket_row(B, start + r, oi, q);
       bad = dec == D || query_bad(A, q);
     }
     orig[r] = oi;

@@ -46,8 +46,7 @@ __global__ void __launch_bounds__(kTile) k_decode_fp32(Assets A, WeightImages W,
     uint32_t oi = 0;
     bool bad = false;
     if (valid) {
-      q = load_query(B.sorted + start + r);
-      oi = __ldg(B.perm + start + r);
+      bucket_row(B, start + r, oi, q);
       bad = dec == D || query_bad(A, q);
     }
     count_bad(valid && bad, err);

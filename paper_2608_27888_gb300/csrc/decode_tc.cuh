@@ -381,36 +381,33 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t pc = role % NC, pq = role / NC;  // serves consumer pc, tiles j = pq mod R
     auto tile_of = [&](uint32_t j) { return pc + NC * j; };
     uint32_t j = pq;
-    uint32_t dec = D, start = 0, len = 0, oi = 0;
-    ntc_query q;
     TileWalk walk;
     walk.ident_n = B.identity_n;
-    if (tile_of(j) < K) {
-      walk.at(seg, tst, D, blockIdx.x + tile_of(j) * grid, dec, start, len);
-      if ((uint32_t)row < len) {
-        q = load_query(B.sorted + start + row);
-        oi = B.identity_n ? start + row : __ldg(B.perm + start + row);
-      }
-    }
+    // this thread's row of the producer's tile jj: its output row (kNoRow
+    // past the tile's end) and query record.  A row of the bad bucket (set id
+    // out of range) needs no flag of its own: query_bad() rejects it.
+    constexpr uint32_t kNoRow = 0xFFFFFFFFu;  // never a row: n <= 2^32 - 256
+    auto fetch_row = [&](uint32_t jj, uint32_t &oi_, ntc_query &q_) {
+      oi_ = kNoRow;
+      if (tile_of(jj) >= K) return;
+      uint32_t d_, st_, len_;
+      walk.at(seg, tst, D, blockIdx.x + tile_of(jj) * grid, d_, st_, len_);
+      if ((uint32_t)row < len_) bucket_row(B, st_ + row, oi_, q_);
+    };
+    uint32_t oi;
+    ntc_query q;
+    fetch_row(j, oi, q);
     for (; tile_of(j) < K; j += R) {
       if (*abort_flag) break;
       // the next tile's query record and output row go in flight early: before
       // the taps, or (TRI, where registers are scarcer) once the first mip's
       // taps are consumed
-      uint32_t ndec = D, nstart = 0, nlen = 0, noi = 0;
+      uint32_t noi;
       ntc_query nq;
-      auto prefetch = [&]() {
-        if (tile_of(j + R) < K) {
-          walk.at(seg, tst, D, blockIdx.x + tile_of(j + R) * grid, ndec, nstart, nlen);
-          if ((uint32_t)row < nlen) {
-            nq = load_query(B.sorted + nstart + row);
-            noi = B.identity_n ? nstart + row : __ldg(B.perm + nstart + row);
-          }
-        }
-      };
+      auto prefetch = [&]() { fetch_row(j + R, noi, nq); };
       if (!TRI) prefetch();
-      const bool valid = (uint32_t)row < len;
-      const bool good = valid && dec < D && !query_bad(A, q);
+      const bool valid = oi != kNoRow;
+      const bool good = valid && !query_bad(A, q);
       Taps taps;
       MipPick mp;
       TapIdx ti[kLevels];
@@ -479,8 +476,6 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(full_bar(s));
-      dec = ndec;
-      len = nlen;
       q = nq;
       oi = noi;
     }

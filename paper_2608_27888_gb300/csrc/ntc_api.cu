@@ -43,11 +43,9 @@ struct ntc_ctx {
   unsigned long long *d_err = nullptr;
   unsigned int *d_status = nullptr;  // nonzero: a decode kernel gave up a bounded wait
   // bucketing scratch (grows on demand, stream-ordered)
-  size_t cap_n = 0, cap_desc = 0;
-  uint32_t *d_perm = nullptr, *d_meta = nullptr;
+  size_t cap_n = 0, cap_counts = 0;
+  uint32_t *d_perm = nullptr, *d_meta = nullptr, *d_counts = nullptr;
   ntc_query *d_sorted = nullptr;
-  unsigned long long *d_desc = nullptr;  // look-back descriptors of the bucketing
-  uint32_t epoch = 0;                    // the last bucketing call's descriptor epoch
   // staging for ntc_decode_host, and its copy streams and chunk events
   size_t cap_host = 0;
   ntc_query *d_hq = nullptr;
@@ -175,9 +173,9 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_err);
   cudaFree(c->d_status);
   cudaFree(c->d_perm);
-  cudaFree(c->d_sorted);
   cudaFree(c->d_meta);
-  cudaFree(c->d_desc);
+  cudaFree(c->d_counts);
+  cudaFree(c->d_sorted);
   cudaFree(c->d_hq);
   cudaFree(c->d_hout);
 }
@@ -185,23 +183,22 @@ void release(ntc_ctx *c) {
 size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 // Make sure the bucketing scratch holds n queries (stream-ordered
-// allocation): perm and sorted records [n], the tile table with the totals and
-// tickets (zeroed once), and the look-back descriptors (zeroed whenever they
-// are allocated, so no stale word can carry a live epoch).
+// allocation): perm and the sorted query records [n], the per-chunk counts,
+// and the tile table with the totals and the ticket (zeroed once; the
+// bucketing leaves the ticket at zero).
 ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
-  const size_t desc = bucket_desc_words(c->D, n);
+  const size_t counts = bucket_count_words(c->D, n);
   if (!c->d_meta) {
     const size_t words = bucket_meta_words(c->D);
     CK(cudaMallocAsync((void **)&c->d_meta, words * 4, st), "scratch allocation");
     CK(cudaMemsetAsync(c->d_meta, 0, words * 4, st), "scratch clear");
   }
-  if (desc > c->cap_desc) {
-    if (c->d_desc) CK(cudaFreeAsync(c->d_desc, st), "scratch free");
-    c->d_desc = nullptr;
-    c->cap_desc = 0;
-    CK(cudaMallocAsync((void **)&c->d_desc, desc * 8, st), "scratch allocation");
-    CK(cudaMemsetAsync(c->d_desc, 0, desc * 8, st), "scratch clear");
-    c->cap_desc = desc;
+  if (counts > c->cap_counts) {
+    if (c->d_counts) CK(cudaFreeAsync(c->d_counts, st), "scratch free");
+    c->d_counts = nullptr;
+    c->cap_counts = 0;
+    CK(cudaMallocAsync((void **)&c->d_counts, counts * 4, st), "scratch allocation");
+    c->cap_counts = counts;
   }
   if (n > c->cap_n) {
     if (c->d_perm) CK(cudaFreeAsync(c->d_perm, st), "scratch free");
@@ -216,18 +213,13 @@ ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
   return NTC_OK;
 }
 
-// The scratch of the next bucketing call, with a fresh descriptor epoch.
-ntc_status next_scratch(ntc_ctx *c, cudaStream_t st, Scratch &s) {
-  if (++c->epoch >= kBucketEpochs) {  // wrapped: no old word may match a reused epoch
-    CK(cudaMemsetAsync(c->d_desc, 0, c->cap_desc * 8, st), "scratch clear");
-    c->epoch = 1;
-  }
+Scratch scratch_of(const ntc_ctx *c) {
+  Scratch s;
   s.perm = c->d_perm;
-  s.sorted = c->d_sorted;
   s.meta = c->d_meta;
-  s.desc = c->d_desc;
-  s.epoch = c->epoch;
-  return NTC_OK;
+  s.counts = c->d_counts;
+  s.sorted = c->d_sorted;
+  return s;
 }
 
 ntc_status check_queries(const ntc_ctx *ctx, const void *q, size_t n) {
@@ -510,19 +502,17 @@ ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, voi
   }
   Buckets B;
   if (shared) {
-    B.sorted = q;
+    B.queries = q;
     B.perm = nullptr;
     B.meta = nullptr;
     B.identity_n = (uint32_t)n;
   } else {
-    Scratch sc;
-    s = next_scratch(c, st, sc);
-    if (s != NTC_OK) return s;
-    e = launch_bucket(A, q, n, sc, st, &launches, c->d_status);
+    e = launch_bucket(A, q, n, scratch_of(c), st, &launches);
     if (e != cudaSuccess) {
       c->launches += launches;
       return cuda_fail(e, "bucketing launch");
     }
+    B.queries = q;
     B.sorted = c->d_sorted;
     B.perm = c->d_perm;
     B.meta = c->d_meta;
@@ -665,10 +655,7 @@ ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *
   }
   s = ensure_scratch(c, n, st);
   if (s != NTC_OK) return s;
-  Scratch sc;
-  s = next_scratch(c, st, sc);
-  if (s != NTC_OK) return s;
-  cudaError_t e = launch_bucket(assets_of(c), q, n, sc, st, &launches, c->d_status);
+  cudaError_t e = launch_bucket(assets_of(c), q, n, scratch_of(c), st, &launches);
   if (e == cudaSuccess) e = cudaMemcpyAsync(perm, c->d_perm, n * 4, cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && (counts || tiles || num_tiles))
     e = launch_tiles_export(c->d_meta, c->D, tiles, num_tiles, counts, ntc_max_tiles(c, n), st, &launches);

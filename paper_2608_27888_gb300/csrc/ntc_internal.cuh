@@ -123,13 +123,15 @@ inline __host__ __device__ size_t gen_fma_image_bytes(uint32_t in_dim, uint32_t 
   return (w + 15) / 16 * 16 + ((size_t)layers * H + CP) * 4;
 }
 
-// Bucketing results on the device.  identity_n != 0: one decoder and no
-// sorting; `sorted` is the caller's query array itself (identity_n queries),
-// perm and meta are unused.
+// Bucketing results on the device: row i of the bucketed order is query
+// perm[i] of the caller's array, whose record is sorted[i].  identity_n != 0:
+// one decoder and no sorting, row i is query i of `queries` (identity_n
+// queries); sorted, perm and meta are unused.
 struct Buckets {
-  const ntc_query *sorted;  // queries in (decoder, index) order
-  const uint32_t *perm;     // original index of each sorted query
-  const uint32_t *meta;     // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
+  const ntc_query *queries;  // the caller's queries, in their own order
+  const ntc_query *sorted;   // the query records in (decoder, index) order
+  const uint32_t *perm;      // original index of each row
+  const uint32_t *meta;      // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
   uint32_t identity_n = 0;
 };
 inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2); }
@@ -419,6 +421,13 @@ __device__ __forceinline__ ntc_query load_query(const ntc_query *q) {
   return out;
 }
 
+// Row `pos` of the bucketed order: its output row (original index) and query
+// (two independent loads).
+__device__ __forceinline__ void bucket_row(const Buckets &B, uint32_t pos, uint32_t &oi, ntc_query &q) {
+  oi = B.identity_n ? pos : __ldg(B.perm + pos);
+  q = load_query((B.identity_n ? B.queries : B.sorted) + pos);
+}
+
 // Tile t of the bucketed order: decoder, first sorted position and length.
 __device__ __forceinline__ void tile_info(const uint32_t *meta, uint32_t D, uint32_t t,
                                           uint32_t &dec, uint32_t &start, uint32_t &len) {
@@ -462,25 +471,22 @@ struct TileWalk {
 
 // Device scratch of one bucketing call.
 struct Scratch {
-  uint32_t *perm;             // [n]
-  ntc_query *sorted;          // [n]
-  uint32_t *meta;             // bucket_meta_words(D): the tile table, then the
-                              // totals [D+1] and two tickets, zero between calls
-  unsigned long long *desc;   // [bucket_desc_words(D, n)] look-back descriptors
-  uint32_t epoch;             // 1 .. kBucketEpochs - 1, different from the
-                              // previous call's on the same descriptors
+  uint32_t *perm;     // [n]
+  ntc_query *sorted;  // [n] the query records in bucket order
+  uint32_t *meta;     // bucket_meta_words(D): the tile table, then the totals
+                      // [D+1] and a ticket (zero between calls)
+  uint32_t *counts;   // [bucket_count_words(D, n)] per-chunk counts, then offsets
 };
-constexpr uint32_t kBucketEpochs = 1u << 30;  // descriptors are cleared when the epoch wraps
 
 constexpr int kBucketThreads = 256;
 constexpr int kBucketItems = 8;  // queries per thread
 constexpr int kBucketChunk = kBucketThreads * kBucketItems;
 size_t bucket_chunks(size_t n);
-size_t bucket_desc_words(uint32_t D, size_t n);
+size_t bucket_count_words(uint32_t D, size_t n);
 size_t bucket_meta_words(uint32_t D);
 
-cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s,
-                          cudaStream_t st, int *launches, unsigned int *status);
+cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s, cudaStream_t st,
+                          int *launches);
 cudaError_t launch_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,
                                 uint32_t *counts, size_t max_tiles, cudaStream_t st, int *launches);
 cudaError_t launch_decode_fp32(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,

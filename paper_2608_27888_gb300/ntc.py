@@ -22,10 +22,15 @@ NTC_MODE_BUCKETED, NTC_MODE_DIVERGENT, NTC_MODE_BUCKETED_MMA, NTC_MODE_DIVERGENT
 NTC_MAX_DECODERS = 4095
 NTC_TILE_ROWS = 128
 
+# ntc_debug_row (include/ntc.h), 512 bytes
+DEBUG_ROW = np.dtype([("idx", "<u8", (2, 2, 4)), ("raw", "<u4", (2, 2, 4, 4)), ("w", "<f4", (2, 2, 4)),
+                      ("t", "<f4"), ("lo", "<u4"), ("feat", "<u4", (8,)), ("pad", "<u4", (6,))])
+assert DEBUG_ROW.itemsize == 512
+
 PRECISIONS = {"fp16": NTC_PREC_TC_FP16, "bf16": NTC_PREC_TC_BF16, "fp32": NTC_PREC_FP32}
 MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucketed_mma": NTC_MODE_BUCKETED_MMA,
          "divergent_fma": NTC_MODE_DIVERGENT_FMA}
-EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps",
+EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps", "ntc_debug_decode_rows",
            "ntc_debug_features", "ntc_debug_bucket", "ntc_max_tiles", "ntc_get_error_count",
            "ntc_reset_error_count", "ntc_launch_count", "ntc_set_stage_timing", "ntc_stage_times",
            "ntc_bucket_static", "ntc_kmeans_map", "ntc_debug_wait_timeout", "ntc_last_error",
@@ -75,6 +80,7 @@ def _load():
         "ntc_destroy": ([P], I),
         "ntc_debug_taps": ([P, P, S, P, P, P, P], I),
         "ntc_debug_features": ([P, P, S, P, P], I),
+        "ntc_debug_decode_rows": ([P, P, S, P, P, P], I),
         "ntc_debug_bucket": ([P, P, S, P, P, P, P, P], I),
         "ntc_max_tiles": ([P, S], S),
         "ntc_get_error_count": ([P, P], I),
@@ -83,7 +89,7 @@ def _load():
         "ntc_launch_count": ([P], ctypes.c_uint64),
         "ntc_set_stage_timing": ([P, I], I),
         "ntc_stage_times": ([P, P], I),
-        "ntc_bucket_static": ([P, ctypes.c_uint32, ctypes.c_uint32, P, S, P, P, P, P], I),
+        "ntc_bucket_static": ([P, ctypes.c_uint32, ctypes.c_uint32, P, S, P, P, P], I),
         "ntc_kmeans_map": ([P, ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, P, ctypes.c_uint32, P, P, P], I),
         "ntc_last_error": ([], ctypes.c_char_p),
         "ntc_status_string": ([I], ctypes.c_char_p),
@@ -131,6 +137,10 @@ def ntc_debug_features(ctx, d_queries, n, d_feat, stream):
     _check(_lib.ntc_debug_features(ctx, d_queries, n, d_feat, stream))
 
 
+def ntc_debug_decode_rows(ctx, d_queries, n, d_out, d_rows, stream):
+    _check(_lib.ntc_debug_decode_rows(ctx, d_queries, n, d_out, d_rows, stream))
+
+
 def ntc_debug_bucket(ctx, d_queries, n, d_perm, d_counts, d_tiles, d_num_tiles, stream):
     _check(_lib.ntc_debug_bucket(ctx, d_queries, n, d_perm, d_counts, d_tiles, d_num_tiles, stream))
 
@@ -167,11 +177,10 @@ def ntc_stage_times(ctx):
     return float(t[0]), float(t[1])
 
 
-def ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm, d_sorted, d_status,
-                      stream):
+def ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm, d_sorted, stream):
     """Allocation-free bucketing (no context): see include/ntc.h."""
     _check(_lib.ntc_bucket_static(h_set_to_decoder, num_sets, num_decoders, d_queries, n, d_perm,
-                                  d_sorted, d_status, stream))
+                                  d_sorted, stream))
 
 
 def ntc_kmeans_map(h_features, n, dim, m, h_init, max_iters, h_map, h_centroids, iters_run):
@@ -298,6 +307,17 @@ class Decoder:
         f = torch.empty((n, self.in_dim), dtype=torch.float32, device=queries.device)
         ntc_debug_features(self.ctx, _ptr(queries), n, _ptr(f), _stream(stream))
         return f
+
+    def decode_rows(self, queries, stream=None):
+        """The bucketed tensor-core decode through its debug build: (outputs,
+        rows) with rows a numpy structured array of ``DEBUG_ROW`` records
+        (ntc_debug_row; rows of bad queries keep their fill of 0xFF bytes)."""
+        import torch
+        n = queries.shape[0]
+        out = torch.empty((n, self.out_dim), dtype=torch.float32, device=queries.device)
+        rows = torch.full((max(1, n), DEBUG_ROW.itemsize), 255, dtype=torch.uint8, device=queries.device)
+        ntc_debug_decode_rows(self.ctx, _ptr(queries), n, _ptr(out), _ptr(rows), _stream(stream))
+        return out, rows[:n].cpu().numpy().view(DEBUG_ROW).reshape(n)
 
     def bucket(self, queries, stream=None):
         import torch
