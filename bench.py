@@ -1,27 +1,29 @@
 #!/usr/bin/env python3
 """Benchmark: decoded queries/s of the neural-texture decode on one GB300.
 
-Workload (one "step" = one ntc_decode over one batch): 16 texture sets of
-1024^2 (latents 512^2x8 + 256^2x8 fp16 each), 16 decoders 16->64->64->8 (the
-non-shared baseline, one decoder per set), 4,194,304 queries with a uniform
-random set id, uniform UV in [0,1)^2 and lod 0 -- fully divergent (about 14
-distinct decoders per 32-query warp).  Inputs are resident in HBM; L2 is
-flushed (a 256 MiB write, then a 256 MiB read of another buffer, so no dirty
-flush lines are written back inside a step) before every timed step and the flush is outside the
-step's CUDA events.
+Headline workload (one "step" = one ntc_decode over one batch): 4 frames of a
+3840x2160 G-buffer query stream -- 33,177,600 queries from 2000 Voronoi regions
+over 512 texture sets of 2048^2 (latents 1024^2x8 + 512^2x8 fp16 with their mip
+chains, 13.3 GiB), 8 shared decoders 16->128->128->9, a continuous lod per
+region in [0, 3) (trilinear: two mips per latent grid).  Inputs are resident in
+HBM; L2 is flushed (a 256 MiB write, then a 256 MiB read of another buffer, so
+no dirty flush lines are written back inside a step) before every timed step
+and the flush is outside the step's CUDA events.
 
-Beside the headline the line carries the in-run comparisons: the unsorted
-mma.sync ("divergent") and per-lane FMA ("divergent_fma") kernels on the same
-batch, a sweep over exactly d distinct decoders per warp, and a mirror of the
-paper's Tables 5-6 (shared vs non-shared decoders at 5 and 10 decoders per warp,
-512^2 to 8192^2 queries).
+The same JSON line carries every other workload (a 256^2 texel-centre raster,
+4M uniform queries over 16 decoders, the 1080p and 2160p G-buffers under each
+of their decoder groupings), the unsorted mma.sync ("divergent") and per-lane
+FMA ("divergent_fma") kernels on the headline batch, a sweep over exactly d
+distinct decoders per warp, a mirror of the paper's Tables 5-6, the decode
+under the groupings of Table 2, and Sec. 4's own decoder shape.
 
-Prints one JSON line.  ``--impl reference`` times the CPU oracle instead (the
-only other code that computes the same result) on a bounded query sample.
+``--impl reference`` times the CPU oracle instead (the only other code that
+computes the same result) on a bounded, evenly spaced query sample.
 
-Multi-GPU (torchrun): every rank decodes its own 4M-query batch against a full
-replica of the assets -- queries are independent, so there is no collective on
-the data path (weak scaling); the step time is the max over ranks.
+Multi-GPU (torchrun): every rank decodes its own query stream of the same
+recipe against a full replica of the assets -- queries are independent, so
+there is no collective on the data path (weak scaling); the step time is the
+max over ranks.
 """
 from __future__ import annotations
 
@@ -43,15 +45,23 @@ sys.path.insert(0, ROOT)
 
 METRIC = "decoded queries/sec on 1 GB300 vs distinct decoders per warp; % of roofline"
 UNIT = "queries/s"
-WORKLOAD = ("uniform-4m: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16), 16 decoders "
-            "16->64->64->8 (one per set), 4,194,304 queries: uniform set id, uniform UV, lod 0")
+HEADLINE = "gbuffer-2160p-x4-trilinear"
+DESCRIPTIONS = {
+    "gbuffer-2160p-x4-trilinear": "gbuffer-2160p-x4-trilinear: 4 frames of a 3840x2160 G-buffer (33,177,600 queries, "
+                                  "2000 Voronoi regions, lod ~U[0,3) per region, trilinear) over 512 texture sets of "
+                                  "2048^2 (latents 1024^2x8 + 512^2x8 fp16 with mip chains), 8 decoders "
+                                  "16->128->128->9 (random partition)",
+    "uniform-4m": "uniform-4m: 16 texture sets of 1024^2 (latents 512^2x8 + 256^2x8 fp16), 16 decoders "
+                  "16->64->64->8 (one per set), 4,194,304 queries: uniform set id, uniform UV, lod 0",
+}
 L2_FLUSH_BYTES = 256 << 20
-KERNEL_NAMES = {("bucketed", False): "k_decode_tc (tcgen05/TMEM gather-decode)",
+KERNEL_NAMES = {("bucketed", False): "k_decode_tm (tcgen05/TMEM gather-decode)",
                 ("bucketed", True): "k_decode_fp32 (FFMA gather-decode)",
                 ("bucketed_mma", False): "k_decode_mma (mma.sync gather-decode)",
                 ("divergent", False): "k_decode_divergent (mma.sync, unsorted)",
                 ("divergent_fma", False): "k_decode_divergent_fma (per-lane FFMA, unsorted)",
                 ("divergent_fma", True): "k_decode_divergent_fma (per-lane FFMA, unsorted)"}
+NAMED = ("raster-256", "uniform-4m", "gbuffer-1080p", "gbuffer-2160p", "gbuffer-2160p-x4-trilinear")
 
 
 def parse():
@@ -62,19 +72,18 @@ def parse():
     p.add_argument("--impl", default="ntc", choices=["ntc", "reference"])
     p.add_argument("--mode", default="bucketed", choices=["bucketed", "bucketed_mma", "divergent", "divergent_fma"])
     p.add_argument("--precision", default="fp16", choices=["fp16", "bf16", "fp32"])
+    p.add_argument("--workload", default=HEADLINE, choices=list(NAMED) + ["paper-decoder"],
+                   help="the timed batch (default: the 4-frame 2160p trilinear G-buffer); paper-decoder is "
+                        "Sec. 4's decoder (256^2x4 grid, positional encoding, LeakyReLU, 64x3) on a 1080p G-buffer")
+    p.add_argument("--variant", default=None, help="decoder grouping of the timed gbuffer-1080p / gbuffer-2160p batch")
+    p.add_argument("--no-workloads", action="store_true", help="skip the per-workload table")
     p.add_argument("--no-sweep", action="store_true", help="skip the decoders-per-warp sweep")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     p.add_argument("--no-mirror", action="store_true", help="skip the mirror of the paper's Tables 5-6")
-    p.add_argument("--maps", action="store_true",
-                   help="also decode a 586-set workload under the five groupings of Table 2")
-    p.add_argument("--variants", action="store_true",
-                   help="also time Sec. 4's decoder and the A x B sizes of its MLP ablation")
-    p.add_argument("--workloads", action="store_true",
-                   help="also time every full-size named workload and its groupings; adds about two minutes")
-    p.add_argument("--small", action="store_true", help="tiny workload (profiling captures)")
-    p.add_argument("--workload", default="uniform-4m", choices=["uniform-4m", "paper-decoder"],
-                   help="the timed batch: the 4M-query 16-decoder workload (default), or Sec. 4's "
-                        "decoder (256^2x4 grid, positional encoding, LeakyReLU, 64x3) on a 1080p G-buffer")
+    p.add_argument("--no-maps", action="store_true", help="skip the Table 2 groupings of a 586-set workload")
+    p.add_argument("--no-variants", action="store_true", help="skip Sec. 4's decoder shape")
+    p.add_argument("--variants", action="store_true", help="also time every A x B size of Sec. 4's MLP ablation")
+    p.add_argument("--small", action="store_true", help="the small size of the timed workload (profiling captures)")
     return p.parse_args()
 
 
@@ -148,16 +157,16 @@ def peaks():
 
 # the sources each recorded decode kernel is built from
 KERNEL_SOURCES = {
-    "bucketed-fp16": ("decode_tc.cu", "tcgen05.cuh", "ntc_internal.cuh"),
-    "bucketed-fp16-paper-decoder": ("decode_gen.cu", "tcgen05.cuh", "ntc_internal.cuh"),
+    "k_decode_tm": ("decode_tc.cuh", "decode_tc.cu", "tcgen05.cuh", "ntc_internal.cuh"),
+    "k_decode_gen_tc": ("decode_gen.cu", "tcgen05.cuh", "ntc_internal.cuh"),
 }
 
 
-def kernel_source_hash(kernel_tag):
+def kernel_source_hash(kernel):
     """Hash of one decode kernel's sources with comments and blank space
     removed, so a comment edit does not detach the recorded DRAM traffic."""
     h = hashlib.sha1()
-    for f in KERNEL_SOURCES[kernel_tag]:
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2608_27888_gb300", "csrc", f)) as fh:
             src = fh.read()
         src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
@@ -166,19 +175,49 @@ def kernel_source_hash(kernel_tag):
     return h.hexdigest()[:12]
 
 
-def recorded_traffic(kernel_tag):
+def recorded_traffic(kernel, workload):
     """DRAM bytes per decode launch from the committed ncu summary, if it was
-    taken on the current kernel source."""
+    taken on the current kernel source (a capture on a reduced case is scaled
+    to the full launch by its query count, as the record says)."""
     path = os.path.join(ROOT, "profiles", "decode_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
-        r = rec.get(kernel_tag)
-        if r and kernel_tag in KERNEL_SOURCES and r.get("source_hash") == kernel_source_hash(kernel_tag):
+        r = rec.get(f"{kernel}:{workload}")
+        if r and r.get("source_hash") == kernel_source_hash(kernel):
             return float(r["dram_bytes_per_launch"])
     except Exception:
         pass
     return None
+
+
+def compulsory(workload):
+    """The oracle's count of the bytes a decode of this workload must move
+    (tests/golden/compulsory_bytes.json, written by make_compulsory.py)."""
+    try:
+        with open(os.path.join(ROOT, "tests", "golden", "compulsory_bytes.json")) as f:
+            return json.load(f)["workloads"].get(workload)
+    except Exception:
+        return None
+
+
+def cpu_model():
+    """The host CPU as /proc/cpuinfo names it (Arm parts by implementer/part)."""
+    arm_parts = {0xd4f: "Neoverse-V2", 0xd40: "Neoverse-V1", 0xd0c: "Neoverse-N1", 0xd49: "Neoverse-N2"}
+    try:
+        txt = open("/proc/cpuinfo").read()
+    except OSError:
+        return "unknown"
+    m = re.search(r"^model name\s*:\s*(.+)$", txt, re.M)
+    if m:
+        return m.group(1).strip()
+    imp = re.search(r"^CPU implementer\s*:\s*(\S+)", txt, re.M)
+    part = re.search(r"^CPU part\s*:\s*(\S+)", txt, re.M)
+    if part:
+        p = int(part.group(1), 16)
+        name = arm_parts.get(p, f"part {part.group(1)}")
+        return f"{'Arm ' if imp and imp.group(1) == '0x41' else ''}{name}"
+    return "unknown"
 
 
 def dist_env():
@@ -191,7 +230,7 @@ def dist_env():
 def shape_costs(a, q):
     """Algorithmic bytes and FLOPs per query of a workload: the query record,
     every tap's latent texel (both mips when the lod is fractional), the fp32
-    outputs; 2 x the MACs of the MLP."""
+    outputs; 2 x the MACs of the MLP; and the fp16 weights of every decoder."""
     tri = a.num_mips > 1 and bool((q["lod"] != np.floor(q["lod"])).any())
     bpq = 16 + (2 if tri else 1) * a.num_levels * 4 * a.channels * 2 + 4 * a.out_dim
     H = a.hidden
@@ -200,17 +239,14 @@ def shape_costs(a, q):
     return bpq, flops, w_bytes
 
 
-def workload(small: bool, rank: int, name: str = "uniform-4m"):
+def workload(name: str, small: bool, rank: int, variant=None):
     """The benchmark batch of one rank: the same assets on every rank, a
-    rank-specific query stream (queries are sharded, assets replicated)."""
+    rank-specific query stream of the same recipe (queries are sharded, assets
+    replicated)."""
     from paper_2608_27888_gb300 import workloads as W
     if name == "paper-decoder":
         return W.paper_decoder("small" if small else "full")
-    seed = W.BASE_SEED + 2
-    S, T, n = (16, 128, 40_077) if small else (16, 1024, 4_194_304)
-    a = W.make_assets(seed, S, T, 1, S, W.map_identity(S))
-    q = W.queries_uniform(seed + 1000 * rank, n, S)
-    return W.Workload("uniform-4m-small" if small else "uniform-4m-full", a, q, {})
+    return W.named(name, "small" if small else "full", variant, query_tag=rank)
 
 
 def aggregate(n_per_rank: int, ms_local: float, dist=None):
@@ -236,15 +272,21 @@ def mean_distinct(q, assets):
 
 # -------------------------------------------------------------- reference arm
 
+def cpu_sample(q):
+    """The bounded CPU sample of a batch: every 32nd query (about 1M of the
+    headline's 33M), so it spans every frame and region."""
+    stride = max(1, len(q) // (1 << 20))
+    return q[::stride], stride
+
+
 def run_reference(args, ws, rank):
     if rank != 0:
         return
     import oracle
-    w = workload(args.small, 0, args.workload)
-    n = len(w.queries)
+    w = workload(args.workload, args.small, 0, args.variant)
+    q, stride = cpu_sample(w.queries)
+    sample = len(q)
     cores = os.cpu_count() or 1
-    sample = min(n, 1 << 20)
-    q = w.queries[:sample]
     for _ in range(max(0, args.warmup)):
         oracle.decode(w.assets, q[:4096], nthreads=cores)
     times = []
@@ -254,13 +296,15 @@ def run_reference(args, ws, rank):
         times.append(time.perf_counter() - t0)
     ms = 1e3 * statistics.mean(times)
     value = sample / (ms / 1e3)
-    desc = f"first {sample:,} queries of the workload per step, oracle on {cores} host threads"
+    desc = (f"every {stride}th query of the workload ({sample:,} of {len(w.queries):,}) per step, oracle on "
+            f"{cores} host threads ({cpu_model()})")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD if args.workload == "uniform-4m" else w.name, "sample_queries": sample},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
+        "config": {"workload": DESCRIPTIONS.get(args.workload, w.name), "sample_queries": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
+                         "sample": desc},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
@@ -281,7 +325,7 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     from paper_2608_27888_gb300 import ntc
 
-    w = workload(args.small, rank, args.workload)
+    w = workload(args.workload, args.small, rank, args.variant)
     n = len(w.queries)
     C = w.assets.out_dim
     dec = ntc.Decoder(w.assets, args.precision)
@@ -336,19 +380,31 @@ def main():
     bucket_ms = statistics.mean(s[0] for s in stages)
     decode_ms = statistics.mean(s[1] for s in stages)
 
-    # roofline of the dominant kernel (the gather-decode)
+    # roofline of the dominant kernel (the gather-decode), by algorithmic bytes;
+    # beside it the compulsory bytes the oracle counted (distinct texels)
     peak, peak_kind = peaks()
     bpq, flops_q, w_bytes = shape_costs(w.assets, w.queries)
     alg_bytes = n * bpq + w_bytes
     achieved = alg_bytes / (decode_ms / 1e3) / 1e9
-    kernel_tag = f"{args.mode}-{args.precision}" + ("" if args.workload == "uniform-4m" else f"-{args.workload}")
+    general = args.workload == "paper-decoder"
+    kernel = "k_decode_gen_tc" if general else "k_decode_tm"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": recorded_traffic(kernel_tag),
-                "kernel": KERNEL_NAMES[(args.mode, args.precision == "fp32")] if args.workload == "uniform-4m"
-                else "k_decode_gen_tc (general-shape tcgen05 gather-decode)",
+                "frac": achieved / peak, "traffic": recorded_traffic(kernel, args.workload),
+                "kernel": ("k_decode_gen_tc (general-shape tcgen05 gather-decode)" if general
+                           else KERNEL_NAMES[(args.mode, args.precision == "fp32")]),
                 "kernel_ms": decode_ms, "bucketing_ms": bucket_ms,
                 "peak_kind": f"{peak_kind} HBM copy bandwidth",
-                "algorithmic_bytes_per_launch": alg_bytes}
+                "algorithmic_bytes_per_launch": alg_bytes, "algorithmic_bytes_per_query": bpq,
+                "step_frac": (n * bpq + w_bytes) / (ms_step / 1e3) / 1e9 / peak}
+    comp = compulsory(args.workload) if not args.small else None
+    if comp and comp["queries"] == n:
+        cb = comp["compulsory_bytes_excluding_weights"] + w_bytes
+        roofline["compulsory"] = {
+            "bytes_per_launch": cb, "bytes_per_query": cb / n,
+            "touched_texels": comp["touched_texels"],
+            "achieved": cb / (decode_ms / 1e3) / 1e9, "frac": cb / (decode_ms / 1e3) / 1e9 / peak,
+            "step_frac": cb / (ms_step / 1e3) / 1e9 / peak,
+            "what": "queries + outputs + distinct latent texels touched (counted by the oracle) + weights"}
 
     # end to end through the public host-buffer call
     hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
@@ -364,16 +420,26 @@ def main():
     e2e_ms = 1e3 * statistics.mean(e2e_t)
     e2e = {"value": n * ws / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": n * 16,
            "d2h_bytes_per_step": n * C * 4, "ms_per_step": e2e_ms}
+    del hq, hout
 
-    # the in-run comparison: the unsorted divergent kernel on the same batch
+    # the in-run comparison: the unsorted kernels on the same batch
     extra = {}
     for other in ("divergent", "divergent_fma"):
-        if args.mode == other or (other == "divergent" and (args.precision == "fp32" or args.workload != "uniform-4m")):
+        if args.mode == other or (other == "divergent" and (args.precision == "fp32" or general)):
             continue
-        dms, _, _ = timed_steps(other, max(5, args.steps // 2), 2)
+        dms, _, _ = timed_steps(other, 3 if n > 10_000_000 else 5, 1)
         extra[other] = {"value": n * ws / (statistics.mean(dms) / 1e3), "unit": UNIT,
                         "ms_per_step": statistics.mean(dms)}
     dd = mean_distinct(w.queries, w.assets)
+    headline_row = {"workload": w.name, "queries": n, "decoders": w.assets.num_decoders,
+                    "hidden": w.assets.hidden, "mean_distinct_decoders_per_warp": dd,
+                    "divergence_score_eq1": dd - 1.0, "bucketed": value / ws, "ms_per_step": ms_step,
+                    "bucketing_ms": bucket_ms, "decode_ms": decode_ms, "bytes_per_query": bpq,
+                    "roofline_rate": peak * 1e9 / bpq, "frac_of_roofline": value / ws / (peak * 1e9 / bpq),
+                    **{k: v["value"] / ws for k, v in extra.items()}}
+    dec.close()
+    del qd, out, dec
+    torch.cuda.empty_cache()
 
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
@@ -382,28 +448,28 @@ def main():
         "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f16" if args.precision == "fp16" else args.precision.replace("fp", "f"),
         "data": "synthetic",
-        "config": {"workload": (WORKLOAD if args.workload == "uniform-4m" else w.name) if not args.small else w.name,
+        "config": {"workload": DESCRIPTIONS.get(args.workload, w.name) if not args.small else w.name,
                    "queries_per_gpu": n,
                    "decoders": w.assets.num_decoders, "mode": args.mode, "precision": args.precision,
                    "mean_distinct_decoders_per_warp": dd,
-                   "l2": "flushed before every timed step (256 MiB write, then a 256 MiB read of another buffer; outside the step events)",
+                   "l2": "flushed before every timed step (256 MiB write, then a 256 MiB read of another buffer; "
+                         "outside the step events); inputs larger than L2",
                    "parallelism": f"{ws} independent replicas (queries sharded, no collective)"},
         "roofline": roofline, "e2e": e2e, "gpu_launches": launches, "clocks": clocks,
         "flops_per_query": flops_q, "bytes_per_query": bpq,
         **extra,
     }
-
-    if not args.no_sweep and not args.small and rank == 0:
-        result["sweep"] = sweep(ntc, torch, args.precision)
-    if not args.no_mirror and not args.small and rank == 0 and args.precision != "fp32":
-        result["paper_mirror"] = paper_mirror(ntc, torch, args.precision)
-    if args.workloads and rank == 0:
-        result["workloads"] = per_workload(ntc, torch, args.precision)
-    if args.maps and rank == 0:
-        result["maps"] = map_sources(ntc, torch, args.precision)
-    if args.variants and rank == 0:
-        result["variants"] = decoder_variants(ntc, torch, args.precision)
-
+    if rank == 0 and not args.small:
+        if not args.no_workloads:
+            result["workloads"] = per_workload(ntc, torch, args.precision, headline=(args.workload, headline_row))
+        if not args.no_sweep:
+            result["sweep"] = sweep(ntc, torch, args.precision)
+        if not args.no_mirror and args.precision != "fp32":
+            result["paper_mirror"] = paper_mirror(ntc, torch, args.precision)
+        if not args.no_maps:
+            result["maps"] = map_sources(ntc, torch, args.precision)
+        if not args.no_variants:
+            result["variants"] = decoder_variants(ntc, torch, args.precision, every_size=args.variants)
     if rank == 0 and not args.no_cpu and ws == 1:
         result["cpu_baseline"] = cpu_baseline(w)
     if rank == 0:
@@ -474,19 +540,22 @@ def paper_mirror(ntc, torch, precision, sizes=(512, 1024, 2048, 4096, 8192), ds=
             "what": "32 sets of 1024^2, N x N texel-centre raster, d distinct sets per warp; times in us"}
 
 
-def decoder_variants(ntc, torch, precision):
+def decoder_variants(ntc, torch, precision, every_size=False):
     """Sec. 4's decoder (one 256x256x4 grid per set with a 4-mip chain,
-    positional encoding of 4 frequencies, LeakyReLU, 64 x 3) and the A x B sizes
-    of its MLP ablation (A neurons, B layers), 16 sets in 4 clusters, on a
-    1920x1080 G-buffer with a continuous lod (trilinear).  Queries/s of the
-    whole ntc_decode (bucketed: the general tcgen05 kernel for fp16/bf16) and of
-    the per-lane FMA mode, with the HBM-bound rate of the algorithmic bytes."""
+    positional encoding of 4 frequencies, LeakyReLU, 64 x 3), and with
+    every_size the A x B sizes of its MLP ablation (A neurons, B layers), 16
+    sets in 4 clusters, on a 1920x1080 G-buffer with a continuous lod
+    (trilinear).  Queries/s of the whole ntc_decode (bucketed: the general
+    tcgen05 kernel for fp16/bf16) and of the per-lane FMA mode, with the
+    HBM-bound rate of the algorithmic bytes."""
     from paper_2608_27888_gb300 import workloads as W
     peak, _ = peaks()
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     rows = []
-    shapes = [(64, 3)] + [(a, b) for a in (32, 64, 128) for b in (2, 3, 4, 5) if (a, b) != (64, 3)]
+    shapes = [(64, 3)]
+    if every_size:
+        shapes += [(a, b) for a in (32, 64, 128) for b in (2, 3, 4, 5) if (a, b) != (64, 3)]
     for A_, B_ in shapes:
         w = W.paper_decoder("full", hidden=A_, layers=B_ - 1)
         a, q = w.assets, w.queries
@@ -552,10 +621,12 @@ def map_sources(ntc, torch, precision):
             "what": "586 sets of 1024^2, 1920x1080 G-buffer, 600 regions; Gq/s of the whole ntc_decode"}
 
 
-def per_workload(ntc, torch, precision):
-    """Every full-size workload: queries/s of the whole ntc_decode (bucketed),
-    the bucketing / gather-decode split, the unsorted kernels, and the whole
-    step against the roofline rate of that workload's algorithmic bytes."""
+def per_workload(ntc, torch, precision, headline=None):
+    """Every full-size workload under each of its decoder groupings: queries/s
+    of the whole ntc_decode (bucketed), the bucketing / gather-decode split,
+    the unsorted kernels, and the whole step against the roofline rate of that
+    workload's algorithmic bytes and against the compulsory bytes the oracle
+    counted.  The headline workload's row is the one measured above."""
     from paper_2608_27888_gb300 import workloads as W
     peak, _ = peaks()
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
@@ -565,37 +636,44 @@ def per_workload(ntc, torch, precision):
                           ("gbuffer-1080p", "clustered4"), ("gbuffer-1080p", "shared"), ("gbuffer-2160p", "128"),
                           ("gbuffer-2160p", "16"), ("gbuffer-2160p", "8"), ("gbuffer-2160p", "1"),
                           ("gbuffer-2160p-x4-trilinear", None)):
-        w = W.named(name, "full", variant)
-        a, q = w.assets, w.queries
-        n, C = len(q), a.out_dim
-        dec = ntc.Decoder(a, precision)
-        qd = ntc.queries_to_device(q)
-        out = torch.empty((n, C), dtype=torch.float32, device="cuda")
-        ms = time_decode(torch, dec, qd, out, "bucketed", flush, flush_rd, reps=10, warm=3)
-        dec.set_stage_timing(True)
-        st = []
-        for _ in range(5):
-            flush.zero_()
-            flush_rd.sum()
-            dec.decode(qd, out, mode="bucketed")
-            st.append(dec.stage_times())
-        dec.set_stage_timing(False)
-        tri = a.num_mips > 1 and bool((q["lod"] != np.floor(q["lod"])).any())
-        bpq = 16 + (16 if tri else 8) * 16 + 4 * C
-        dd = mean_distinct(q, a)
-        row = {"workload": w.name, "queries": n, "decoders": a.num_decoders, "hidden": a.hidden,
-               "mean_distinct_decoders_per_warp": dd, "divergence_score_eq1": dd - 1.0,
-               "bucketed": n / (ms / 1e3), "ms_per_step": ms,
-               "bucketing_ms": statistics.mean(t[0] for t in st), "decode_ms": statistics.mean(t[1] for t in st),
-               "bytes_per_query": bpq, "roofline_rate": peak * 1e9 / bpq}
-        row["frac_of_roofline"] = row["bucketed"] / row["roofline_rate"]
-        reps = 3 if n > 10_000_000 else 5
-        for m in (("divergent_fma",) if precision == "fp32" else ("divergent", "divergent_fma")):
-            row[m] = n / (time_decode(torch, dec, qd, out, m, flush, flush_rd, reps=reps, warm=1) / 1e3)
+        comp = compulsory(name)
+        if headline and headline[0] == name and variant is None:
+            row = dict(headline[1])
+        else:
+            w = W.named(name, "full", variant)
+            a, q = w.assets, w.queries
+            n, C = len(q), a.out_dim
+            dec = ntc.Decoder(a, precision)
+            qd = ntc.queries_to_device(q)
+            out = torch.empty((n, C), dtype=torch.float32, device="cuda")
+            ms = time_decode(torch, dec, qd, out, "bucketed", flush, flush_rd, reps=10, warm=3)
+            dec.set_stage_timing(True)
+            st = []
+            for _ in range(5):
+                flush.zero_()
+                flush_rd.sum()
+                dec.decode(qd, out, mode="bucketed")
+                st.append(dec.stage_times())
+            dec.set_stage_timing(False)
+            bpq, _, _ = shape_costs(a, q)
+            dd = mean_distinct(q, a)
+            row = {"workload": w.name, "queries": n, "decoders": a.num_decoders, "hidden": a.hidden,
+                   "mean_distinct_decoders_per_warp": dd, "divergence_score_eq1": dd - 1.0,
+                   "bucketed": n / (ms / 1e3), "ms_per_step": ms,
+                   "bucketing_ms": statistics.mean(t[0] for t in st), "decode_ms": statistics.mean(t[1] for t in st),
+                   "bytes_per_query": bpq, "roofline_rate": peak * 1e9 / bpq}
+            row["frac_of_roofline"] = row["bucketed"] / row["roofline_rate"]
+            reps = 3 if n > 10_000_000 else 5
+            for m in (("divergent_fma",) if precision == "fp32" else ("divergent", "divergent_fma")):
+                row[m] = n / (time_decode(torch, dec, qd, out, m, flush, flush_rd, reps=reps, warm=1) / 1e3)
+            dec.close()
+            del qd, out, w, a, q
+            torch.cuda.empty_cache()
+        if comp and comp["queries"] == row["queries"]:
+            cpq = comp["compulsory_bytes_per_query_excluding_weights"]
+            row["compulsory_bytes_per_query"] = cpq
+            row["frac_of_compulsory_roofline"] = row["bucketed"] / (peak * 1e9 / cpq)
         rows.append(row)
-        dec.close()
-        del qd, out, w, a, q
-        torch.cuda.empty_cache()
     return rows
 
 
@@ -630,12 +708,13 @@ def sweep(ntc, torch, precision):
 def cpu_baseline(w):
     import oracle
     cores = os.cpu_count() or 1
-    n = len(w.queries)
+    q, stride = cpu_sample(w.queries)
     t0 = time.perf_counter()
-    oracle.decode(w.assets, w.queries, nthreads=cores)
+    oracle.decode(w.assets, q, nthreads=cores)
     dt = time.perf_counter() - t0
-    return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"all {n:,} queries of one step (full workload), oracle on {cores} host threads, {dt:.1f} s"}
+    return {"value": len(q) / dt, "unit": UNIT, "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
+            "sample": f"every {stride}th query of the timed batch ({len(q):,} of {len(w.queries):,}), oracle on "
+                      f"{cores} host threads, {dt:.1f} s"}
 
 
 if __name__ == "__main__":

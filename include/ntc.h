@@ -213,10 +213,15 @@ NTC_API ntc_status ntc_debug_features(ntc_ctx *ctx, const ntc_query *d_queries, 
  * query with an out-of-range set id counts as decoder num_decoders.  d_counts (may be NULL): [num_decoders+1] queries per decoder.
  * d_tiles (may be NULL): [ntc_max_tiles(ctx, n)][3] = (decoder, first position
  * in perm, length) of every 128-query tile, in decoder order; d_num_tiles (may
- * be NULL): [1] the number of tiles written.  Device pointers; async. */
+ * be NULL): [1] the number of tiles written.  d_divergence (may be NULL): [2]
+ * = { 1 if the query records were copied in bucket order, else 0;  the sum
+ * over groups of 32 consecutive queries of (distinct decoders - 1), out-of-
+ * range set ids counting as decoder num_decoders } -- Eq. 1's numerator; the
+ * records are copied when that sum exceeds 4 x the number of groups.  Device
+ * pointers; async. */
 NTC_API ntc_status ntc_debug_bucket(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, uint32_t *d_perm,
                             uint32_t *d_counts, uint32_t *d_tiles, uint32_t *d_num_tiles,
-                            void *cuda_stream);
+                            uint32_t *d_divergence, void *cuda_stream);
 
 /* One query row as the default tensor-core decode (BUCKETED, TC_FP16/TC_BF16,
  * the standard shape) built it -- the bilinear fetch of Sec. 1's latent grids

@@ -5,20 +5,27 @@
 // bucket keeps the original order) turns the interleaved stream into runs of
 // single-decoder 128-query tiles.  Three kernels, none of which waits for
 // another CTA:
-//   k_count  per 2048-query chunk: the chunk's count of every decoder (set ->
-//            decoder map; out-of-range set ids form the extra bucket D)
+//   k_count  per 2048-query chunk: every query's decoder (set -> decoder map;
+//            out-of-range set ids form the extra bucket D), written as one
+//            byte (two beyond 255 decoders), the chunk's count of every
+//            decoder, and the divergence of its 32-query groups (Eq. 1:
+//            distinct decoders in a group - 1, summed)
 //   k_scan   one CTA per decoder scans that decoder's per-chunk counts into
 //            the chunk offsets; the last CTA to finish (atomic ticket) scans
-//            the decoder totals into the segment starts and the tile starts
-//   k_place  per chunk: the records arrive in shared memory by one bulk copy
-//            (TMA); each query's rank among the equal decoders of its chunk
-//            (stable); its place = segment start + chunk offset + rank; the
-//            chunk is sorted in shared memory and copied out with coalesced
-//            stores: perm[] and the query records in bucket order, which the
-//            decode then reads contiguously
-// Equal decoders within a warp are found with one ballot per bit of the
-// decoder id.  The permutation is exactly std::stable_sort of the indices by
-// decoder.
+//            the decoder totals into the segment starts and the tile starts,
+//            and decides from Eq. 1's score whether the records are copied
+//   k_place  per chunk: each query's rank among the equal decoders of its
+//            chunk (stable); its place = segment start + chunk offset + rank;
+//            the chunk is sorted in shared memory and copied out with
+//            coalesced stores: perm[] and, when k_scan chose to, the query
+//            records in bucket order (staged in shared memory by cp.async)
+// Divergence-aware: when the score is low (a G-buffer: most 32-query groups
+// need one decoder) a decoder's queries lie in long runs of the caller's
+// array, and the decode reads query perm[i] there directly; only a scattered
+// stream (score above kCopyAboveScore) pays for the copy, so its decode reads
+// contiguous records.  Equal decoders within a warp are found with one ballot
+// per bit of the decoder id.  The permutation is exactly std::stable_sort of
+// the indices by decoder.
 #include "ntc_internal.cuh"
 
 namespace ntc {
@@ -68,11 +75,15 @@ __device__ __forceinline__ uint32_t match_key(uint32_t key, int nbits) {
 
 // ------------------------------------------------------------------ k_count
 
-__global__ void __launch_bounds__(kBucketThreads, 8) k_count(Assets A, const ntc_query *q, size_t n,
-                                                          uint32_t chunks, uint32_t *counts) {
+template <typename DecT>
+__global__ void __launch_bounds__(kBucketThreads) k_count(Assets A, const ntc_query *q, size_t n,
+                                                             uint32_t chunks, uint32_t *counts, uint32_t *div_sum,
+                                                             DecT *dec_out) {
   extern __shared__ uint32_t cnt[];  // [kWarps][D+2]; column D+1 counts nothing
+  __shared__ uint32_t s_div;
   pdl_trigger();                     // k_scan may launch (it waits for this grid before reading)
   const uint32_t D = A.num_decoders, DW = D + 2;
+  if (threadIdx.x == 0) s_div = 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (uint32_t i = threadIdx.x; i < kWarps * DW; i += blockDim.x) cnt[i] = 0;
   __syncthreads();
@@ -87,16 +98,23 @@ __global__ void __launch_bounds__(kBucketThreads, 8) k_count(Assets A, const ntc
     s[it] = j < n ? __ldg(sid + 4 * j) : 0u;
   }
   uint32_t *my = cnt + warp * DW;
+  uint32_t div = 0;  // this warp's groups: distinct decoders - 1
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
     const size_t j = wbase + it * 32 + lane;
     const uint32_t dl = lookup(A, s[it]);  // every lane: the lookup shuffles
     const uint32_t d = j < n ? dl : D + 1;
+    if (dec_out && j < n) dec_out[j] = (DecT)d;
     const uint32_t m = match_key(d, nbits);
-    if (lane == __ffs(m) - 1) my[d] += __popc(m);
+    const bool leader = lane == __ffs(m) - 1;
+    if (leader) my[d] += __popc(m);
+    const uint32_t runs = __popc(__ballot_sync(0xFFFFFFFFu, leader && d <= D));
+    div += runs ? runs - 1 : 0u;
     __syncwarp();
   }
+  if (lane == 0 && div) atomicAdd(&s_div, div);
   __syncthreads();
+  if (threadIdx.x == 0 && s_div) atomicAdd(div_sum, s_div);
   for (uint32_t d = threadIdx.x; d <= D; d += blockDim.x) {
     uint32_t t = 0;
 #pragma unroll
@@ -158,13 +176,15 @@ __device__ uint32_t block_scan_inplace(uint32_t *a, uint32_t len, uint32_t *ws) 
   return carry;
 }
 
-// meta layout: [0] num_tiles, [1 .. D+2] seg_start, [D+3 .. 2D+4] tile_start;
-// then totals [D+1] and the ticket (zero between calls).
-__global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks, uint32_t D, uint32_t *meta) {
+// meta layout: [0] num_tiles, [1 .. D+2] seg_start, [D+3 .. 2D+4] tile_start,
+// [2D+5] copied, [2D+6] divergence; then totals [D+1], the ticket and the
+// divergence sum of k_count (zero between calls).
+__global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks, uint32_t D, uint32_t *meta,
+                                               int force_copy) {
   __shared__ uint32_t ws[32];
   __shared__ bool last;
   const uint32_t d = blockIdx.x;
-  uint32_t *totals = meta + meta_words(D), *ticket = totals + (D + 1);
+  uint32_t *totals = meta + meta_words(D), *ticket = totals + (D + 1), *div_sum = ticket + 1;
   pdl_wait();     // the per-chunk counts of k_count
   pdl_trigger();  // k_place may launch (it waits for this grid before reading)
   const uint32_t tot = block_scan_inplace(counts + (size_t)d * chunks, chunks, ws);
@@ -191,6 +211,12 @@ __global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks
     seg[D + 1] = ns;  // == n
     tst[D + 1] = nt;
     meta[0] = nt;
+    // Eq. 1's score: divergence sum over the ceil(n / 32) groups
+    const uint32_t div = *(volatile uint32_t *)div_sum;
+    const uint64_t groups = ((uint64_t)ns + 31) / 32;
+    meta[meta_copied(D)] = force_copy || (uint64_t)div > (uint64_t)kCopyAboveScore * groups ? 1u : 0u;
+    meta[meta_divergence(D)] = div;
+    *div_sum = 0;
     *ticket = 0;
   }
 }
@@ -231,8 +257,12 @@ __device__ __forceinline__ void cp_async16(void *smem_dst, const void *src) {
                : "memory");
 }
 
-__global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_query *q, size_t n,
-                                                          uint32_t chunks, const uint32_t *offs,
+// FROM_Q: the decoders come from the staged records (always copied);
+// otherwise from k_count's decoder array, and the records are staged only
+// when k_scan chose to copy them.
+template <typename DecT, bool FROM_Q>
+__global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc_query *q, const DecT *dec_in,
+                                                          size_t n, uint32_t chunks, const uint32_t *offs,
                                                           const uint32_t *meta, uint32_t *perm,
                                                           ntc_query *sorted) {
   // shared memory: the chunk's records [chunk] (16 B), the chunk-local index
@@ -249,13 +279,18 @@ __global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_qu
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
   const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
-  // the chunk's records (the caller's queries: no dependence on k_scan)
-  for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) cp_async16(srec + i, q + cbase + i);
-  asm volatile("cp.async.commit_group;\n" ::: "memory");
+  auto stage_records = [&]() {
+    for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) cp_async16(srec + i, q + cbase + i);
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+  };
+  if (FROM_Q) stage_records();  // the caller's queries: no dependence on k_scan
   for (uint32_t i = threadIdx.x; i < kWarps * DW; i += blockDim.x) cnt[i] = 0;
   const MapLookup lookup(A);
   const int nbits = key_bits(D);
-  asm volatile("cp.async.wait_all;\n" ::: "memory");
+  pdl_wait();  // k_scan's chunk offsets, segment starts and decision (and k_count's decoders)
+  const bool copy = FROM_Q || __ldcg(meta + meta_copied(D)) != 0u;
+  if (!FROM_Q && copy) stage_records();
+  if (FROM_Q) asm volatile("cp.async.wait_all;\n" ::: "memory");
   __syncthreads();
   const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
   uint32_t *my = cnt + warp * DW;
@@ -265,8 +300,13 @@ __global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_qu
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
     const uint32_t j = wbase + it * 32 + lane;
-    const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
-    const uint32_t d = j < valid ? dl : D + 1;
+    uint32_t d;
+    if (FROM_Q) {
+      const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
+      d = j < valid ? dl : D + 1;
+    } else {
+      d = j < valid ? (uint32_t)__ldcg(dec_in + cbase + j) : D + 1;
+    }
     const uint32_t m = match_key(d, nbits);
     dec[it] = d;
     rank[it] = my[d] + __popc(m & lt);
@@ -274,7 +314,6 @@ __global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_qu
     if (lane == __ffs(m) - 1) my[d] += __popc(m);
     __syncwarp();
   }
-  pdl_wait();  // the chunk offsets and segment starts of k_scan
   __syncthreads();
   // per decoder: warp prefix (in place), the chunk's count and its global base
   const uint32_t *seg = meta + 1;
@@ -300,6 +339,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_qu
     sidx[lp] = (uint16_t)(wbase + it * 32 + lane);
     sdec[lp] = (uint16_t)d;
   }
+  if (!FROM_Q && copy) asm volatile("cp.async.wait_all;\n" ::: "memory");
   __syncthreads();
   pdl_trigger();  // the decode may launch (it waits for this grid before reading)
   // coalesced copy-out: consecutive slots of one decoder go to consecutive
@@ -308,7 +348,7 @@ __global__ void __launch_bounds__(kBucketThreads) k_place(Assets A, const ntc_qu
     const uint32_t d = sdec[i], j = sidx[i];
     const uint32_t pos = gbase[d] + (i - loff[d]);
     perm[pos] = (uint32_t)(cbase + j);
-    reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
+    if (copy) reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
   }
 }
 
@@ -333,14 +373,17 @@ __global__ void k_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles
 
 size_t bucket_chunks(size_t n) { return (n + kBucketChunk - 1) / kBucketChunk; }
 size_t bucket_count_words(uint32_t D, size_t n) { return ((size_t)D + 1) * bucket_chunks(n); }
-size_t bucket_meta_words(uint32_t D) { return meta_words(D) + ((size_t)D + 1) + 1; }
+size_t bucket_meta_words(uint32_t D) { return meta_words(D) + ((size_t)D + 1) + 2; }
 
-cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s, cudaStream_t st,
-                          int *launches) {
+namespace {
+template <typename DecT>
+cudaError_t launch_bucket_t(const Assets &A, const ntc_query *q, size_t n, const Scratch &s, cudaStream_t st,
+                            int *launches, int copy) {
   const uint32_t chunks = (uint32_t)bucket_chunks(n);
   const uint32_t D = A.num_decoders, DW = D + 2;
   const size_t smem_count = (size_t)kWarps * DW * sizeof(uint32_t);
   const size_t smem_place = (size_t)kBucketChunk * (16 + 2 + 2) + (size_t)(kWarps + 2) * DW * sizeof(uint32_t);
+  const bool from_q = s.dec == nullptr;
   static PerDevice attrs;
   cudaError_t e = attrs.once([]() {
     // as much dynamic shared memory as the device allows a block: the
@@ -348,25 +391,47 @@ cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const S
     int dev = 0, optin = 0;
     cudaError_t r = cudaGetDevice(&dev);
     if (r == cudaSuccess) r = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    cudaFuncAttributes fc, fp;
-    if (r == cudaSuccess) r = cudaFuncGetAttributes(&fc, k_count);
-    if (r == cudaSuccess) r = cudaFuncGetAttributes(&fp, k_place);
-    if (r == cudaSuccess)
-      r = cudaFuncSetAttribute(k_count, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fc.sharedSizeBytes);
-    if (r == cudaSuccess)
-      r = cudaFuncSetAttribute(k_place, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fp.sharedSizeBytes);
+    auto allow = [&](auto kernel) {
+      cudaFuncAttributes fa;
+      cudaError_t x = cudaFuncGetAttributes(&fa, kernel);
+      if (x == cudaSuccess)
+        x = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
+      return x;
+    };
+    if (r == cudaSuccess) r = allow(k_count<DecT>);
+    if (r == cudaSuccess) r = allow(k_place<DecT, false>);
+    if (r == cudaSuccess) r = allow(k_place<DecT, true>);
     return r;
   });
   if (e != cudaSuccess) return e;
   *launches += 3;
-  k_count<<<chunks, kBucketThreads, smem_count, st>>>(A, q, n, chunks, s.counts);
+  uint32_t *div_sum = s.meta + meta_words(D) + (D + 1) + 1;
+  DecT *dec = reinterpret_cast<DecT *>(s.dec);
+  k_count<DecT><<<chunks, kBucketThreads, smem_count, st>>>(A, q, n, chunks, s.counts, div_sum, dec);
   e = cudaGetLastError();
-  if (e == cudaSuccess) e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, s.meta);
-  if (e == cudaSuccess)
-    e = launch_pdl(k_place, dim3(chunks), dim3(kBucketThreads), smem_place, st, A, q, n, chunks,
-                   (const uint32_t *)s.counts, (const uint32_t *)s.meta, s.perm, s.sorted);
+  if (e == cudaSuccess) e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, s.meta, copy);
+  if (e == cudaSuccess) {
+    if (from_q)
+      e = launch_pdl(k_place<DecT, true>, dim3(chunks), dim3(kBucketThreads), smem_place, st, A, q,
+                     (const DecT *)nullptr, n, chunks, (const uint32_t *)s.counts, (const uint32_t *)s.meta,
+                     s.perm, s.sorted);
+    else
+      e = launch_pdl(k_place<DecT, false>, dim3(chunks), dim3(kBucketThreads), smem_place, st, A, q,
+                     (const DecT *)dec, n, chunks, (const uint32_t *)s.counts, (const uint32_t *)s.meta, s.perm,
+                     s.sorted);
+  }
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+}  // namespace
+
+size_t bucket_dec_bytes(uint32_t D) { return D + 1 <= 256 ? 1 : 2; }
+
+cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s, cudaStream_t st,
+                          int *launches, int copy) {
+  if (!s.dec && !copy) return cudaErrorInvalidValue;  // without the decoder array the records are always staged
+  if (bucket_dec_bytes(A.num_decoders) == 1) return launch_bucket_t<uint8_t>(A, q, n, s, st, launches, copy);
+  return launch_bucket_t<uint16_t>(A, q, n, s, st, launches, copy);
 }
 
 cudaError_t launch_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,

@@ -23,7 +23,7 @@ using namespace ntc;
 namespace {
 
 constexpr size_t kMapWords = 65536;    // set->decoder map copy
-constexpr size_t kMetaWords = 12544;   // tile table, totals, ticket (<= 12292 words for D <= 4095)
+constexpr size_t kMetaWords = 12544;   // tile table, totals, ticket, divergence sum (<= 12295 words for D <= 4095)
 constexpr size_t kCountWords = 262144; // (D+1) * ceil(n / 2048) per-chunk counts
 constexpr size_t kStaticWords = kMapWords + kMetaWords + kCountWords;  // 1,360,896 bytes
 
@@ -96,8 +96,9 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
   s.meta = meta;
   s.counts = counts;
   s.sorted = d_sorted;
+  s.dec = nullptr;  // no room for a decoder per query: the placement reads the staged records
   int launches = 0;
-  e = launch_bucket(A, d_queries, n, s, st, &launches);
+  e = launch_bucket(A, d_queries, n, s, st, &launches, 1);  // d_sorted is always written
   if (e != cudaSuccess) return failed(NTC_ERR_CUDA, cudaGetErrorString(e));
   return NTC_OK;
 }

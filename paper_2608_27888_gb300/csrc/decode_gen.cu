@@ -159,6 +159,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
   const uint32_t tAH = tmem_slot + H;          // hidden A operand, H / 2 columns
   const uint32_t tA1 = tmem_slot + H + H / 2;  // ring stages, K1 / 2 columns each
   const uint32_t T = __ldg(B.meta);
+  const bool copied = rows_copied(B, D);
   const uint32_t grid = gridDim.x;
   // this CTA's tiles: a contiguous range t0 .. t0 + K - 1 of the tile list, so
   // consecutive tiles share their decoder and the weights are copied rarely
@@ -177,7 +178,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
       if (jj >= K) return;
       uint32_t d_, st_, len_;
       walk.at(seg, tst, D, t0 + jj, d_, st_, len_);
-      if (row < len_) bucket_row(B, st_ + row, oi_, q_);
+      if (row < len_) bucket_row(B, copied, st_ + row, oi_, q_);
     };
     uint32_t oi;
     ntc_query q;
@@ -450,12 +451,12 @@ __device__ __forceinline__ float act_f(float x, uint32_t act, float slope) {
   return x > 0.0f ? x : (act == 1 ? slope * x : 0.0f);
 }
 
-// Per-lane decode of a general shape; row i is qs[i] written to out[perm[i]]
-// (or query i itself when perm is null).
+// Per-lane decode of a general shape; row i is row i of the bucketed order B
+// (bucketed != 0) or query i of qs itself, written to its output row.
 template <typename T>
-__global__ void __launch_bounds__(128) k_decode_gen_fma(Assets A, GenWeights G, const ntc_query *qs,
-                                                        const uint32_t *perm, size_t n, float *out,
-                                                        unsigned long long *err) {
+__global__ void __launch_bounds__(128) k_decode_gen_fma(Assets A, GenWeights G, const ntc_query *qs, int bucketed,
+                                                        Buckets B, size_t n, float *out, unsigned long long *err) {
+  const bool copied = bucketed && rows_copied(B, A.num_decoders);
   using E = Op<T>;
   const uint32_t H = G.hidden, I = G.in_dim, C = G.out_dim, NL = G.layers, CP = out_pad(C);
   const size_t wbytes = (((size_t)H * I + (size_t)(NL - 1) * H * H + (size_t)H * CP) * sizeof(T) + 15) / 16 * 16;
@@ -467,8 +468,12 @@ __global__ void __launch_bounds__(128) k_decode_gen_fma(Assets A, GenWeights G, 
     uint32_t oi = 0;
     bool bad = false;
     if (valid) {
-      q = load_query(qs + i);
-      oi = perm ? __ldg(perm + i) : (uint32_t)i;
+      if (bucketed) {
+        bucket_row(B, copied, (uint32_t)i, oi, q);
+      } else {
+        q = load_query(qs + i);
+        oi = (uint32_t)i;
+      }
       bad = query_bad(A, q);
     }
     count_bad_warp(valid && bad, err);
@@ -613,7 +618,7 @@ cudaError_t launch_gen_fma_t(const Assets &A, const GenWeights &G, const Buckets
   const size_t blocks = (n + 127) / 128;
   size_t grid = (size_t)num_sms * occ * 4;
   if (grid > blocks) grid = blocks;
-  k_decode_gen_fma<T><<<(unsigned)grid, 128, 0, st>>>(A, G, B ? B->sorted : q, B ? B->perm : nullptr, n, out, err);
+  k_decode_gen_fma<T><<<(unsigned)grid, 128, 0, st>>>(A, G, q, B ? 1 : 0, B ? *B : Buckets{}, n, out, err);
   return cudaGetLastError();
 }
 

@@ -286,6 +286,7 @@ __global__ void __launch_bounds__(kTile) k_decode_mma(Assets A, WeightImages W, 
   uint16_t *stage = stage_all + warp * 32 * kFeatStride;
   const uint32_t D = A.num_decoders, C = W.out_dim;
   const uint32_t T = __ldg(B.meta);
+  const bool copied = rows_copied(B, D);
   const uint32_t t0 = (uint32_t)((unsigned long long)T * blockIdx.x / gridDim.x);
   const uint32_t t1 = (uint32_t)((unsigned long long)T * (blockIdx.x + 1) / gridDim.x);
   const SmemB W1{smem_u32(sw), I::s1}, W2{smem_u32(sw + I::off_w2), I::s2},
@@ -308,7 +309,7 @@ __global__ void __launch_bounds__(kTile) k_decode_mma(Assets A, WeightImages W, 
     bool bad = false;
     uint32_t oi = 0;
     if (valid) {
-      bucket_row(B, start + r, oi, q);
+      bucket_row(B, copied, start + r, oi, q);
       bad = dec == D || query_bad(A, q);
     }
     orig[r] = oi;

@@ -26,6 +26,7 @@ __global__ void __launch_bounds__(kTile) k_decode_fp32(Assets A, WeightImages W,
               *b3 = W3t + H * CP;
   const uint32_t D = A.num_decoders, C = W.out_dim;
   const uint32_t T = __ldg(B.meta);
+  const bool copied = rows_copied(B, D);
   const uint32_t t0 = (uint32_t)((unsigned long long)T * blockIdx.x / gridDim.x);
   const uint32_t t1 = (uint32_t)((unsigned long long)T * (blockIdx.x + 1) / gridDim.x);
   const size_t img_floats = f32_image_floats(H, C);
@@ -46,7 +47,7 @@ __global__ void __launch_bounds__(kTile) k_decode_fp32(Assets A, WeightImages W,
     uint32_t oi = 0;
     bool bad = false;
     if (valid) {
-      bucket_row(B, start + r, oi, q);
+      bucket_row(B, copied, start + r, oi, q);
       bad = dec == D || query_bad(A, q);
     }
     count_bad(valid && bad, err);

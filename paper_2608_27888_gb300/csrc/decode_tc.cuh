@@ -381,30 +381,60 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t pc = role % NC, pq = role / NC;  // serves consumer pc, tiles j = pq mod R
     auto tile_of = [&](uint32_t j) { return pc + NC * j; };
     uint32_t j = pq;
+    // Records read through perm (the caller's array, when the bucketing did
+    // not copy them): the output rows are loaded two tiles ahead and the
+    // query records one tile ahead, so a record never waits on its own perm
+    // load (DEEP; the H = 64 kernels that blend mips have no registers to
+    // spare for it).  Otherwise a row's output row and record are loaded
+    // together, one tile ahead.
+    constexpr bool DEEP = H > 64 || !TRI;
+    const bool copied = rows_copied(B, D);
+    const bool two_stage = DEEP && !copied;
     TileWalk walk;
     walk.ident_n = B.identity_n;
-    // this thread's row of the producer's tile jj: its output row (kNoRow
-    // past the tile's end) and query record.  A row of the bad bucket (set id
-    // out of range) needs no flag of its own: query_bad() rejects it.
+    // this thread's row of the producer's tile jj: its output row, or kNoRow
+    // past the tile's end.  A row of the bad bucket (set id out of range)
+    // needs no flag of its own: query_bad() rejects it.
     constexpr uint32_t kNoRow = 0xFFFFFFFFu;  // never a row: n <= 2^32 - 256
+    auto out_row = [&](uint32_t jj) -> uint32_t {
+      if (tile_of(jj) >= K) return kNoRow;
+      uint32_t d_, st_, len_;
+      walk.at(seg, tst, D, blockIdx.x + tile_of(jj) * grid, d_, st_, len_);
+      if ((uint32_t)row >= len_) return kNoRow;
+      return B.identity_n ? st_ + row : __ldg(B.perm + st_ + row);
+    };
+    // one stage: the row's output row and query record together
     auto fetch_row = [&](uint32_t jj, uint32_t &oi_, ntc_query &q_) {
       oi_ = kNoRow;
       if (tile_of(jj) >= K) return;
       uint32_t d_, st_, len_;
       walk.at(seg, tst, D, blockIdx.x + tile_of(jj) * grid, d_, st_, len_);
-      if ((uint32_t)row < len_) bucket_row(B, st_ + row, oi_, q_);
+      if ((uint32_t)row < len_) bucket_row(B, copied, st_ + row, oi_, q_);
     };
-    uint32_t oi;
+    uint32_t oi, noi = kNoRow;
     ntc_query q;
-    fetch_row(j, oi, q);
+    if (two_stage) {
+      oi = out_row(j);
+      noi = out_row(j + R);
+      if (oi != kNoRow) q = load_query(B.queries + oi);
+    } else {
+      fetch_row(j, oi, q);
+    }
     for (; tile_of(j) < K; j += R) {
       if (*abort_flag) break;
-      // the next tile's query record and output row go in flight early: before
-      // the taps, or (TRI, where registers are scarcer) once the first mip's
-      // taps are consumed
-      uint32_t noi;
+      // the next tile's query record (and, two-stage, the output row of the
+      // tile after it) go in flight early: before the taps, or (TRI, where
+      // registers are scarcer) once the first mip's taps are consumed
+      uint32_t nnoi = kNoRow;
       ntc_query nq;
-      auto prefetch = [&]() { fetch_row(j + R, noi, nq); };
+      auto prefetch = [&]() {
+        if (two_stage) {
+          if (noi != kNoRow) nq = load_query(B.queries + noi);
+          nnoi = out_row(j + 2 * R);
+        } else {
+          fetch_row(j + R, noi, nq);
+        }
+      };
       if (!TRI) prefetch();
       const bool valid = oi != kNoRow;
       const bool good = valid && !query_bad(A, q);
@@ -478,6 +508,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       if (lane == 0) mbar_arrive(full_bar(s));
       q = nq;
       oi = noi;
+      if (two_stage) noi = nnoi;
     }
   } else {
     // ------------------------------------------------------------ consumer

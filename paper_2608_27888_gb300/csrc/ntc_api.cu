@@ -46,6 +46,7 @@ struct ntc_ctx {
   size_t cap_n = 0, cap_counts = 0;
   uint32_t *d_perm = nullptr, *d_meta = nullptr, *d_counts = nullptr;
   ntc_query *d_sorted = nullptr;
+  void *d_dec = nullptr;  // decoder per query (1 or 2 bytes)
   // staging for ntc_decode_host, and its copy streams and chunk events
   size_t cap_host = 0;
   ntc_query *d_hq = nullptr;
@@ -176,6 +177,7 @@ void release(ntc_ctx *c) {
   cudaFree(c->d_meta);
   cudaFree(c->d_counts);
   cudaFree(c->d_sorted);
+  cudaFree(c->d_dec);
   cudaFree(c->d_hq);
   cudaFree(c->d_hout);
 }
@@ -183,9 +185,9 @@ void release(ntc_ctx *c) {
 size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 // Make sure the bucketing scratch holds n queries (stream-ordered
-// allocation): perm and the sorted query records [n], the per-chunk counts,
-// and the tile table with the totals and the ticket (zeroed once; the
-// bucketing leaves the ticket at zero).
+// allocation): perm, the sorted query records and the decoder ids [n], the
+// per-chunk counts, and the tile table with the totals, the ticket and the
+// divergence sum (zeroed once; the bucketing leaves them at zero).
 ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
   const size_t counts = bucket_count_words(c->D, n);
   if (!c->d_meta) {
@@ -203,11 +205,14 @@ ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
   if (n > c->cap_n) {
     if (c->d_perm) CK(cudaFreeAsync(c->d_perm, st), "scratch free");
     if (c->d_sorted) CK(cudaFreeAsync(c->d_sorted, st), "scratch free");
+    if (c->d_dec) CK(cudaFreeAsync(c->d_dec, st), "scratch free");
     c->d_perm = nullptr;
     c->d_sorted = nullptr;
+    c->d_dec = nullptr;
     c->cap_n = 0;
     CK(cudaMallocAsync((void **)&c->d_perm, n * 4, st), "scratch allocation");
     CK(cudaMallocAsync((void **)&c->d_sorted, n * sizeof(ntc_query), st), "scratch allocation");
+    CK(cudaMallocAsync(&c->d_dec, n * bucket_dec_bytes(c->D), st), "scratch allocation");
     c->cap_n = n;
   }
   return NTC_OK;
@@ -219,6 +224,7 @@ Scratch scratch_of(const ntc_ctx *c) {
   s.meta = c->d_meta;
   s.counts = c->d_counts;
   s.sorted = c->d_sorted;
+  s.dec = c->d_dec;
   return s;
 }
 
@@ -641,7 +647,8 @@ size_t ntc_max_tiles(const ntc_ctx *c, size_t n) {
 }
 
 ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *perm,
-                            uint32_t *counts, uint32_t *tiles, uint32_t *num_tiles, void *stream) {
+                            uint32_t *counts, uint32_t *tiles, uint32_t *num_tiles, uint32_t *divergence,
+                            void *stream) {
   ntc_status s = check_queries(c, q, n);
   if (s != NTC_OK) return s;
   if (n && !perm) return fail(NTC_ERR_INVALID_ARG, "null perm pointer");
@@ -651,6 +658,7 @@ ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *
   if (n == 0) {
     if (counts) CK(cudaMemsetAsync(counts, 0, (c->D + 1) * 4, st), "clear");
     if (num_tiles) CK(cudaMemsetAsync(num_tiles, 0, 4, st), "clear");
+    if (divergence) CK(cudaMemsetAsync(divergence, 0, 8, st), "clear");
     return NTC_OK;
   }
   s = ensure_scratch(c, n, st);
@@ -659,6 +667,8 @@ ntc_status ntc_debug_bucket(ntc_ctx *c, const ntc_query *q, size_t n, uint32_t *
   if (e == cudaSuccess) e = cudaMemcpyAsync(perm, c->d_perm, n * 4, cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && (counts || tiles || num_tiles))
     e = launch_tiles_export(c->d_meta, c->D, tiles, num_tiles, counts, ntc_max_tiles(c, n), st, &launches);
+  if (e == cudaSuccess && divergence)  // the words copied, divergence are adjacent
+    e = cudaMemcpyAsync(divergence, c->d_meta + meta_copied(c->D), 8, cudaMemcpyDeviceToDevice, st);
   c->launches += launches;
   if (e != cudaSuccess) return cuda_fail(e, "bucketing");
   return NTC_OK;

@@ -124,17 +124,30 @@ inline __host__ __device__ size_t gen_fma_image_bytes(uint32_t in_dim, uint32_t 
 }
 
 // Bucketing results on the device: row i of the bucketed order is query
-// perm[i] of the caller's array, whose record is sorted[i].  identity_n != 0:
+// perm[i] of the caller's array; when the bucketing copied the records
+// (meta[meta_copied(D)] != 0) that record is also sorted[i].  identity_n != 0:
 // one decoder and no sorting, row i is query i of `queries` (identity_n
 // queries); sorted, perm and meta are unused.
 struct Buckets {
   const ntc_query *queries;  // the caller's queries, in their own order
-  const ntc_query *sorted;   // the query records in (decoder, index) order
+  const ntc_query *sorted;   // the query records in (decoder, index) order, if copied
   const uint32_t *perm;      // original index of each row
-  const uint32_t *meta;      // [0] num_tiles, then seg_start[D+2], tile_start[D+2]
+  const uint32_t *meta;      // [0] num_tiles, seg_start[D+2], tile_start[D+2], copied, divergence
   uint32_t identity_n = 0;
 };
-inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2); }
+inline __host__ __device__ uint32_t meta_words(uint32_t D) { return 1 + 2 * (D + 2) + 2; }
+// meta[meta_copied(D)]: 1 when the bucketing wrote the query records in bucket
+// order (Buckets::sorted); 0 when the decode reads query perm[i] of the
+// caller's array
+inline __host__ __device__ uint32_t meta_copied(uint32_t D) { return 1 + 2 * (D + 2); }
+// meta[meta_divergence(D)]: the call's sum over groups of 32 consecutive
+// queries of (distinct decoders in the group - 1), Eq. 1's numerator
+inline __host__ __device__ uint32_t meta_divergence(uint32_t D) { return 2 + 2 * (D + 2); }
+// The bucketing copies the records when Eq. 1's score (the mean over 32-query
+// groups of distinct decoders - 1) exceeds this: the queries of one decoder
+// are then scattered over the array, and reading them through perm would
+// touch each sector once per decoder
+constexpr uint32_t kCopyAboveScore = 4;
 
 // ------------------------------------------------------------- device helpers
 
@@ -421,11 +434,16 @@ __device__ __forceinline__ ntc_query load_query(const ntc_query *q) {
   return out;
 }
 
-// Row `pos` of the bucketed order: its output row (original index) and query
-// (two independent loads).
-__device__ __forceinline__ void bucket_row(const Buckets &B, uint32_t pos, uint32_t &oi, ntc_query &q) {
+// Whether the query records of this launch's bucketing were copied (read
+// once the bucketing has finished; false without bucketing).
+__device__ __forceinline__ bool rows_copied(const Buckets &B, uint32_t D) {
+  return !B.identity_n && __ldg(B.meta + meta_copied(D)) != 0u;
+}
+
+// Row `pos` of the bucketed order: its output row (original index) and query.
+__device__ __forceinline__ void bucket_row(const Buckets &B, bool copied, uint32_t pos, uint32_t &oi, ntc_query &q) {
   oi = B.identity_n ? pos : __ldg(B.perm + pos);
-  q = load_query((B.identity_n ? B.queries : B.sorted) + pos);
+  q = load_query(copied ? B.sorted + pos : B.queries + oi);
 }
 
 // Tile t of the bucketed order: decoder, first sorted position and length.
@@ -474,8 +492,12 @@ struct Scratch {
   uint32_t *perm;     // [n]
   ntc_query *sorted;  // [n] the query records in bucket order
   uint32_t *meta;     // bucket_meta_words(D): the tile table, then the totals
-                      // [D+1] and a ticket (zero between calls)
+                      // [D+1], a ticket and the divergence sum (zero between
+                      // calls)
   uint32_t *counts;   // [bucket_count_words(D, n)] per-chunk counts, then offsets
+  void *dec;          // [n] decoder per query, bucket_dec_bytes(D) bytes each;
+                      // null: k_place reads the decoders from the records, which
+                      // it then always stages and copies (copy must be 1)
 };
 
 constexpr int kBucketThreads = 256;
@@ -484,9 +506,12 @@ constexpr int kBucketChunk = kBucketThreads * kBucketItems;
 size_t bucket_chunks(size_t n);
 size_t bucket_count_words(uint32_t D, size_t n);
 size_t bucket_meta_words(uint32_t D);
+size_t bucket_dec_bytes(uint32_t D);
 
+// copy: 0 = copy the records when Eq. 1's score exceeds kCopyAboveScore, 1 =
+// always copy them
 cudaError_t launch_bucket(const Assets &A, const ntc_query *q, size_t n, const Scratch &s, cudaStream_t st,
-                          int *launches);
+                          int *launches, int copy = 0);
 cudaError_t launch_tiles_export(const uint32_t *meta, uint32_t D, uint32_t *tiles, uint32_t *num_tiles,
                                 uint32_t *counts, size_t max_tiles, cudaStream_t st, int *launches);
 cudaError_t launch_decode_fp32(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,

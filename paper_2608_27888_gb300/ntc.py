@@ -81,7 +81,7 @@ def _load():
         "ntc_debug_taps": ([P, P, S, P, P, P, P], I),
         "ntc_debug_features": ([P, P, S, P, P], I),
         "ntc_debug_decode_rows": ([P, P, S, P, P, P], I),
-        "ntc_debug_bucket": ([P, P, S, P, P, P, P, P], I),
+        "ntc_debug_bucket": ([P, P, S, P, P, P, P, P, P], I),
         "ntc_max_tiles": ([P, S], S),
         "ntc_get_error_count": ([P, P], I),
         "ntc_reset_error_count": ([P], I),
@@ -141,8 +141,9 @@ def ntc_debug_decode_rows(ctx, d_queries, n, d_out, d_rows, stream):
     _check(_lib.ntc_debug_decode_rows(ctx, d_queries, n, d_out, d_rows, stream))
 
 
-def ntc_debug_bucket(ctx, d_queries, n, d_perm, d_counts, d_tiles, d_num_tiles, stream):
-    _check(_lib.ntc_debug_bucket(ctx, d_queries, n, d_perm, d_counts, d_tiles, d_num_tiles, stream))
+def ntc_debug_bucket(ctx, d_queries, n, d_perm, d_counts, d_tiles, d_num_tiles, d_divergence, stream):
+    _check(_lib.ntc_debug_bucket(ctx, d_queries, n, d_perm, d_counts, d_tiles, d_num_tiles, d_divergence,
+                                 stream))
 
 
 def ntc_max_tiles(ctx, n) -> int:
@@ -319,7 +320,9 @@ class Decoder:
         ntc_debug_decode_rows(self.ctx, _ptr(queries), n, _ptr(out), _ptr(rows), _stream(stream))
         return out, rows[:n].cpu().numpy().view(DEBUG_ROW).reshape(n)
 
-    def bucket(self, queries, stream=None):
+    def bucket(self, queries, stream=None, divergence=False):
+        """(perm, counts, tiles) of the bucketing; with divergence=True also
+        (copied, sum over 32-query groups of distinct decoders - 1)."""
         import torch
         n = queries.shape[0]
         dev = queries.device
@@ -328,9 +331,13 @@ class Decoder:
         counts = torch.empty((self.num_decoders + 1,), dtype=torch.int32, device=dev)
         tiles = torch.empty((mt, 3), dtype=torch.int32, device=dev)
         nt = torch.zeros((1,), dtype=torch.int32, device=dev)
-        ntc_debug_bucket(self.ctx, _ptr(queries), n, _ptr(perm), _ptr(counts), _ptr(tiles), _ptr(nt),
+        dv = torch.zeros((2,), dtype=torch.int32, device=dev)
+        ntc_debug_bucket(self.ctx, _ptr(queries), n, _ptr(perm), _ptr(counts), _ptr(tiles), _ptr(nt), _ptr(dv),
                          _stream(stream))
         k = int(nt.item())
+        if divergence:
+            c, s = dv.cpu().numpy().astype(np.uint32).tolist()
+            return perm[:n], counts, tiles[:k], (c, s)
         return perm[:n], counts, tiles[:k]
 
     def error_count(self) -> int:

@@ -287,13 +287,30 @@ _SEED = {"raster-256": 1, "uniform-4m": 2, "gbuffer-1080p": 3, "gbuffer-2160p": 
 WORKLOADS = tuple(_SEED)
 
 
-def named(name: str, size: str = "full", variant: str | None = None) -> Workload:
+def named(name: str, size: str = "full", variant: str | None = None, query_tag: int = 0) -> Workload:
     """One of WORKLOADS.  variant: the set->decoder grouping of gbuffer-1080p
     ("identity", "clustered4", "shared") or the decoder count of gbuffer-2160p
-    ("128", "16", "8", "1")."""
+    ("128", "16", "8", "1").  query_tag != 0 draws another query stream of the
+    same recipe over the same assets (one per rank of a multi-GPU run)."""
     if name not in _SEED:
         raise ValueError(f"unknown workload {name}")
     seed = BASE_SEED + _SEED[name]
+    if query_tag:
+        w = named(name, size, variant)
+        qseed = seed + 1000 * query_tag
+        if name == "raster-256":
+            return w  # a raster of texel centres has only one query stream
+        if name == "uniform-4m":
+            q = queries_uniform(qseed, len(w.queries), w.assets.num_sets)
+        else:
+            W_, H_, R, F = {("gbuffer-1080p", True): (1920, 1080, 200, 1), ("gbuffer-1080p", False): (240, 136, 40, 1),
+                            ("gbuffer-2160p", True): (3840, 2160, 800, 1), ("gbuffer-2160p", False): (320, 180, 120, 1),
+                            ("gbuffer-2160p-x4-trilinear", True): (3840, 2160, 2000, 4),
+                            ("gbuffer-2160p-x4-trilinear", False): (256, 128, 60, 2)}[(name, size == "full")]
+            tri = name == "gbuffer-2160p-x4-trilinear"
+            q = queries_gbuffer(qseed, W_, H_, R, w.assets.num_sets, w.info["T"], lod_mode=1 if tri else 0,
+                                lod_max=3.0, frames=F)
+        return Workload(f"{w.name}-q{query_tag}", w.assets, q, dict(w.info, query_tag=query_tag))
     full = size == "full"
     if name == "raster-256":
         T = 256 if full else 64

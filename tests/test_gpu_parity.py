@@ -489,3 +489,51 @@ def test_every_tile_switches_decoder(hidden, out_dim, mips):
     assert dec.error_count() == 0
     dec.close()
     torch.cuda.empty_cache()
+
+
+# ------------------------------- divergence-aware bucketing (Sec. 2, Eq. 1)
+
+def _eq1_sum(q, a):
+    ids = oracle.decoder_ids(q["set_id"], a.set_to_decoder, a.num_decoders)
+    return int((oracle.divergence_map(ids, 32) - 1).sum())
+
+
+@pytest.mark.parametrize("name,variant", SMALL)
+def test_divergence_score_and_copy_decision_match_the_oracle(name, variant):
+    """k_count sums Eq. 1's |D_w - 1| over the 32-query groups; the records are
+    copied in bucket order exactly when that mean exceeds 4."""
+    w = small(name, variant)
+    if w.assets.num_decoders == 1 and name != "uniform-4m":
+        pytest.skip("one decoder: nothing is bucketed")
+    _, _, _, (copied, s) = decoder(name, variant, "fp16").bucket(dq(w.queries), divergence=True)
+    ref = _eq1_sum(w.queries, w.assets)
+    groups = (len(w.queries) + 31) // 32
+    assert s == ref
+    assert copied == int(ref > 4 * groups)
+
+
+@pytest.mark.parametrize("d", [1, 2, 4, 5, 6, 8, 16, 32])
+def test_divergence_sweep_decodes_on_both_sides_of_the_copy_threshold(d):
+    """Exactly d distinct decoders in every warp: d <= 5 reads the queries
+    through perm, d >= 6 reads copied records (Eq. 1 score d - 1 against 4).
+    Outputs are compared with the oracle, the perm with its stable sort."""
+    wl = W.sweep(d, 256, "small")
+    a, q = wl.assets, wl.queries
+    dec = ntc().Decoder(a, "fp16")
+    perm, _, _, (copied, s) = dec.bucket(dq(q), divergence=True)
+    groups = (len(q) + 31) // 32
+    assert s == _eq1_sum(q, a) == (d - 1) * groups
+    assert copied == int(d - 1 > 4)
+    p, _, _, _ = oracle.bucket(q["set_id"], a.set_to_decoder, a.num_decoders)
+    assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
+    ref, _ = oracle.decode(a, q)
+    for prec in ("fp16", "bf16"):
+        d2 = dec if prec == "fp16" else ntc().Decoder(a, prec)
+        check_tc(d2.decode(dq(q)).cpu().numpy(), ref, f"sweep d={d} {prec}")
+        if d2 is not dec:
+            d2.close()
+    fp = ntc().Decoder(a, "fp32")
+    assert np.abs(fp.decode(dq(q)).cpu().numpy() - ref).max() <= FP32_TOL
+    assert np.abs(dec.decode(dq(q), mode="bucketed_mma").cpu().numpy() - ref).max() <= TC_MAX
+    fp.close()
+    dec.close()
