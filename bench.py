@@ -83,8 +83,13 @@ def parse():
     p.add_argument("--no-maps", action="store_true", help="skip the Table 2 groupings of a 586-set workload")
     p.add_argument("--no-variants", action="store_true", help="skip Sec. 4's decoder shape")
     p.add_argument("--variants", action="store_true", help="also time every A x B size of Sec. 4's MLP ablation")
-    p.add_argument("--small", action="store_true", help="the small size of the timed workload (profiling captures)")
-    return p.parse_args()
+    p.add_argument("--small", action="store_true", help="the small size of the timed workload")
+    p.add_argument("--medium", action="store_true",
+                   help="the profiling size of gbuffer-2160p-x4-trilinear: one frame over 32 sets (a few GB)")
+    a = p.parse_args()
+    a.size = "small" if a.small else ("medium" if a.medium else "full")
+    a.small = a.small or a.medium  # every reduced size skips the other legs
+    return a
 
 
 # ------------------------------------------------------------------ clocks
@@ -239,14 +244,15 @@ def shape_costs(a, q):
     return bpq, flops, w_bytes
 
 
-def workload(name: str, small: bool, rank: int, variant=None):
+def workload(name: str, small, rank: int, variant=None):
     """The benchmark batch of one rank: the same assets on every rank, a
     rank-specific query stream of the same recipe (queries are sharded, assets
-    replicated)."""
+    replicated).  small: True / "small", "medium", or False / "full"."""
     from paper_2608_27888_gb300 import workloads as W
+    size = small if isinstance(small, str) else ("small" if small else "full")
     if name == "paper-decoder":
-        return W.paper_decoder("small" if small else "full")
-    return W.named(name, "small" if small else "full", variant, query_tag=rank)
+        return W.paper_decoder("small" if size != "full" else "full")
+    return W.named(name, size, variant, query_tag=rank if size != "medium" else 0)
 
 
 def aggregate(n_per_rank: int, ms_local: float, dist=None):
@@ -283,7 +289,7 @@ def run_reference(args, ws, rank):
     if rank != 0:
         return
     import oracle
-    w = workload(args.workload, args.small, 0, args.variant)
+    w = workload(args.workload, args.size, 0, args.variant)
     q, stride = cpu_sample(w.queries)
     sample = len(q)
     cores = os.cpu_count() or 1
@@ -325,7 +331,7 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     from paper_2608_27888_gb300 import ntc
 
-    w = workload(args.workload, args.small, rank, args.variant)
+    w = workload(args.workload, args.size, rank, args.variant)
     n = len(w.queries)
     C = w.assets.out_dim
     dec = ntc.Decoder(w.assets, args.precision)

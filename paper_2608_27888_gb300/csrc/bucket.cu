@@ -26,6 +26,8 @@
 // contiguous records.  Equal decoders within a warp are found with one ballot
 // per bit of the decoder id.  The permutation is exactly std::stable_sort of
 // the indices by decoder.
+#include <algorithm>
+
 #include "ntc_internal.cuh"
 
 namespace ntc {
@@ -62,8 +64,10 @@ struct MapLookup {
 __device__ __forceinline__ int key_bits(uint32_t D) { return 32 - __clz(D + 1); }
 
 // The lanes of the warp whose key equals this lane's: one ballot per key bit
-// (each lane keeps the lanes that agree with it on that bit).
+// (each lane keeps the lanes that agree with it on that bit), after a check
+// for the common case of a G-buffer, one key in the whole warp.
 __device__ __forceinline__ uint32_t match_key(uint32_t key, int nbits) {
+  if (__all_sync(0xFFFFFFFFu, key == __shfl_sync(0xFFFFFFFFu, key, 0))) return 0xFFFFFFFFu;
   uint32_t m = 0xFFFFFFFFu;
   for (int b = 0; b < nbits; ++b) {
     const bool bit = (key >> b) & 1u;
@@ -259,16 +263,18 @@ __device__ __forceinline__ void cp_async16(void *smem_dst, const void *src) {
 
 // FROM_Q: the decoders come from the staged records (always copied);
 // otherwise from k_count's decoder array, and the records are staged only
-// when k_scan chose to copy them.
+// when k_scan chose to copy them.  A resident grid: each CTA takes chunks
+// blockIdx.x, + gridDim.x, ... and loads the next chunk's decoders and chunk
+// offsets while it ranks and places the current one.
 template <typename DecT, bool FROM_Q>
 __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc_query *q, const DecT *dec_in,
-                                                          size_t n, uint32_t chunks, const uint32_t *offs,
-                                                          const uint32_t *meta, uint32_t *perm,
-                                                          ntc_query *sorted) {
+                                                             size_t n, uint32_t chunks, const uint32_t *offs,
+                                                             const uint32_t *meta, uint32_t *perm,
+                                                             ntc_query *sorted) {
   // shared memory: the chunk's records [chunk] (16 B), the chunk-local index
   // and decoder of every sorted slot [chunk] (u16 each), per-warp counters
-  // [kWarps][D+2], and per decoder the chunk-local run start and the global
-  // base [D+2] each
+  // [kWarps][D+2], and per decoder the chunk-local run start, the global base
+  // and the segment start [D+2] each
   extern __shared__ uint4 srec[];
   uint16_t *sidx = reinterpret_cast<uint16_t *>(srec + kBucketChunk);
   uint16_t *sdec = sidx + kBucketChunk;
@@ -276,79 +282,130 @@ __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc
   const uint32_t D = A.num_decoders, DW = D + 2;
   uint32_t *loff = cnt + kWarps * DW;
   uint32_t *gbase = loff + DW;
+  uint32_t *sseg = gbase + DW;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const size_t cbase = (size_t)blockIdx.x * kBucketChunk;
-  const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
-  auto stage_records = [&]() {
+  const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in a chunk
+  const uint32_t lt = (1u << lane) - 1u;
+  const bool own_offset = D + 1 <= (uint32_t)blockDim.x;       // thread d prefetches decoder d's offset
+  auto stage_records = [&](size_t cbase, uint32_t valid) {
     for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) cp_async16(srec + i, q + cbase + i);
     asm volatile("cp.async.commit_group;\n" ::: "memory");
   };
-  if (FROM_Q) stage_records();  // the caller's queries: no dependence on k_scan
+  auto load_decoders = [&](uint32_t c, uint32_t (&d)[kBucketItems]) {
+    const size_t cbase = (size_t)c * kBucketChunk;
+    const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+#pragma unroll
+    for (int it = 0; it < kBucketItems; ++it) {
+      const uint32_t j = wbase + it * 32 + lane;
+      d[it] = j < valid ? (uint32_t)__ldcg(dec_in + cbase + j) : D + 1;
+    }
+  };
+  uint32_t c = blockIdx.x;
+  if (FROM_Q && c < chunks)  // the caller's queries: no dependence on k_scan
+    stage_records((size_t)c * kBucketChunk, (uint32_t)min((size_t)kBucketChunk, n - (size_t)c * kBucketChunk));
   for (uint32_t i = threadIdx.x; i < kWarps * DW; i += blockDim.x) cnt[i] = 0;
   const MapLookup lookup(A);
   const int nbits = key_bits(D);
   pdl_wait();  // k_scan's chunk offsets, segment starts and decision (and k_count's decoders)
   const bool copy = FROM_Q || __ldcg(meta + meta_copied(D)) != 0u;
-  if (!FROM_Q && copy) stage_records();
-  if (FROM_Q) asm volatile("cp.async.wait_all;\n" ::: "memory");
-  __syncthreads();
-  const uint32_t wbase = (uint32_t)warp * (kBucketItems * 32);  // this warp's run in the chunk
-  uint32_t *my = cnt + warp * DW;
-  // rank of each query among the equal decoders of this warp's run, in order
-  uint32_t dec[kBucketItems], rank[kBucketItems];
-  const uint32_t lt = (1u << lane) - 1u;
-#pragma unroll
-  for (int it = 0; it < kBucketItems; ++it) {
-    const uint32_t j = wbase + it * 32 + lane;
-    uint32_t d;
+  for (uint32_t d = threadIdx.x; d <= D; d += blockDim.x) sseg[d] = __ldcg(meta + 1 + d);
+  uint32_t next_dec[kBucketItems], next_off = 0;
+  if (!FROM_Q && c < chunks) load_decoders(c, next_dec);
+  if (own_offset && threadIdx.x <= D && c < chunks) next_off = __ldcg(offs + (size_t)threadIdx.x * chunks + c);
+  for (; c < chunks; c += gridDim.x) {
+    const size_t cbase = (size_t)c * kBucketChunk;
+    const uint32_t valid = (uint32_t)min((size_t)kBucketChunk, n - cbase);
+    const bool last = c + gridDim.x >= chunks;
+    if (!FROM_Q && copy) stage_records(cbase, valid);
+    uint32_t dec[kBucketItems];
+    const uint32_t off = next_off;
     if (FROM_Q) {
-      const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
-      d = j < valid ? dl : D + 1;
+      asm volatile("cp.async.wait_all;\n" ::: "memory");
+      __syncthreads();
+#pragma unroll
+      for (int it = 0; it < kBucketItems; ++it) {
+        const uint32_t j = wbase + it * 32 + lane;
+        const uint32_t dl = lookup(A, j < valid ? srec[j].x : 0u);  // every lane: the lookup shuffles
+        dec[it] = j < valid ? dl : D + 1;
+      }
     } else {
-      d = j < valid ? (uint32_t)__ldcg(dec_in + cbase + j) : D + 1;
-    }
-    const uint32_t m = match_key(d, nbits);
-    dec[it] = d;
-    rank[it] = my[d] + __popc(m & lt);
-    __syncwarp();
-    if (lane == __ffs(m) - 1) my[d] += __popc(m);
-    __syncwarp();
-  }
-  __syncthreads();
-  // per decoder: warp prefix (in place), the chunk's count and its global base
-  const uint32_t *seg = meta + 1;
-  for (uint32_t d = threadIdx.x; d <= D; d += blockDim.x) {
-    uint32_t run = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      const uint32_t x = cnt[w * DW + d];
-      cnt[w * DW + d] = run;
-      run += x;
+      for (int it = 0; it < kBucketItems; ++it) dec[it] = next_dec[it];
+      if (!last) load_decoders(c + gridDim.x, next_dec);  // in flight while this chunk is placed
     }
-    loff[d] = run;
-    gbase[d] = __ldcg(seg + d) + __ldcg(offs + (size_t)d * chunks + blockIdx.x);
-  }
-  __syncthreads();
-  block_scan(loff, D + 1);  // exclusive scan of the chunk's counts over decoders
-  // stable local sort of (local index, decoder) pairs
+    if (own_offset && threadIdx.x <= D && !last)
+      next_off = __ldcg(offs + (size_t)threadIdx.x * chunks + c + gridDim.x);
+    // rank of each query among the equal decoders of this warp's run, in order
+    uint32_t *my = cnt + warp * DW;
+    uint32_t rank[kBucketItems];
 #pragma unroll
-  for (int it = 0; it < kBucketItems; ++it) {
-    const uint32_t d = dec[it];
-    if (d > D) continue;
-    const uint32_t lp = loff[d] + cnt[warp * DW + d] + rank[it];
-    sidx[lp] = (uint16_t)(wbase + it * 32 + lane);
-    sdec[lp] = (uint16_t)d;
-  }
-  if (!FROM_Q && copy) asm volatile("cp.async.wait_all;\n" ::: "memory");
-  __syncthreads();
-  pdl_trigger();  // the decode may launch (it waits for this grid before reading)
-  // coalesced copy-out: consecutive slots of one decoder go to consecutive
-  // positions of that decoder's segment
-  for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
-    const uint32_t d = sdec[i], j = sidx[i];
-    const uint32_t pos = gbase[d] + (i - loff[d]);
-    perm[pos] = (uint32_t)(cbase + j);
-    if (copy) reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
+    for (int it = 0; it < kBucketItems; ++it) {
+      const uint32_t d = dec[it];
+      const uint32_t m = match_key(d, nbits);
+      rank[it] = my[d] + __popc(m & lt);
+      __syncwarp();
+      if (lane == __ffs(m) - 1) my[d] += __popc(m);
+      __syncwarp();
+    }
+    __syncthreads();
+    // per decoder: warp prefix (in place), the chunk's count and its global base
+    for (uint32_t d = threadIdx.x; d <= D; d += blockDim.x) {
+      uint32_t run = 0;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        const uint32_t x = cnt[w * DW + d];
+        cnt[w * DW + d] = run;
+        run += x;
+      }
+      loff[d] = run;
+      gbase[d] = sseg[d] + (own_offset ? off : __ldcg(offs + (size_t)d * chunks + c));
+    }
+    __syncthreads();
+    if (!copy) {
+      // only perm: each query's place is its decoder's base + its warp's
+      // prefix + its rank, and the equal decoders of a 32-query group get
+      // consecutive places, so the stores of a group of one decoder (most of
+      // a G-buffer's) coalesce without a local sort
+      if (last) pdl_trigger();  // the decode may launch (it waits for this grid before reading)
+#pragma unroll
+      for (int it = 0; it < kBucketItems; ++it) {
+        const uint32_t d = dec[it];
+        if (d <= D) perm[gbase[d] + cnt[warp * DW + d] + rank[it]] = (uint32_t)(cbase + wbase + it * 32 + lane);
+      }
+      __syncthreads();  // cnt and gbase are reused by the next chunk
+      for (uint32_t i = threadIdx.x; i < kWarps * DW; i += blockDim.x) cnt[i] = 0;
+      __syncthreads();
+      continue;
+    }
+    block_scan(loff, D + 1);  // exclusive scan of the chunk's counts over decoders
+    // stable local sort of (local index, decoder) pairs
+#pragma unroll
+    for (int it = 0; it < kBucketItems; ++it) {
+      const uint32_t d = dec[it];
+      if (d > D) continue;
+      const uint32_t lp = loff[d] + cnt[warp * DW + d] + rank[it];
+      sidx[lp] = (uint16_t)(wbase + it * 32 + lane);
+      sdec[lp] = (uint16_t)d;
+    }
+    if (!FROM_Q) asm volatile("cp.async.wait_all;\n" ::: "memory");
+    __syncthreads();
+    if (last) pdl_trigger();  // the decode may launch (it waits for this grid before reading)
+    // the counters are free again: cleared for the next chunk while this one
+    // is copied out
+    for (uint32_t i = threadIdx.x; i < kWarps * DW; i += blockDim.x) cnt[i] = 0;
+    // coalesced copy-out of perm and the records: consecutive slots of one
+    // decoder go to consecutive positions of that decoder's segment
+    for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
+      const uint32_t d = sdec[i], j = sidx[i];
+      const uint32_t pos = gbase[d] + (i - loff[d]);
+      perm[pos] = (uint32_t)(cbase + j);
+      reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
+    }
+    __syncthreads();  // srec, sidx, sdec, loff and gbase are reused by the next chunk
+    if (FROM_Q && !last) {
+      const size_t nb = (size_t)(c + gridDim.x) * kBucketChunk;
+      stage_records(nb, (uint32_t)min((size_t)kBucketChunk, n - nb));
+    }
   }
 }
 
@@ -382,8 +439,18 @@ cudaError_t launch_bucket_t(const Assets &A, const ntc_query *q, size_t n, const
   const uint32_t chunks = (uint32_t)bucket_chunks(n);
   const uint32_t D = A.num_decoders, DW = D + 2;
   const size_t smem_count = (size_t)kWarps * DW * sizeof(uint32_t);
-  const size_t smem_place = (size_t)kBucketChunk * (16 + 2 + 2) + (size_t)(kWarps + 2) * DW * sizeof(uint32_t);
+  const size_t smem_place = (size_t)kBucketChunk * (16 + 2 + 2) + (size_t)(kWarps + 3) * DW * sizeof(uint32_t);
   const bool from_q = s.dec == nullptr;
+  // k_place runs a resident grid: at most 5 CTAs per SM (its register
+  // bound), fewer when its shared memory (which grows with D) allows fewer
+  int dev = 0, sms = 1, smem_sm = 233472;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+  size_t per_sm = (size_t)smem_sm / (smem_place + 2048);
+  if (per_sm > 5) per_sm = 5;
+  if (per_sm < 1) per_sm = 1;
+  const uint32_t place_grid = (uint32_t)std::min<size_t>(chunks, (size_t)sms * per_sm);
   static PerDevice attrs;
   cudaError_t e = attrs.once([]() {
     // as much dynamic shared memory as the device allows a block: the
@@ -412,11 +479,11 @@ cudaError_t launch_bucket_t(const Assets &A, const ntc_query *q, size_t n, const
   if (e == cudaSuccess) e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, s.meta, copy);
   if (e == cudaSuccess) {
     if (from_q)
-      e = launch_pdl(k_place<DecT, true>, dim3(chunks), dim3(kBucketThreads), smem_place, st, A, q,
+      e = launch_pdl(k_place<DecT, true>, dim3(place_grid), dim3(kBucketThreads), smem_place, st, A, q,
                      (const DecT *)nullptr, n, chunks, (const uint32_t *)s.counts, (const uint32_t *)s.meta,
                      s.perm, s.sorted);
     else
-      e = launch_pdl(k_place<DecT, false>, dim3(chunks), dim3(kBucketThreads), smem_place, st, A, q,
+      e = launch_pdl(k_place<DecT, false>, dim3(place_grid), dim3(kBucketThreads), smem_place, st, A, q,
                      (const DecT *)dec, n, chunks, (const uint32_t *)s.counts, (const uint32_t *)s.meta, s.perm,
                      s.sorted);
   }

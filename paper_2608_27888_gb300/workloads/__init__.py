@@ -280,6 +280,8 @@ def make_assets(seed, num_sets, T, num_mips, num_decoders, set_to_decoder, hidde
 #                               16->128->128->9 decoders, continuous lods;
 # small = the same recipes shrunk so the oracle finishes in seconds, still
 #         spanning many 128-query tiles and a ragged tail.
+# medium (gbuffer-2160p-x4-trilinear only) = one frame over 32 of the sets,
+#         about 3 GB on the device: the size of a full ncu capture.
 
 # seed offset of each named workload (the generated inputs depend on it)
 _SEED = {"raster-256": 1, "uniform-4m": 2, "gbuffer-1080p": 3, "gbuffer-2160p": 4,
@@ -340,8 +342,11 @@ def named(name: str, size: str = "full", variant: str | None = None, query_tag: 
         a = make_assets(seed, S, T, 4, D, m, out_dim=9)
         q = queries_gbuffer(seed, W, H, R, S, T, lod_mode=0)
         return Workload(f"{name}-{size}-{D}", a, q, {"T": T, "maps": f"random{D}"})
-    S, T = (512, 2048) if full else (24, 128)
-    W, H, R, F = (3840, 2160, 2000, 4) if full else (256, 128, 60, 2)
+    if size == "medium":  # the profiling size: same grids, decoders and screen, 32 sets, one frame
+        S, T, (W, H, R, F) = 32, 2048, (3840, 2160, 2000, 1)
+    else:
+        S, T = (512, 2048) if full else (24, 128)
+        W, H, R, F = (3840, 2160, 2000, 4) if full else (256, 128, 60, 2)
     D = 8
     a = make_assets(seed, S, T, 4, D, map_random_partition(seed, S, D), hidden=128, out_dim=9)
     q = queries_gbuffer(seed, W, H, R, S, T, lod_mode=1, lod_max=3.0, frames=F)
