@@ -251,14 +251,21 @@ struct TmSmem {
 // zeros elsewhere: the A operand of every layer's bias K step (the decoder image
 // keeps each layer's bias as the first row of an extra 16-row K block); then
 // each consumer's own 16-column accumulator for the output layer, so that the
-// next tile's layer 1 can run in the hidden accumulator meanwhile.
+// next tile's layer 1 can run in the hidden accumulator meanwhile.  With
+// split_out<H>() the output layer's K steps are split over two accumulators
+// (each consumer's second one follows all the first ones).
+template <int H>
+__host__ __device__ constexpr bool split_out() {
+  return H >= 128;
+}
+
 template <int H, int NC, int SC>
 struct TmCols {
   static constexpr uint32_t HID = NC * H;
   static constexpr uint32_t STG = HID + NC * (H / 2);
   static constexpr uint32_t ONES = STG + NC * SC * 8;
   static constexpr uint32_t OUT = (ONES + 8 + 15) / 16 * 16;
-  static constexpr uint32_t used = OUT + NC * 16;
+  static constexpr uint32_t used = OUT + NC * 16 * (split_out<H>() ? 2 : 1);
   static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
   static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
   static __device__ __forceinline__ uint32_t acc(uint32_t c) { return c * H; }
@@ -266,6 +273,7 @@ struct TmCols {
   // layer-1 A operand of stage s (= consumer * SC + st)
   static __device__ __forceinline__ uint32_t a1(uint32_t s) { return STG + 8 * s; }
   static __device__ __forceinline__ uint32_t out(uint32_t c) { return OUT + 16 * c; }
+  static __device__ __forceinline__ uint32_t out2(uint32_t c) { return OUT + 16 * (NC + c); }
 };
 
 // Warp-specialised gather-decode with tensor-memory operands.
@@ -300,6 +308,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
                 unsigned int *status, int vec_out, ntc_debug_row *dbg) {
   static_assert(NP % NC == 0 && SC % (NP / NC) == 0, "each ring stage needs one producer");
   constexpr int R = NP / NC;  // producers per consumer
+  constexpr bool SPLIT = split_out<H>();
   constexpr int S = NC * SC;
   using L = TcLayout<H>;
   using M = TmSmem<H, NC, SC>;
@@ -334,7 +343,8 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       mbar_init(full_bar(i), 4);   // one arrival per producer warp
       mbar_init(empty_bar(i), 1);  // the consumer's layer-1 commit
     }
-    for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), 1);
+    // the output barriers (the last NC) take one commit per output-layer issuer
+    for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), i >= 2 * S + 2 * NC && split_out<H>() ? 2 : 1);
     *abort_flag = 0;
     for (int i = 0; i < 2 * NC; ++i) stop_flag[i] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
@@ -519,6 +529,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t tH = tmem_base + TC::hid(c);  // hidden A operand
     const uint32_t tOnes = tmem_base + TC::ONES; // the bias K step's A operand
     const uint32_t tO = tmem_base + TC::out(c);  // the output layer's accumulator
+    const uint32_t tO2 = tmem_base + TC::out2(c);  // its second half-K accumulator (SPLIT)
     const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
     const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
     const uint32_t obar = saddr(bars + 2 * S + 2 * NC + c);  // the output layer's completion
@@ -598,13 +609,81 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         }
       }
     };
+    // the sigmoid epilogue of one tile: its output accumulator(s) -> out[eoi]
+    auto out_rows = [&](uint32_t eoi, bool egood) {
+      uint32_t o[16];
+      tmem_ld16(tO + lanes, o);
+      if constexpr (SPLIT) {
+        uint32_t o2[16];
+        tmem_ld16(tO2 + lanes, o2);
+        tmem_wait_ld();
+#pragma unroll
+        for (int cc = 0; cc < 16; ++cc) o[cc] = __float_as_uint(__uint_as_float(o[cc]) + __uint_as_float(o2[cc]));
+      } else {
+        tmem_wait_ld();
+      }
+      fence_before();
+      if (egood) {
+        // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
+        float y[CP];
+#pragma unroll
+        for (int cc = 0; cc < CP; ++cc) {
+          float th;
+          asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
+          y[cc] = fmaf(0.5f, th, 0.5f);
+        }
+        float *dst = out + (size_t)eoi * C;
+        if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
+          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]),
+                       "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
+                       : "memory");
+        } else {
+#pragma unroll
+          for (int cc = 0; cc < CP; ++cc)
+            if (cc < (int)C) dst[cc] = y[cc];
+        }
+      }
+    };
     uint32_t k = c, dec = D, oi = 0;
     bool good = false, stop = false;
     if (k < K) begin(k, dec, oi, good, stop);
-    while (k < K) {
-      if (dec < D) {
-#pragma unroll 1
-        for (int layer = 0; layer < 2; ++layer) {
+    if constexpr (SPLIT) {
+      // Tile k: layer 1 (issued by begin) -> convert -> layer 2, issued by warp
+      // 3 while warps 0-2 write the previous tile's outputs (warp 3 its rows
+      // after the issue) -> convert -> the output layer, its K steps split
+      // between warps 1 and 2 and two accumulators -> begin(k + NC).  The
+      // outputs of tile k wait in tO / tO2 until tile k + NC's layer 2 runs.
+      // Layer 1 of a tile may not convert before the previous output layer
+      // has read the hidden operand, so that is waited for first.
+      bool epi = false;  // a tile's outputs wait in tO / tO2
+      uint32_t poi = 0;
+      bool pgood = false;
+      while (k < K) {
+        if (dec < D) {
+          wait_bar(mbar, ph);
+          ph ^= 1;
+          if (out_pending) {
+            wait_bar(obar, oph);
+            oph ^= 1;
+            out_pending = false;
+          }
+          wg_bar(wgid);
+          fence_after();
+          hidden();
+          fence_before();
+          wg_bar(wgid);
+          if (row == 96) {
+            fence_after();
+#pragma unroll
+            for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
+            umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
+            umma_commit(mbar);
+          }
+          if (epi) {
+            __syncwarp();  // warp 3 reconverges after its issue; tcgen05.ld is warp-wide
+            out_rows(poi, pgood);
+            epi = false;
+          }
           wait_bar(mbar, ph);
           ph ^= 1;
           wg_bar(wgid);
@@ -612,70 +691,113 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
           hidden();
           fence_before();
           wg_bar(wgid);
-          if (row == 0) {
+          if (row == 32) {  // bias and the first half of the K steps
             fence_after();
-            if (layer == 0) {
+            umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 0);
 #pragma unroll
-              for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
-              umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
-              umma_commit(mbar);
-            } else {
+            for (uint32_t kq = 0; kq < H / 32; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, 1);
+            umma_commit(obar);
+          } else if (row == 64) {  // the second half
+            fence_after();
 #pragma unroll
-              for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, kq);
-              umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 1);  // + bias
-              umma_commit(obar);
-            }
+            for (uint32_t kq = H / 32; kq < H / 16; ++kq)
+              umma_ta(tO2, tH + 8 * kq, dW3 + 16 * kq, id_out, kq > H / 32);
+            umma_commit(obar);
           }
+          out_pending = true;
+          epi = true;
+          poi = oi;
+          pgood = good;
+        } else if (epi) {  // a tile with nothing to multiply: write the waiting outputs now
+          if (out_pending) {
+            wait_bar(obar, oph);
+            oph ^= 1;
+            out_pending = false;
+          }
+          wg_bar(wgid);
+          fence_after();
+          out_rows(poi, pgood);
+          epi = false;
         }
-        out_pending = true;
+        const uint32_t kn = k + NC;
+        uint32_t ndec = D, noi = 0;
+        bool ngood = false, nstop = false;
+        if (kn < K && !stop) begin(kn, ndec, noi, ngood, nstop);
+        if (stop || nstop) {  // every warp of this warpgroup read the same flags
+          if (nstop && ndec < D) wait_bar(mbar, ph);  // issued MMAs end before TMEM is released
+          if (out_pending) wait_bar(obar, oph);
+          epi = false;
+          break;
+        }
+        k = kn;
+        dec = ndec;
+        oi = noi;
+        good = ngood;
       }
-      // the next tile's layer 1 runs while this tile's output layer finishes
-      // and its outputs are written (the hidden accumulator has been read)
-      const uint32_t kn = k + NC;
-      uint32_t ndec = D, noi = 0;
-      bool ngood = false, nstop = false;
-      if (kn < K && !stop) begin(kn, ndec, noi, ngood, nstop);
-      if (dec < D) {
-        uint32_t o[16];
-        if (out_pending) {  // not already waited for by begin()
+      if (epi) {  // the last tile's outputs
+        if (out_pending) {
           wait_bar(obar, oph);
           oph ^= 1;
           out_pending = false;
         }
         wg_bar(wgid);
         fence_after();
-        tmem_ld16(tO + lanes, o);
-        tmem_wait_ld();
-        fence_before();
-        if (good) {
-          // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
-          float y[CP];
+        out_rows(poi, pgood);
+      }
+    } else {
+      while (k < K) {
+        if (dec < D) {
+#pragma unroll 1
+          for (int layer = 0; layer < 2; ++layer) {
+            wait_bar(mbar, ph);
+            ph ^= 1;
+            wg_bar(wgid);
+            fence_after();
+            hidden();
+            fence_before();
+            wg_bar(wgid);
+            if (row == 0) {
+              fence_after();
+              if (layer == 0) {
 #pragma unroll
-          for (int cc = 0; cc < CP; ++cc) {
-            float th;
-            asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
-            y[cc] = fmaf(0.5f, th, 0.5f);
-          }
-          float *dst = out + (size_t)oi * C;
-          if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
-            asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]),
-                         "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
-                         : "memory");
-          } else {
+                for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
+                umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
+                umma_commit(mbar);
+              } else {
 #pragma unroll
-            for (int cc = 0; cc < CP; ++cc)
-              if (cc < (int)C) dst[cc] = y[cc];
+                for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, kq);
+                umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 1);  // + bias
+                umma_commit(obar);
+              }
+            }
           }
+          out_pending = true;
         }
+        // the next tile's layer 1 runs while this tile's output layer finishes
+        // and its outputs are written (the hidden accumulator has been read)
+        const uint32_t kn = k + NC;
+        uint32_t ndec = D, noi = 0;
+        bool ngood = false, nstop = false;
+        if (kn < K && !stop) begin(kn, ndec, noi, ngood, nstop);
+        if (dec < D) {
+          if (out_pending) {  // not already waited for by begin()
+            wait_bar(obar, oph);
+            oph ^= 1;
+            out_pending = false;
+          }
+          wg_bar(wgid);
+          fence_after();
+          out_rows(oi, good);
+        }
+        if (stop || nstop) {  // every warp of this warpgroup read the same flags
+          if (nstop && ndec < D) wait_bar(mbar, ph);  // the issued layer 1 ends before TMEM is released
+          break;
+        }
+        k = kn;
+        dec = ndec;
+        oi = noi;
+        good = ngood;
       }
-      if (stop || nstop) {  // every warp of this warpgroup read the same flags
-        if (nstop && ndec < D) wait_bar(mbar, ph);  // the issued layer 1 ends before TMEM is released
-        break;
-      }
-      k = kn;
-      dec = ndec;
-      oi = noi;
-      good = ngood;
     }
   }
   fence_before();
