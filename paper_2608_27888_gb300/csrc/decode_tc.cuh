@@ -225,6 +225,41 @@ constexpr uint32_t kSmemGrids = 1024;      // staged when S * 2 * M <= this
 // (the B operands) and bookkeeping live in shared memory; every A operand and
 // accumulator lives in tensor memory, so most of the SM's L1/shared array stays
 // L1, which holds the in-flight latent gathers.
+// Whether each consumer has MMA-issuing warps of its own.  One thread issues
+// a tcgen05.mma about every 65-90 cycles whatever N is (two warps issue in
+// parallel; two lanes of one warp barely do), so at H = 128 (20 MMAs a tile)
+// a consumer warpgroup that issued its own MMAs would spend about a third of
+// each tile issuing while its other warps wait.  With issuer warps the four
+// epilogue warps only convert accumulators and write outputs.  Issuer A
+// issues layers 1 and 2 and prepares the next tile while layer 2's result is
+// converted; issuer B issues the output layer, its first K steps while the
+// second half of its operand is still being converted, its last ones while A
+// issues the next tile's layer 1.  The H = 64 kernel (four consumers, 1024
+// threads) has no registers to spare for the extra warps.
+template <int H>
+__host__ __device__ constexpr bool issuer_warp() {
+  return H >= 128;
+}
+
+// Named barriers between a consumer's epilogue warps (E) and its issuers A and
+// B (ids above the warpgroup barriers 1..NP+NC), with their thread counts:
+// T A hands a tile over to E and B (192), X E has converted layer 1's result
+// (A waits, 160), Y E has converted the first half of layer 2's result and
+// read the previous tile's outputs (B waits, 160), Z E has converted all of it
+// (A and B wait, 192).
+constexpr int kIssT = 0, kIssX = 1, kIssY = 2, kIssZ = 3;
+constexpr int kIssTN = 192, kIssXN = 160, kIssYN = 160, kIssZN = 192;
+template <int NP, int NC>
+__device__ __forceinline__ int iss_bar(int c, int which) {
+  return NP + NC + 1 + 4 * c + which;
+}
+__device__ __forceinline__ void named_sync(int id, int n) {
+  asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void named_arrive(int id, int n) {
+  asm volatile("bar.arrive %0, %1;\n" ::"r"(id), "r"(n) : "memory");
+}
+
 template <int H, int NC, int SC>
 struct TmSmem {
   using L = TcLayout<H>;
@@ -236,7 +271,8 @@ struct TmSmem {
   // that reads late never sees the following tile's rows.
   static constexpr size_t oidx = weights + (size_t)NC * L::WIMG;
   static constexpr size_t bars = oidx + (size_t)S * 2 * 128 * 4;
-  static constexpr int nbars = 2 * S + 3 * NC;                          // full, empty, mma, weights, output
+  // full, empty, mma, weights, output; with issuer warps each issuer's final commit
+  static constexpr int nbars = 2 * S + 3 * NC + (issuer_warp<H>() ? 2 * NC : 0);
   static constexpr size_t misc = bars + (size_t)nbars * 8;
   static constexpr size_t tiles = misc + 64;
   static constexpr size_t grids = tiles + 2 * kSmemTileTable * 4;
@@ -251,13 +287,7 @@ struct TmSmem {
 // zeros elsewhere: the A operand of every layer's bias K step (the decoder image
 // keeps each layer's bias as the first row of an extra 16-row K block); then
 // each consumer's own 16-column accumulator for the output layer, so that the
-// next tile's layer 1 can run in the hidden accumulator meanwhile.  With
-// split_out<H>() the output layer's K steps are split over two accumulators
-// (each consumer's second one follows all the first ones).
-template <int H>
-__host__ __device__ constexpr bool split_out() {
-  return H >= 128;
-}
+// next tile's layer 1 can run in the hidden accumulator meanwhile.
 
 template <int H, int NC, int SC>
 struct TmCols {
@@ -265,7 +295,7 @@ struct TmCols {
   static constexpr uint32_t STG = HID + NC * (H / 2);
   static constexpr uint32_t ONES = STG + NC * SC * 8;
   static constexpr uint32_t OUT = (ONES + 8 + 15) / 16 * 16;
-  static constexpr uint32_t used = OUT + NC * 16 * (split_out<H>() ? 2 : 1);
+  static constexpr uint32_t used = OUT + NC * 16;
   static constexpr uint32_t alloc = used <= 256 ? 256 : 512;
   static_assert(used <= 512, "tensor memory plan exceeds 512 columns");
   static __device__ __forceinline__ uint32_t acc(uint32_t c) { return c * H; }
@@ -273,7 +303,6 @@ struct TmCols {
   // layer-1 A operand of stage s (= consumer * SC + st)
   static __device__ __forceinline__ uint32_t a1(uint32_t s) { return STG + 8 * s; }
   static __device__ __forceinline__ uint32_t out(uint32_t c) { return OUT + 16 * c; }
-  static __device__ __forceinline__ uint32_t out2(uint32_t c) { return OUT + 16 * (NC + c); }
 };
 
 // Warp-specialised gather-decode with tensor-memory operands.
@@ -303,12 +332,12 @@ struct TmCols {
 // row it built -- texel indices, the 16 bytes blended for each tap, their
 // weights, the mip pick and the packed feature row -- in dbg[output row].
 template <int H, bool BF16, bool TRI, bool WRAP, int CP, int NP, int NC, int SC, bool DBG>
-__global__ void __launch_bounds__((NP + NC) * 128, 1)
+__global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 : 0), 1)
     k_decode_tm(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
                 unsigned int *status, int vec_out, ntc_debug_row *dbg) {
   static_assert(NP % NC == 0 && SC % (NP / NC) == 0, "each ring stage needs one producer");
   constexpr int R = NP / NC;  // producers per consumer
-  constexpr bool SPLIT = split_out<H>();
+  constexpr bool ISS = issuer_warp<H>();
   constexpr int S = NC * SC;
   using L = TcLayout<H>;
   using M = TmSmem<H, NC, SC>;
@@ -343,8 +372,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       mbar_init(full_bar(i), 4);   // one arrival per producer warp
       mbar_init(empty_bar(i), 1);  // the consumer's layer-1 commit
     }
-    // the output barriers (the last NC) take one commit per output-layer issuer
-    for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), i >= 2 * S + 2 * NC && split_out<H>() ? 2 : 1);
+    for (int i = 2 * S; i < M::nbars; ++i) mbar_init(saddr(bars + i), 1);
     *abort_flag = 0;
     for (int i = 0; i < 2 * NC; ++i) stop_flag[i] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
@@ -520,7 +548,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
       oi = noi;
       if (two_stage) noi = nnoi;
     }
-  } else {
+  } else if (role < NP + NC) {
     // ------------------------------------------------------------ consumer
     const int c = role - NP;
     const int wgid = role;  // named barrier id role + 1
@@ -529,7 +557,6 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     const uint32_t tH = tmem_base + TC::hid(c);  // hidden A operand
     const uint32_t tOnes = tmem_base + TC::ONES; // the bias K step's A operand
     const uint32_t tO = tmem_base + TC::out(c);  // the output layer's accumulator
-    const uint32_t tO2 = tmem_base + TC::out2(c);  // its second half-K accumulator (SPLIT)
     const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
     const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
     const uint32_t obar = saddr(bars + 2 * S + 2 * NC + c);  // the output layer's completion
@@ -544,10 +571,10 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         *abort_flag = 1;
       }
     };
-    // TMEM accumulator -> ReLU -> fp16/bf16 pairs -> hidden A operand
-    auto hidden = [&]() {
+    // TMEM accumulator columns [c_lo, c_hi) -> ReLU -> fp16/bf16 pairs -> hidden A operand
+    auto hidden = [&](int c_lo = 0, int c_hi = H) {
 #pragma unroll 1
-      for (int c0 = 0; c0 < H; c0 += 32) {
+      for (int c0 = c_lo; c0 < c_hi; c0 += 32) {
         uint32_t v[32];
         tmem_ld32(tD + lanes + c0, v);
         tmem_wait_ld();
@@ -613,15 +640,7 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
     auto out_rows = [&](uint32_t eoi, bool egood) {
       uint32_t o[16];
       tmem_ld16(tO + lanes, o);
-      if constexpr (SPLIT) {
-        uint32_t o2[16];
-        tmem_ld16(tO2 + lanes, o2);
-        tmem_wait_ld();
-#pragma unroll
-        for (int cc = 0; cc < 16; ++cc) o[cc] = __float_as_uint(__uint_as_float(o[cc]) + __uint_as_float(o2[cc]));
-      } else {
-        tmem_wait_ld();
-      }
+      tmem_wait_ld();
       fence_before();
       if (egood) {
         // sigmoid(x) = 0.5 + 0.5 * tanh(x / 2)
@@ -644,107 +663,87 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         }
       }
     };
-    uint32_t k = c, dec = D, oi = 0;
-    bool good = false, stop = false;
-    if (k < K) begin(k, dec, oi, good, stop);
-    if constexpr (SPLIT) {
-      // Tile k: layer 1 (issued by begin) -> convert -> layer 2, issued by warp
-      // 3 while warps 0-2 write the previous tile's outputs (warp 3 its rows
-      // after the issue) -> convert -> the output layer, its K steps split
-      // between warps 1 and 2 and two accumulators -> begin(k + NC).  The
-      // outputs of tile k wait in tO / tO2 until tile k + NC's layer 2 runs.
-      // Layer 1 of a tile may not convert before the previous output layer
-      // has read the hidden operand, so that is waited for first.
-      bool epi = false;  // a tile's outputs wait in tO / tO2
+    if constexpr (ISS) {
+      // The epilogue warps of a consumer with issuer warps.  Per tile: A's
+      // arrival on T hands the tile over (its rows' output indices, the
+      // decision to stop); layer 1's result is converted (arrive on X); the
+      // previous tile's outputs are written while layer 2 runs; layer 2's
+      // result is converted in two halves (arrive on Y, then on Z), and B
+      // issues the output layer's first K steps in between.  A tile's outputs
+      // wait in tO until the next tile's layer 2.  Layer 1's result is
+      // converted only once the previous output layer, which reads the hidden
+      // operand, has completed.
+      const int bT = iss_bar<NP, NC>(c, kIssT), bX = iss_bar<NP, NC>(c, kIssX);
+      const int bY = iss_bar<NP, NC>(c, kIssY), bZ = iss_bar<NP, NC>(c, kIssZ);
+      bool epi = false;    // a tile's outputs wait in tO
+      bool opend = false;  // an output layer was issued and not yet waited for
+      bool stopped = false;
       uint32_t poi = 0;
       bool pgood = false;
-      while (k < K) {
+      for (uint32_t k = c; k < K; k += NC) {
+        const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
+        uint32_t dec, start, len;
+        cwalk.at(seg, tst, D, t, dec, start, len);
+        named_sync(bT, kIssTN);
+        if (stop_flag[2 * c + (jc & 1)]) {
+          stopped = true;
+          break;
+        }
+        const uint32_t oi = reinterpret_cast<const uint32_t *>(smem + M::oidx)[(s * 2 + (n & 1)) * 128 + row];
+        const bool good = oi != 0xFFFFFFFFu;
         if (dec < D) {
-          wait_bar(mbar, ph);
+          wait_bar(mbar, ph);  // layer 1
           ph ^= 1;
-          if (out_pending) {
+          if (opend) {  // the previous output layer has read the hidden operand
             wait_bar(obar, oph);
             oph ^= 1;
-            out_pending = false;
+            opend = false;
           }
           wg_bar(wgid);
           fence_after();
           hidden();
           fence_before();
-          wg_bar(wgid);
-          if (row == 96) {
-            fence_after();
-#pragma unroll
-            for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
-            umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
-            umma_commit(mbar);
-          }
+          named_arrive(bX, kIssXN);
           if (epi) {
-            __syncwarp();  // warp 3 reconverges after its issue; tcgen05.ld is warp-wide
             out_rows(poi, pgood);
             epi = false;
           }
-          wait_bar(mbar, ph);
+          wait_bar(mbar, ph);  // layer 2
           ph ^= 1;
           wg_bar(wgid);
           fence_after();
-          hidden();
+          hidden(0, H / 2);
           fence_before();
-          wg_bar(wgid);
-          if (row == 32) {  // bias and the first half of the K steps
-            fence_after();
-            umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 0);
-#pragma unroll
-            for (uint32_t kq = 0; kq < H / 32; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, 1);
-            umma_commit(obar);
-          } else if (row == 64) {  // the second half
-            fence_after();
-#pragma unroll
-            for (uint32_t kq = H / 32; kq < H / 16; ++kq)
-              umma_ta(tO2, tH + 8 * kq, dW3 + 16 * kq, id_out, kq > H / 32);
-            umma_commit(obar);
-          }
-          out_pending = true;
+          named_arrive(bY, kIssYN);
+          hidden(H / 2, H);
+          fence_before();
+          named_arrive(bZ, kIssZN);
           epi = true;
+          opend = true;
           poi = oi;
           pgood = good;
         } else if (epi) {  // a tile with nothing to multiply: write the waiting outputs now
-          if (out_pending) {
+          if (opend) {
             wait_bar(obar, oph);
             oph ^= 1;
-            out_pending = false;
+            opend = false;
           }
           wg_bar(wgid);
           fence_after();
           out_rows(poi, pgood);
           epi = false;
         }
-        const uint32_t kn = k + NC;
-        uint32_t ndec = D, noi = 0;
-        bool ngood = false, nstop = false;
-        if (kn < K && !stop) begin(kn, ndec, noi, ngood, nstop);
-        if (stop || nstop) {  // every warp of this warpgroup read the same flags
-          if (nstop && ndec < D) wait_bar(mbar, ph);  // issued MMAs end before TMEM is released
-          if (out_pending) wait_bar(obar, oph);
-          epi = false;
-          break;
-        }
-        k = kn;
-        dec = ndec;
-        oi = noi;
-        good = ngood;
       }
-      if (epi) {  // the last tile's outputs
-        if (out_pending) {
-          wait_bar(obar, oph);
-          oph ^= 1;
-          out_pending = false;
-        }
+      if (epi && !stopped) {  // the last tile's outputs
+        if (opend) wait_bar(obar, oph);
         wg_bar(wgid);
         fence_after();
         out_rows(poi, pgood);
       }
     } else {
+      uint32_t k = c, dec = D, oi = 0;
+      bool good = false, stop = false;
+      if (k < K) begin(k, dec, oi, good, stop);
       while (k < K) {
         if (dec < D) {
 #pragma unroll 1
@@ -799,6 +798,141 @@ __global__ void __launch_bounds__((NP + NC) * 128, 1)
         good = ngood;
       }
     }
+  } else if constexpr (ISS) {
+    // ------------------------------------------------------------ MMA issuers
+    // Warps 2c (A) and 2c + 1 (B) after the warpgroups issue consumer c's
+    // MMAs (lane 0).  A prepares each tile -- waits for the stage's features
+    // and, when the decoder changes, for the previous output layer (it reads
+    // W3 of the image the copy replaces) and the new weights -- and hands it
+    // over on T with the decision to stop, so every warp of the consumer
+    // stops at the same tile.  A issues layer 1, layer 2 once X arrives, and
+    // prepares the next tile while the epilogue converts layer 2's result; B
+    // issues the output layer's bias and first K steps once Y arrives and the
+    // rest once Z arrives.  Every wait is bounded.
+    const int iw = (int)((threadIdx.x - (NP + NC) * 128) >> 5);
+    const int c = iw >> 1;
+    const bool issuer_a = (iw & 1) == 0;
+    const uint32_t tD = tmem_base + TC::acc(c), tH = tmem_base + TC::hid(c), tOnes = tmem_base + TC::ONES;
+    const uint32_t tO = tmem_base + TC::out(c);
+    const uint32_t sW1 = sbase + (uint32_t)(M::weights + c * L::WIMG), sW2 = sW1 + L::W1, sW3 = sW2 + L::W2;
+    const uint32_t mbar = saddr(bars + 2 * S + c), wbar = saddr(bars + 2 * S + NC + c);
+    const uint32_t obar = saddr(bars + 2 * S + 2 * NC + c);
+    const uint32_t fbar = saddr(bars + 2 * S + 3 * NC + 2 * c + (issuer_a ? 0 : 1));
+    const int bT = iss_bar<NP, NC>(c, kIssT), bX = iss_bar<NP, NC>(c, kIssX);
+    const int bY = iss_bar<NP, NC>(c, kIssY), bZ = iss_bar<NP, NC>(c, kIssZ);
+    constexpr uint32_t id_hidden = instr_desc<BF16>(H), id_out = instr_desc<BF16>(16);
+    const uint64_t dW1 = smem_desc(sW1, kTcKA), dW2 = smem_desc(sW2, L::KH), dW3 = smem_desc(sW3, L::KH);
+    bool issued = false;
+    auto wait = [&](uint32_t b, uint32_t parity) {  // lane 0
+      if (!mbar_wait(b, parity)) {
+        atomicOr(status, 1u);
+        *abort_flag = 1;
+      }
+    };
+    TileWalk iwalk;
+    iwalk.ident_n = B.identity_n;
+    if (issuer_a) {
+      uint32_t cur = 0xFFFFFFFFu, wph = 0, l3 = 0;  // l3: output layers issued (by B)
+      // Tile k's stage holds its features; returns the decision to stop
+      // (lane 0's, not yet shared) and whether the weights must be replaced
+      // first, which waits for the previous output layer and so is left for
+      // after Z.
+      auto prepare = [&](uint32_t k, uint32_t &dec, bool &swap) -> uint32_t {
+        const uint32_t jc = k / NC, t = blockIdx.x + k * grid, s = c * SC + jc % SC, n = jc / SC;
+        uint32_t start, len;
+        iwalk.at(seg, tst, D, t, dec, start, len);
+        swap = dec < D && dec != cur;
+        uint32_t stop = 0;
+        if (lane == 0) {
+          wait(full_bar(s), n & 1);  // the features and the rows' output indices
+          stop = *abort_flag;
+        }
+        return stop;
+      };
+      auto load_weights = [&](uint32_t dec) {  // lane 0
+        if (l3) wait(obar, (l3 - 1) & 1);
+        fence_after();
+        bulk_g2s(sW1, W.tc + (size_t)dec * W.tc_stride, L::WIMG, wbar);
+        wait(wbar, wph);
+        wph ^= 1;
+      };
+      uint32_t dec = D;
+      bool swap = false;
+      uint32_t stop = c < K ? prepare(c, dec, swap) : 0;
+      for (uint32_t k = c; k < K; k += NC) {
+        const uint32_t jc = k / NC, s = c * SC + jc % SC;
+        if (lane == 0) {
+          if (swap && !stop && !*abort_flag) {
+            load_weights(dec);
+            cur = dec;
+          }
+          stop |= *abort_flag;
+          stop_flag[2 * c + (jc & 1)] = stop;
+        }
+        stop = __shfl_sync(0xFFFFFFFFu, stop, 0);
+        named_arrive(bT, kIssTN);
+        if (stop) break;
+        const uint32_t tdec = dec;
+        if (tdec < D) {
+          if (lane == 0) {
+            fence_after();
+            umma_ta(tD, tmem_base + TC::a1(s), dW1, id_hidden, 0);
+            umma_ta(tD, tOnes, dW1 + 16, id_hidden, 1);  // + bias
+            umma_commit(mbar);
+            umma_commit(empty_bar(s));
+          }
+          issued = true;
+          __syncwarp();
+          named_sync(bX, kIssXN);
+          if (lane == 0) {
+            fence_after();
+#pragma unroll
+            for (uint32_t kq = 0; kq < H / 16; ++kq) umma_ta(tD, tH + 8 * kq, dW2 + 16 * kq, id_hidden, kq);
+            umma_ta(tD, tOnes, dW2 + 16 * (H / 16), id_hidden, 1);  // + bias
+            umma_commit(mbar);
+          }
+          ++l3;
+        } else if (lane == 0) {
+          mbar_arrive(empty_bar(s));  // a tile of bad queries: nothing to multiply
+        }
+        __syncwarp();
+        // the next tile, while layer 2's result is converted
+        stop = k + NC < K ? prepare(k + NC, dec, swap) : 0;
+        __syncwarp();
+        if (tdec < D) named_sync(bZ, kIssZN);  // layer 1 of the next tile overwrites the accumulator
+      }
+    } else {
+      for (uint32_t k = c; k < K; k += NC) {
+        const uint32_t jc = k / NC, t = blockIdx.x + k * grid;
+        uint32_t dec, start, len;
+        iwalk.at(seg, tst, D, t, dec, start, len);
+        named_sync(bT, kIssTN);
+        if (stop_flag[2 * c + (jc & 1)]) break;
+        if (dec >= D) continue;
+        named_sync(bY, kIssYN);
+        if (lane == 0) {  // the bias, then the K steps of the converted half
+          fence_after();
+          umma_ta(tO, tOnes, dW3 + 16 * (H / 16), id_out, 0);
+#pragma unroll
+          for (uint32_t kq = 0; kq < H / 32; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, 1);
+        }
+        issued = true;
+        __syncwarp();
+        named_sync(bZ, kIssZN);
+        if (lane == 0) {
+          fence_after();
+#pragma unroll
+          for (uint32_t kq = H / 32; kq < H / 16; ++kq) umma_ta(tO, tH + 8 * kq, dW3 + 16 * kq, id_out, 1);
+          umma_commit(obar);
+        }
+        __syncwarp();
+      }
+    }
+    if (lane == 0 && issued) {  // no MMA of this issuer is in flight when tensor memory is released
+      umma_commit(fbar);
+      wait(fbar, 0);
+    }
+    __syncwarp();
   }
   fence_before();
   __syncthreads();
@@ -835,7 +969,7 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   size_t grid = (size_t)num_sms;
   if (grid > max_tiles) grid = max_tiles;
   const int vec_out = ((uintptr_t)out & 31) == 0;  // 32-byte rows need a 32-byte aligned base
-  const unsigned threads = (NP + NC) * 128;
+  const unsigned threads = (NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 : 0);
   // launched as a programmatic dependent of the bucketing: its prologue overlaps
   // the end of k_scatter
   cudaError_t e;
