@@ -82,6 +82,7 @@ def parse():
     p.add_argument("--no-mirror", action="store_true", help="skip the mirror of the paper's Tables 5-6")
     p.add_argument("--no-maps", action="store_true", help="skip the Table 2 groupings of a 586-set workload")
     p.add_argument("--no-variants", action="store_true", help="skip Sec. 4's decoder shape")
+    p.add_argument("--no-fp16-out", action="store_true", help="skip the fp16-output-row step")
     p.add_argument("--variants", action="store_true", help="also time every A x B size of Sec. 4's MLP ablation")
     p.add_argument("--small", action="store_true", help="the small size of the timed workload")
     p.add_argument("--medium", action="store_true",
@@ -414,19 +415,21 @@ def main():
 
     # end to end through the public host-buffer call
     hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
-    hout = torch.empty((n, C), dtype=torch.float32).pin_memory()
-    for _ in range(2):
-        dec.decode_host(hq, hout, mode=args.mode)
-    e2e_t = []
-    for _ in range(max(3, min(args.steps, 10))):
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        dec.decode_host(hq, hout, mode=args.mode)
-        e2e_t.append(time.perf_counter() - t0)
-    e2e_ms = 1e3 * statistics.mean(e2e_t)
-    e2e = {"value": n * ws / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": n * 16,
-           "d2h_bytes_per_step": n * C * 4, "ms_per_step": e2e_ms}
-    del hq, hout
+    e2e_reps = max(3, min(args.steps, 10))
+    e2e = end_to_end(torch, dec, hq, n, C, ws, args.mode, e2e_reps)
+
+    # the same step with fp16 output rows (Sec. 4.4's fp16 kernels write fp16)
+    out_fp16 = None
+    if args.precision != "fp32" and args.mode == "bucketed" and not args.no_fp16_out:
+        d16 = ntc.Decoder(w.assets, args.precision, output="fp16")
+        o16 = torch.empty((n, C), dtype=torch.float16, device="cuda")
+        ms16 = time_decode(torch, d16, qd, o16, "bucketed", flush, flush_rd, reps=e2e_reps, warm=2)
+        out_fp16 = {"value": n * ws / (ms16 / 1e3), "unit": UNIT, "ms_per_step": ms16,
+                    "output_bytes_per_query": 2 * C,
+                    "e2e": end_to_end(torch, d16, hq, n, C, ws, "bucketed", e2e_reps)}
+        d16.close()
+        del o16, d16
+    del hq
 
     # the in-run comparison: the unsorted kernels on the same batch
     extra = {}
@@ -462,6 +465,7 @@ def main():
                          "outside the step events); inputs larger than L2",
                    "parallelism": f"{ws} independent replicas (queries sharded, no collective)"},
         "roofline": roofline, "e2e": e2e, "gpu_launches": launches, "clocks": clocks,
+        **({"output_fp16": out_fp16} if out_fp16 else {}),
         "flops_per_query": flops_q, "bytes_per_query": bpq,
         **extra,
     }
@@ -482,6 +486,24 @@ def main():
         print(json.dumps(result), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def end_to_end(torch, dec, hq, n, C, ws, mode, reps):
+    """The metric through ntc_decode_host: pinned host queries in, host output
+    rows out (the context's output format), copies inside the timed region."""
+    half = dec.output == "fp16"
+    hout = torch.empty((n, C), dtype=torch.float16 if half else torch.float32).pin_memory()
+    for _ in range(2):
+        dec.decode_host(hq, hout, mode=mode)
+    ts = []
+    for _ in range(reps):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dec.decode_host(hq, hout, mode=mode)
+        ts.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.mean(ts)
+    return {"value": n * ws / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": n * 16,
+            "d2h_bytes_per_step": n * C * (2 if half else 4), "ms_per_step": ms}
 
 
 def time_decode(torch, dec, qd, out, mode, flush, flush_rd, reps=5, warm=2):

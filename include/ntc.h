@@ -75,8 +75,9 @@ typedef struct {
 } ntc_query;
 
 /* Arithmetic of the MLP.  TC_*: tensor cores with fp16/bf16 operands and fp32
- * accumulation; FP32: CUDA-core fp32 reference mode. Features, bilinear
- * weights, bias, sigmoid and the output are fp32 in every mode. */
+ * accumulation; FP32: CUDA-core fp32 reference mode.  Bias and sigmoid are
+ * fp32 in every mode; the output rows are fp32 unless ntc_desc.output_format
+ * asks for fp16 rows. */
 typedef enum {
   NTC_PREC_TC_FP16 = 0,
   NTC_PREC_TC_BF16 = 1,
@@ -150,7 +151,18 @@ typedef struct {
                                  output with a positional encoding             */
   uint32_t activation;        /* 0 = ReLU, 1 = LeakyReLU (Sec. 4)               */
   float leaky_slope;          /* LeakyReLU slope for x <= 0 (e.g. 0.01)         */
+  uint32_t output_format;     /* NTC_OUTPUT_FP32 or NTC_OUTPUT_FP16, below      */
 } ntc_desc;
+
+/* Output element type of ntc_decode.  FP32: out_dim floats per row.  FP16:
+ * out_dim IEEE binary16 values per row, each the fp32 sigmoid rounded to
+ * nearest even (a C = 8 row is 16 bytes, one vector store); the paper's fp16
+ * kernels are fp16 end to end (Sec. 4.4, Tables 5-6).  FP16 rows are written
+ * by the BUCKETED mode with the tensor-core precisions (ntc_create refuses
+ * FP16 rows with NTC_PREC_FP32; ntc_decode returns NTC_ERR_UNSUPPORTED for the
+ * other modes).  A bad query's row is NaN (0x7E00) in every channel. */
+#define NTC_OUTPUT_FP32 0u
+#define NTC_OUTPUT_FP16 1u
 
 /* Decoder shapes.  The standard shape (2 levels x 8 channels, no encoding, 2
  * hidden layers of 64 or 128, ReLU) runs every mode on the specialised
@@ -167,13 +179,17 @@ typedef struct {
  * and return a context in *out.  Synchronous.  On failure *out is NULL. */
 NTC_API ntc_status ntc_create(const ntc_desc *desc, ntc_ctx **out);
 
-/* Decode n queries: d_out[i][c] = channel c of D_{c(set_i)}(features of query
- * i), for c < out_dim, in the queries' original order.  d_queries: device
- * array of n records (16-byte aligned); d_out: device array of n*out_dim
- * floats.  Asynchronous on `cuda_stream` (a cudaStream_t; NULL is the legacy
- * default stream); no host synchronisation.  n = 0 is a no-op.  Output for a
- * bad query is NaN in every channel. */
-NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_out,
+/* Decode n queries: every query's latent features go through the MLP decoder
+ * of its texture set's group (the per-pixel decode of Sec. 2; set i uses the
+ * shared decoder c(i) of Sec. 3.1): d_out[i][c] = channel c of
+ * D_{c(set_i)}(features of query i), for c < out_dim, in the queries' original
+ * order.  d_queries: device array of n records (16-byte aligned); d_out:
+ * device array of n*out_dim elements of the context's output format (floats,
+ * 4-byte aligned; or IEEE halves, 2-byte aligned).  Asynchronous on
+ * `cuda_stream` (a cudaStream_t; NULL is the legacy default stream); no host
+ * synchronisation.  n = 0 is a no-op.  Output for a bad query is NaN in every
+ * channel. */
+NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, void *d_out,
                       void *cuda_stream, ntc_mode mode);
 
 /* ntc_decode on HOST buffers: copies the queries to context-owned device
@@ -184,7 +200,7 @@ NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n
  * `cuda_stream`, decodes on `cuda_stream`.  Each chunk is bucketed on its own;
  * outputs are the same as one ntc_decode over all n.  Pinned host memory is
  * needed for the copies to overlap. */
-NTC_API ntc_status ntc_decode_host(ntc_ctx *ctx, const ntc_query *h_queries, size_t n, float *h_out,
+NTC_API ntc_status ntc_decode_host(ntc_ctx *ctx, const ntc_query *h_queries, size_t n, void *h_out,
                            void *cuda_stream, ntc_mode mode);
 
 /* Free the context and everything it owns.  NULL is accepted. */
@@ -254,7 +270,7 @@ typedef struct {
  * d_rows[i] (device array of n records; rows of bad queries are not
  * written).  TC_FP16/TC_BF16 contexts of the standard shape only
  * (NTC_ERR_UNSUPPORTED otherwise).  Device pointers; async. */
-NTC_API ntc_status ntc_debug_decode_rows(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_out,
+NTC_API ntc_status ntc_debug_decode_rows(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, void *d_out,
                                          ntc_debug_row *d_rows, void *cuda_stream);
 
 /* Upper bound on the number of 128-query tiles of n queries. */

@@ -97,7 +97,7 @@ __host__ __device__ inline uint32_t gen_tmem_need(uint32_t H, uint32_t K1) {
 // (its completion empties the stage) and every further layer from the hidden
 // operand; consumer thread r runs row r's epilogues.
 template <bool BF16, int L, int C>
-__global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, float *out,
+__global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_decode_gen_tc(Assets A, GenWeights G, Buckets B, void *out,
                                                        unsigned long long *err, unsigned int *status,
                                                        uint32_t tmem_cols, uint32_t img_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -193,8 +193,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
       const bool good = valid && !query_bad(A, q);
       const bool bad = valid && !good;
       count_bad_warp(bad, err);
-      if (bad)
-        for (uint32_t c = 0; c < OC; ++c) out[(size_t)oi * OC + c] = __int_as_float(0x7fc00000);
+      if (bad) put_nan_row(out, oi, OC, G.out_half);
       // the feature row, packed to fp16/bf16 pairs as it is produced: the
       // latent features, then sin/cos pairs of the encoding (zeros beyond)
       constexpr int LW = L * C / 2, NW = NP / 2;
@@ -399,7 +398,6 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
       tmem_wait_ld();
       if (good) {
         const float4 *bo = reinterpret_cast<const float4 *>(bias + NL * H);
-        float *dst = out + (size_t)oi * OC;
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
           if (c < (int)OC) {
@@ -408,7 +406,7 @@ __global__ void __launch_bounds__(256, L * C <= 4 ? 4 : (L * C <= 8 ? 3 : 2)) k_
             const float x = __uint_as_float(o[c]) + (c % 4 == 0 ? b.x : c % 4 == 1 ? b.y : c % 4 == 2 ? b.z : b.w);
             float th;
             asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * x));
-            dst[c] = fmaf(0.5f, th, 0.5f);
+            put_out(out, (size_t)oi * OC + c, fmaf(0.5f, th, 0.5f), G.out_half);
           }
         }
       }
@@ -579,7 +577,7 @@ uint32_t gen_tmem_cols(const GenWeights &G) {
 }
 
 template <bool BF16, int L, int C>
-cudaError_t launch_gen_tc_t(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+cudaError_t launch_gen_tc_t(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, void *out,
                             unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
   const uint32_t img = (uint32_t)gen_tc_image_bytes(G.in_dim, G.hidden, G.layers);
   const size_t smem = gen_smem_bytes(img);
@@ -600,7 +598,7 @@ cudaError_t launch_gen_tc_t(const Assets &A, const GenWeights &G, const Buckets 
 }
 
 template <bool BF16>
-cudaError_t launch_gen_tc_b(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+cudaError_t launch_gen_tc_b(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, void *out,
                             unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st) {
   if (A.channels == 8)
     return A.num_levels == 2 ? launch_gen_tc_t<BF16, 2, 8>(A, G, B, n, out, err, status, num_sms, st)
@@ -624,7 +622,7 @@ cudaError_t launch_gen_fma_t(const Assets &A, const GenWeights &G, const Buckets
 
 }  // namespace
 
-cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, void *out,
                                  unsigned long long *err, unsigned int *status, bool bf16, int num_sms,
                                  cudaStream_t st, int *launches) {
   *launches += 1;

@@ -49,7 +49,7 @@ cudaError_t launch_pack_tc(const float *w32, uint32_t D, uint32_t H, uint32_t C,
 }
 
 cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
-                             float *out, unsigned long long *err, unsigned int *status, bool bf16,
+                             void *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches) {
   *launches += 1;
   return dispatch_tm<false>(A, W, B, n, out, err, status, bf16, num_sms, st, nullptr);

@@ -333,7 +333,7 @@ struct TmCols {
 // weights, the mip pick and the packed feature row -- in dbg[output row].
 template <int H, bool BF16, bool TRI, bool WRAP, int CP, int NP, int NC, int SC, bool DBG>
 __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 : 0), 1)
-    k_decode_tm(Assets A, WeightImages W, Buckets B, float *out, unsigned long long *err,
+    k_decode_tm(Assets A, WeightImages W, Buckets B, void *out, unsigned long long *err,
                 unsigned int *status, int vec_out, ntc_debug_row *dbg) {
   static_assert(NP % NC == 0 && SC % (NP / NC) == 0, "each ring stage needs one producer");
   constexpr int R = NP / NC;  // producers per consumer
@@ -510,8 +510,7 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
       const bool bad = valid && !good;
       const uint32_t badm = __ballot_sync(0xFFFFFFFFu, bad);
       if (badm && lane == __ffs(badm) - 1) atomicAdd(err, (unsigned long long)__popc(badm));
-      if (bad)
-        for (uint32_t cc = 0; cc < C; ++cc) out[(size_t)oi * C + cc] = __int_as_float(0x7fc00000);
+      if (bad) put_nan_row(out, oi, C, W.out_half);
       __half2 acc[kLevels][4];
       accum_taps<true>(taps, acc);
       if (TRI) prefetch();
@@ -651,15 +650,26 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
           asm("tanh.approx.f32 %0, %1;" : "=f"(th) : "f"(0.5f * __uint_as_float(o[cc])));
           y[cc] = fmaf(0.5f, th, 0.5f);
         }
-        float *dst = out + (size_t)eoi * C;
-        if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
-          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(dst), "f"(y[0]),
-                       "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
+        if (CP == 8 && vec_out && C == 8 && W.out_half) {  // one 16-byte store per row
+          uint32_t h[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const __half2 p = __floats2half2_rn(y[2 * i], y[2 * i + 1]);
+            h[i] = *reinterpret_cast<const uint32_t *>(&p);
+          }
+          asm volatile("st.global.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"l"(reinterpret_cast<__half *>(out) +
+                                                                        (size_t)eoi * 8),
+                       "r"(h[0]), "r"(h[1]), "r"(h[2]), "r"(h[3])
+                       : "memory");
+        } else if (CP == 8 && vec_out && C == 8) {  // one 32-byte store per row
+          asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"l"(
+                           reinterpret_cast<float *>(out) + (size_t)eoi * 8),
+                       "f"(y[0]), "f"(y[1]), "f"(y[2]), "f"(y[3]), "f"(y[4]), "f"(y[5]), "f"(y[6]), "f"(y[7])
                        : "memory");
         } else {
 #pragma unroll
           for (int cc = 0; cc < CP; ++cc)
-            if (cc < (int)C) dst[cc] = y[cc];
+            if (cc < (int)C) put_out(out, (size_t)eoi * C + cc, y[cc], W.out_half);
         }
       }
     };
@@ -944,7 +954,7 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
 }
 
 template <int H, bool BF16, bool TRI, bool WRAP, int NP, int NC, int SC, bool DBG>
-cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, float *out,
+cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, void *out,
                         unsigned long long *err, unsigned int *status, int num_sms, cudaStream_t st,
                         ntc_debug_row *dbg) {
   using M = TmSmem<H, NC, SC>;
@@ -968,7 +978,8 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   const size_t max_tiles = (n + kTile - 1) / kTile + A.num_decoders + 1;
   size_t grid = (size_t)num_sms;
   if (grid > max_tiles) grid = max_tiles;
-  const int vec_out = ((uintptr_t)out & 31) == 0;  // 32-byte rows need a 32-byte aligned base
+  // vector row stores need a base aligned to the row: 32 bytes (fp32) or 16 (fp16)
+  const int vec_out = ((uintptr_t)out & (W.out_half ? 15 : 31)) == 0;
   const unsigned threads = (NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 : 0);
   // launched as a programmatic dependent of the bucketing: its prologue overlaps
   // the end of k_scatter
@@ -989,7 +1000,7 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
 // dispatched at run time: 4 producer + 4 consumer warpgroups at H = 64, 4 + 2
 // at H = 128 (tensor memory holds two 128-column accumulators).
 template <bool DBG>
-cudaError_t dispatch_tm(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, float *out,
+cudaError_t dispatch_tm(const Assets &A, const WeightImages &W, const Buckets &B, size_t n, void *out,
                         unsigned long long *err, unsigned int *status, bool bf16, int num_sms, cudaStream_t st,
                         ntc_debug_row *dbg) {
   const bool tri = A.num_mips > 1, wrap = A.address_mode == 0;

@@ -6,7 +6,7 @@
 namespace ntc {
 
 cudaError_t launch_decode_tc_debug(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
-                                   float *out, unsigned long long *err, unsigned int *status, bool bf16,
+                                   void *out, unsigned long long *err, unsigned int *status, bool bf16,
                                    int num_sms, cudaStream_t st, int *launches, ntc_debug_row *rows) {
   *launches += 1;
   return dispatch_tm<true>(A, W, B, n, out, err, status, bf16, num_sms, st, rows);

@@ -26,6 +26,7 @@ struct ntc_ctx {
   uint32_t L = kLevels, LC = kChannels, F = 0, NL = 2, in_dim = kInDim, act = 0;
   float slope = 0.0f;
   bool general = false;
+  uint32_t out_half = 0;  // output rows are IEEE half (NTC_OUTPUT_FP16)
   uint8_t *d_gtc = nullptr, *d_gfma = nullptr;
   size_t gtc_stride = 0, gfma_stride = 0;
   ntc_precision prec = NTC_PREC_TC_FP16;
@@ -50,7 +51,7 @@ struct ntc_ctx {
   // staging for ntc_decode_host, and its copy streams and chunk events
   size_t cap_host = 0;
   ntc_query *d_hq = nullptr;
-  float *d_hout = nullptr;
+  uint8_t *d_hout = nullptr;  // [cap_host][C] output elements of out_bytes each
   cudaStream_t s_up = nullptr, s_down = nullptr;
   cudaEvent_t ev_begin = nullptr, ev_up[kHostChunksMax] = {}, ev_done[kHostChunksMax] = {};
   uint64_t launches = 0;
@@ -132,6 +133,7 @@ GenWeights gen_of(const ntc_ctx *c) {
   G.out_dim = c->C;
   G.activation = c->act;
   G.slope = c->slope;
+  G.out_half = c->out_half;
   return G;
 }
 
@@ -147,6 +149,7 @@ WeightImages weights_of(const ntc_ctx *c) {
   W.fma_stride = c->fma_stride;
   W.hidden = c->H;
   W.out_dim = c->C;
+  W.out_half = c->out_half;
   return W;
 }
 
@@ -295,6 +298,10 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   if (d->precision != NTC_PREC_TC_FP16 && d->precision != NTC_PREC_TC_BF16 && d->precision != NTC_PREC_FP32)
     return fail(NTC_ERR_INVALID_ARG, "unknown precision");
   if (d->address_mode > 1) return fail(NTC_ERR_INVALID_ARG, "address_mode must be 0 (wrap) or 1 (clamp)");
+  if (d->output_format != NTC_OUTPUT_FP32 && d->output_format != NTC_OUTPUT_FP16)
+    return fail(NTC_ERR_INVALID_ARG, "output_format must be NTC_OUTPUT_FP32 or NTC_OUTPUT_FP16");
+  if (d->output_format == NTC_OUTPUT_FP16 && d->precision == NTC_PREC_FP32)
+    return fail(NTC_ERR_UNSUPPORTED, "fp16 output rows come from the tensor-core precisions only");
   if (d->num_texels < 1) return fail(NTC_ERR_INVALID_ARG, "num_texels must be >= 1");
   const uint32_t S = d->num_sets, M = d->num_mips, L = d->num_levels;
   std::vector<GridDesc> grids((size_t)S * L * M);
@@ -340,6 +347,7 @@ ntc_status ntc_create(const ntc_desc *d, ntc_ctx **out) {
   c->in_dim = d->in_dim;
   c->act = d->activation;
   c->slope = d->activation == 1 ? d->leaky_slope : 0.0f;
+  c->out_half = d->output_format == NTC_OUTPUT_FP16;
   c->general = !(c->L == kLevels && c->LC == kChannels && c->F == 0 && c->NL == 2 && c->act == 0 &&
                  (c->H == 64 || c->H == 128));
   const size_t P = (size_t)c->H * (c->in_dim + 1) + (size_t)(c->NL - 1) * c->H * (c->H + 1) +
@@ -436,16 +444,16 @@ ntc_status ntc_destroy(ntc_ctx *c) {
 }
 
 namespace {
-ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream, ntc_mode mode,
+ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, void *out, void *stream, ntc_mode mode,
                        ntc_debug_row *rows);
 }
 
-ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream,
+ntc_status ntc_decode(ntc_ctx *c, const ntc_query *q, size_t n, void *out, void *stream,
                       ntc_mode mode) {
   return decode_impl(c, q, n, out, stream, mode, nullptr);
 }
 
-ntc_status ntc_debug_decode_rows(ntc_ctx *c, const ntc_query *q, size_t n, float *out, ntc_debug_row *rows,
+ntc_status ntc_debug_decode_rows(ntc_ctx *c, const ntc_query *q, size_t n, void *out, ntc_debug_row *rows,
                                  void *stream) {
   if (!c) return fail(NTC_ERR_INVALID_ARG, "null context");
   if (c->general || c->prec == NTC_PREC_FP32)
@@ -459,12 +467,14 @@ ntc_status ntc_debug_decode_rows(ntc_ctx *c, const ntc_query *q, size_t n, float
 namespace {
 // ntc_decode; with rows != nullptr the tensor-core kernel is the debug
 // instantiation that also records every row it builds.
-ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, void *stream, ntc_mode mode,
+ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, void *vout, void *stream, ntc_mode mode,
                        ntc_debug_row *rows) {
   ntc_status s = check_queries(c, q, n);
   if (s != NTC_OK) return s;
-  if (n && !out) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
-  if (((uintptr_t)out & 3) != 0) return fail(NTC_ERR_INVALID_ARG, "output buffer is not 4-byte aligned");
+  if (n && !vout) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
+  if (((uintptr_t)vout & (c->out_half ? 1 : 3)) != 0)
+    return fail(NTC_ERR_INVALID_ARG, "output buffer is not aligned to its element (%d bytes)", c->out_half ? 2 : 4);
+  float *out = static_cast<float *>(vout);  // the fp32 paths
   if (mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT && mode != NTC_MODE_BUCKETED_MMA &&
       mode != NTC_MODE_DIVERGENT_FMA)
     return fail(NTC_ERR_INVALID_ARG, "unknown mode");
@@ -473,6 +483,8 @@ ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, voi
     return fail(NTC_ERR_UNSUPPORTED, "the fp32 precision has only the bucketed and divergent FMA modes");
   if (c->general && mode != NTC_MODE_BUCKETED && mode != NTC_MODE_DIVERGENT_FMA)
     return fail(NTC_ERR_UNSUPPORTED, "this decoder shape has only the bucketed and divergent FMA modes");
+  if (c->out_half && mode != NTC_MODE_BUCKETED)
+    return fail(NTC_ERR_UNSUPPORTED, "fp16 output rows are written by the bucketed tensor-core decode only");
   if (n == 0) return NTC_OK;
   DeviceGuard g(c->device);
   if (!g.ok) return fail(NTC_ERR_CUDA, "cannot select the context's device");
@@ -527,15 +539,15 @@ ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, voi
   if (c->general && fp32)
     e = launch_decode_gen_fma(A, gen_of(c), &B, nullptr, n, out, c->d_err, c->prec, c->num_sms, st, &launches);
   else if (c->general)
-    e = launch_decode_gen_tc(A, gen_of(c), B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
+    e = launch_decode_gen_tc(A, gen_of(c), B, n, vout, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
   else if (fp32)
     e = launch_decode_fp32(A, W, B, n, out, c->d_err, c->num_sms, st, &launches);
   else if (mode == NTC_MODE_BUCKETED_MMA)
     e = launch_decode_mma(A, W, B, n, out, c->d_err, bf16, c->num_sms, st, &launches);
   else if (rows)
-    e = launch_decode_tc_debug(A, W, B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches, rows);
+    e = launch_decode_tc_debug(A, W, B, n, vout, c->d_err, c->d_status, bf16, c->num_sms, st, &launches, rows);
   else
-    e = launch_decode_tc(A, W, B, n, out, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
+    e = launch_decode_tc(A, W, B, n, vout, c->d_err, c->d_status, bf16, c->num_sms, st, &launches);
   c->launches += launches;
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   if (c->timing) {
@@ -548,8 +560,9 @@ ntc_status decode_impl(ntc_ctx *c, const ntc_query *q, size_t n, float *out, voi
 
 extern "C" {
 
-ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hout, void *stream,
+ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, void *vhout, void *stream,
                            ntc_mode mode) {
+  uint8_t *hout = static_cast<uint8_t *>(vhout);
   ntc_status s = check_queries(c, hq, n);
   if (s != NTC_OK) return s;
   if (n && !hout) return fail(NTC_ERR_INVALID_ARG, "null output pointer");
@@ -566,7 +579,7 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hou
     c->d_hout = nullptr;
     c->cap_host = 0;
     CK(cudaMalloc((void **)&c->d_hq, n * sizeof(ntc_query)), "staging allocation");
-    CK(cudaMalloc((void **)&c->d_hout, n * c->C * sizeof(float)), "staging allocation");
+    CK(cudaMalloc((void **)&c->d_hout, n * c->C * (c->out_half ? 2 : 4)), "staging allocation");
     c->cap_host = n;
   }
   if (!c->s_up) {
@@ -586,7 +599,7 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hou
   if (chunk < kHostChunkMin) chunk = kHostChunkMin;
   chunk = (chunk + kBucketChunk - 1) / kBucketChunk * kBucketChunk;
   const size_t nchunks = (n + chunk - 1) / chunk;
-  const size_t C = c->C;
+  const size_t row = (size_t)c->C * (c->out_half ? 2 : 4);  // bytes of one output row
   CK(cudaEventRecord(c->ev_begin, st), "chunk event");
   CK(cudaStreamWaitEvent(c->s_up, c->ev_begin, 0), "stream order");
   CK(cudaStreamWaitEvent(c->s_down, c->ev_begin, 0), "stream order");
@@ -596,7 +609,7 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hou
        "query upload");
     CK(cudaEventRecord(c->ev_up[i], c->s_up), "chunk event");
     CK(cudaStreamWaitEvent(st, c->ev_up[i], 0), "stream order");
-    s = ntc_decode(c, c->d_hq + off, m, c->d_hout + off * C, stream, mode);
+    s = ntc_decode(c, c->d_hq + off, m, c->d_hout + off * row, stream, mode);
     if (s != NTC_OK) {
       cudaStreamSynchronize(c->s_up);
       cudaStreamSynchronize(c->s_down);
@@ -604,8 +617,7 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, float *hou
     }
     CK(cudaEventRecord(c->ev_done[i], st), "chunk event");
     CK(cudaStreamWaitEvent(c->s_down, c->ev_done[i], 0), "stream order");
-    CK(cudaMemcpyAsync(hout + off * C, c->d_hout + off * C, m * C * sizeof(float), cudaMemcpyDeviceToHost,
-                       c->s_down),
+    CK(cudaMemcpyAsync(hout + off * row, c->d_hout + off * row, m * row, cudaMemcpyDeviceToHost, c->s_down),
        "output download");
   }
   CK(cudaStreamSynchronize(c->s_down), "decode");

@@ -60,6 +60,7 @@ struct WeightImages {
   const uint8_t *fma;       // [D][fma_stride] bytes, per-lane FMA image
   size_t fma_stride;
   uint32_t hidden, out_dim;
+  uint32_t out_half;        // output rows in IEEE half (put_out) instead of fp32
 };
 
 
@@ -104,6 +105,7 @@ struct GenWeights {
   size_t fma_stride;
   uint32_t in_dim, k1, hidden, layers, out_dim, activation;
   float slope;
+  uint32_t out_half;  // output rows in IEEE half (put_out) instead of fp32
 };
 
 inline __host__ __device__ uint32_t gen_k1(uint32_t in_dim) { return (in_dim + 15) / 16 * 16; }
@@ -467,6 +469,24 @@ __device__ __forceinline__ void tile_info(const uint32_t *meta, uint32_t D, uint
 // forward, so a lookup is a few compares instead of a binary search.  With
 // ident_n != 0 (one decoder, nothing sorted) tile t is queries 128t .. of the
 // caller's array.
+// One output value in the context's output format: fp32, or IEEE half rounded
+// to nearest even (the fp16 output of Sec. 4.4's fp16 kernels); a bad query's
+// row is NaN in every channel.
+__device__ __forceinline__ void put_out(void *out, size_t i, float y, bool half) {
+  if (half)
+    reinterpret_cast<__half *>(out)[i] = __float2half_rn(y);
+  else
+    reinterpret_cast<float *>(out)[i] = y;
+}
+__device__ __forceinline__ void put_nan_row(void *out, size_t row, uint32_t C, bool half) {
+  for (uint32_t c = 0; c < C; ++c) {
+    if (half)
+      reinterpret_cast<unsigned short *>(out)[row * C + c] = 0x7E00u;
+    else
+      reinterpret_cast<float *>(out)[row * C + c] = __int_as_float(0x7fc00000);
+  }
+}
+
 struct TileWalk {
   uint32_t d = 0;
   uint32_t ident_n = 0;
@@ -531,7 +551,7 @@ cudaError_t launch_pack_fma(const float *w32, uint32_t D, uint32_t H, uint32_t C
 // General shapes: the tcgen05 decode over bucketed tiles, and the per-lane
 // FMA decode over the queries in bucket order (B non-null) or in their own
 // order (B null).
-cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, float *out,
+cudaError_t launch_decode_gen_tc(const Assets &A, const GenWeights &G, const Buckets &B, size_t n, void *out,
                                  unsigned long long *err, unsigned int *status, bool bf16, int num_sms,
                                  cudaStream_t st, int *launches);
 cudaError_t launch_decode_gen_fma(const Assets &A, const GenWeights &G, const Buckets *B, const ntc_query *q,
@@ -540,10 +560,10 @@ cudaError_t launch_decode_gen_fma(const Assets &A, const GenWeights &G, const Bu
 cudaError_t launch_pack_gen(const float *w32, uint32_t D, const GenWeights &G, ntc_precision prec, uint8_t *tc,
                             uint8_t *fma, cudaStream_t st);
 cudaError_t launch_decode_tc(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
-                             float *out, unsigned long long *err, unsigned int *status, bool bf16,
+                             void *out, unsigned long long *err, unsigned int *status, bool bf16,
                              int num_sms, cudaStream_t st, int *launches);
 cudaError_t launch_decode_tc_debug(const Assets &A, const WeightImages &W, const Buckets &B, size_t n,
-                                   float *out, unsigned long long *err, unsigned int *status, bool bf16,
+                                   void *out, unsigned long long *err, unsigned int *status, bool bf16,
                                    int num_sms, cudaStream_t st, int *launches, ntc_debug_row *rows);
 cudaError_t launch_pack_tc(const float *w32, uint32_t D, uint32_t H, uint32_t C, bool bf16,
                            uint8_t *tc, size_t tc_stride, cudaStream_t st);

@@ -28,6 +28,8 @@ DEBUG_ROW = np.dtype([("idx", "<u8", (2, 2, 4)), ("raw", "<u4", (2, 2, 4, 4)), (
 assert DEBUG_ROW.itemsize == 512
 
 PRECISIONS = {"fp16": NTC_PREC_TC_FP16, "bf16": NTC_PREC_TC_BF16, "fp32": NTC_PREC_FP32}
+NTC_OUTPUT_FP32, NTC_OUTPUT_FP16 = 0, 1
+OUTPUTS = {"fp32": NTC_OUTPUT_FP32, "fp16": NTC_OUTPUT_FP16}
 MODES = {"bucketed": NTC_MODE_BUCKETED, "divergent": NTC_MODE_DIVERGENT, "bucketed_mma": NTC_MODE_BUCKETED_MMA,
          "divergent_fma": NTC_MODE_DIVERGENT_FMA}
 EXPORTS = ("ntc_create", "ntc_decode", "ntc_decode_host", "ntc_destroy", "ntc_debug_taps", "ntc_debug_decode_rows",
@@ -59,6 +61,7 @@ class ntc_desc(ctypes.Structure):
         ("pe_frequencies", ctypes.c_uint32),
         ("activation", ctypes.c_uint32),
         ("leaky_slope", ctypes.c_float),
+        ("output_format", ctypes.c_uint32),
     ]
 
 
@@ -227,7 +230,7 @@ def queries_to_device(q: np.ndarray, device="cuda"):
 class Decoder:
     """An ntc context built from an assets object (see ``workloads.Assets``)."""
 
-    def __init__(self, assets, precision: str = "fp16"):
+    def __init__(self, assets, precision: str = "fp16", output: str = "fp32"):
         self._keep = [
             np.ascontiguousarray(assets.level_dims, dtype=np.uint32),
             np.ascontiguousarray(assets.latent_offsets, dtype=np.uint64),
@@ -257,7 +260,9 @@ class Decoder:
         d.pe_frequencies = getattr(assets, "pe_frequencies", 0)
         d.activation = getattr(assets, "activation", 0)
         d.leaky_slope = getattr(assets, "leaky_slope", 0.0)
+        d.output_format = OUTPUTS[output]
         self.desc = d
+        self.output = output
         self.out_dim = assets.out_dim
         self.num_decoders = assets.num_decoders
         self.num_levels = assets.num_levels
@@ -276,11 +281,15 @@ class Decoder:
         except Exception:
             pass
 
+    def out_dtype(self):
+        import torch
+        return torch.float16 if self.output == "fp16" else torch.float32
+
     def decode(self, queries, out=None, mode: str = "bucketed", stream=None):
         import torch
         n = queries.shape[0]
         if out is None:
-            out = torch.empty((n, self.out_dim), dtype=torch.float32, device=queries.device)
+            out = torch.empty((n, self.out_dim), dtype=self.out_dtype(), device=queries.device)
         ntc_decode(self.ctx, _ptr(queries), n, _ptr(out), _stream(stream), MODES[mode])
         return out
 
@@ -288,7 +297,7 @@ class Decoder:
         import torch
         n = queries.shape[0]
         if out is None:
-            out = torch.empty((n, self.out_dim), dtype=torch.float32, pin_memory=True)
+            out = torch.empty((n, self.out_dim), dtype=self.out_dtype(), pin_memory=True)
         ntc_decode_host(self.ctx, _ptr(queries), n, _ptr(out), _stream(stream), MODES[mode])
         return out
 
@@ -315,7 +324,7 @@ class Decoder:
         (ntc_debug_row; rows of bad queries keep their fill of 0xFF bytes)."""
         import torch
         n = queries.shape[0]
-        out = torch.empty((n, self.out_dim), dtype=torch.float32, device=queries.device)
+        out = torch.empty((n, self.out_dim), dtype=self.out_dtype(), device=queries.device)
         rows = torch.full((max(1, n), DEBUG_ROW.itemsize), 255, dtype=torch.uint8, device=queries.device)
         ntc_debug_decode_rows(self.ctx, _ptr(queries), n, _ptr(out), _ptr(rows), _stream(stream))
         return out, rows[:n].cpu().numpy().view(DEBUG_ROW).reshape(n)

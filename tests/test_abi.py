@@ -85,7 +85,9 @@ def test_descriptor_validation_before_any_device_work(lib):
                         (dict(latent_channels=4), 1),          # in_dim no longer levels x channels
                         (dict(pe_frequencies=2), 1),           # in_dim misses the 8 encoding inputs
                         (dict(pe_frequencies=9, in_dim=52), 2), (dict(activation=2), 1),
-                        (dict(activation=1, leaky_slope=float("inf")), 1)]:
+                        (dict(activation=1, leaky_slope=float("inf")), 1),
+                        (dict(output_format=2), 1),            # neither fp32 nor fp16 rows
+                        (dict(output_format=1, precision=2), 2)]:  # fp16 rows need a tensor-core precision
         assert lib.ntc_create(ctypes.byref(desc(**bad)), ctypes.byref(ctx)) == status, bad
     keep[4][0] = 1  # map entry beyond num_decoders
     assert lib.ntc_create(ctypes.byref(desc()), ctypes.byref(ctx)) == 1
@@ -115,3 +117,23 @@ def test_kmeans_map_validates_on_the_host():
     bad[3, 2] = np.inf
     assert call(F=bad) == ntc.NTC_ERR_INVALID_ARG
     assert b"finite" in ntc._lib.ntc_last_error()
+
+
+def test_descriptor_layout_matches_the_header(tmp_path):
+    """The ctypes ntc_desc has the C struct's fields at the C offsets (a C
+    program built against include/ntc.h prints them)."""
+    import shutil
+    import subprocess
+    from paper_2608_27888_gb300 import ntc
+    if not shutil.which("gcc"):
+        pytest.skip("no C compiler")
+    fields = [f for f, _ in ntc.ntc_desc._fields_]
+    src = tmp_path / "layout.c"
+    body = "\n".join(f'  printf("%zu\\n", offsetof(ntc_desc, {f}));' for f in fields)
+    src.write_text("#include <stddef.h>\n#include <stdio.h>\n#include \"ntc.h\"\nint main(void) {\n"
+                   + body + '\n  printf("%zu\\n", sizeof(ntc_desc));\n  return 0;\n}\n')
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    got = [int(x) for x in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
+    want = [getattr(ntc.ntc_desc, f).offset for f in fields] + [ctypes.sizeof(ntc.ntc_desc)]
+    assert got == want
