@@ -279,6 +279,12 @@ def mean_distinct(q, assets):
 
 # -------------------------------------------------------------- reference arm
 
+def ordinal(k: int) -> str:
+    """1st, 2nd, 3rd, 4th, ..., 11th, 12th, 13th, 21st, 31st."""
+    suf = "th" if 10 <= k % 100 <= 20 else {1: "st", 2: "nd", 3: "rd"}.get(k % 10, "th")
+    return f"{k}{suf}"
+
+
 def cpu_sample(q):
     """The bounded CPU sample of a batch: every 32nd query (about 1M of the
     headline's 33M), so it spans every frame and region."""
@@ -303,7 +309,7 @@ def run_reference(args, ws, rank):
         times.append(time.perf_counter() - t0)
     ms = 1e3 * statistics.mean(times)
     value = sample / (ms / 1e3)
-    desc = (f"every {stride}th query of the workload ({sample:,} of {len(w.queries):,}) per step, oracle on "
+    desc = (f"every {ordinal(stride)} query of the workload ({sample:,} of {len(w.queries):,}) per step, oracle on "
             f"{cores} host threads ({cpu_model()})")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
@@ -741,7 +747,7 @@ def cpu_baseline(w):
     oracle.decode(w.assets, q, nthreads=cores)
     dt = time.perf_counter() - t0
     return {"value": len(q) / dt, "unit": UNIT, "cores": cores, "cpu_model": cpu_model(), "kind": "oracle",
-            "sample": f"every {stride}th query of the timed batch ({len(q):,} of {len(w.queries):,}), oracle on "
+            "sample": f"every {ordinal(stride)} query of the timed batch ({len(q):,} of {len(w.queries):,}), oracle on "
                       f"{cores} host threads, {dt:.1f} s"}
 
 

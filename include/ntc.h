@@ -176,14 +176,16 @@ typedef struct {
 #define NTC_TILE_ROWS 128u
 
 /* Validate `desc`, copy latents, weights and map to the current CUDA device
- * and return a context in *out.  Synchronous.  On failure *out is NULL. */
+ * and return a context in *out: the per-set latents z_{g,i}, the group
+ * decoders D_g and the map c(i) of Sec. 3.3 (with Sec. 4's decoder shapes).
+ * Synchronous.  On failure *out is NULL. */
 NTC_API ntc_status ntc_create(const ntc_desc *desc, ntc_ctx **out);
 
 /* Decode n queries: every query's latent features go through the MLP decoder
- * of its texture set's group (the per-pixel decode of Sec. 2; set i uses the
- * shared decoder c(i) of Sec. 3.1): d_out[i][c] = channel c of
- * D_{c(set_i)}(features of query i), for c < out_dim, in the queries' original
- * order.  d_queries: device array of n records (16-byte aligned); d_out:
+ * of its texture set's group -- the per-pixel decode whose divergence Sec. 2
+ * measures, with the decoder D_g shared by the sets i of group g = c(i)
+ * (Sec. 3.1, Sec. 3.3): d_out[i][c] = channel c of D_{c(set_i)}(features of
+ * query i), for c < out_dim, in the queries' original order.  d_queries: device array of n records (16-byte aligned); d_out:
  * device array of n*out_dim elements of the context's output format (floats,
  * 4-byte aligned; or IEEE halves, 2-byte aligned).  Asynchronous on
  * `cuda_stream` (a cudaStream_t; NULL is the legacy default stream); no host
@@ -203,12 +205,17 @@ NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n
 NTC_API ntc_status ntc_decode_host(ntc_ctx *ctx, const ntc_query *h_queries, size_t n, void *h_out,
                            void *cuda_stream, ntc_mode mode);
 
-/* Free the context and everything it owns.  NULL is accepted. */
+/* Free the context and everything it owns (no paper counterpart).  NULL is
+ * accepted. */
 NTC_API ntc_status ntc_destroy(ntc_ctx *ctx);
 
 /* --------------------------------------------------------------- debug / test */
 
-/* Taps of every query, as the decode computes them.  d_idx: [n][num_levels][2][4]
+/* Taps of every query by the reference addressing (the sampling of Sec. 1's
+ * latent grids as the fp32, mma.sync and divergent paths compute it; the
+ * default tensor-core kernel's own taps, recorded by ntc_debug_decode_rows,
+ * have the same texel indices bit for bit and these weights times the mip
+ * blend factor).  d_idx: [n][num_levels][2][4]
  * uint64 texel indices into `latents`; d_w: same shape, fp32 bilinear weights;
  * d_t: [n] fp32 mip blend factor.  Slot [k][0] holds mip lo, slot [k][1] mip
  * lo+1 and is filled only when t > 0 (otherwise index UINT64_MAX, weight 0);
@@ -217,7 +224,9 @@ NTC_API ntc_status ntc_debug_taps(ntc_ctx *ctx, const ntc_query *d_queries, size
                           float *d_w, float *d_t, void *cuda_stream);
 
 /* The fp32 MLP input of every query, d_feat[n][in_dim]: the latent features
- * of every level, then the positional encoding (NaN rows for bad queries).
+ * of every level, then the positional encoding they are concatenated with
+ * (Sec. 4) (NaN rows for bad queries).  Computed in fp32 from the taps above
+ * (the tensor-core kernels blend in packed fp16 instead; see ntc_debug_row).
  * Device pointers; async. */
 NTC_API ntc_status ntc_debug_features(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, float *d_feat,
                               void *cuda_stream);
@@ -273,10 +282,12 @@ typedef struct {
 NTC_API ntc_status ntc_debug_decode_rows(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, void *d_out,
                                          ntc_debug_row *d_rows, void *cuda_stream);
 
-/* Upper bound on the number of 128-query tiles of n queries. */
+/* Upper bound on the number of 128-query tiles of n queries (no paper
+ * counterpart). */
 NTC_API size_t ntc_max_tiles(const ntc_ctx *ctx, size_t n);
 
-/* Number of bad queries decoded since creation or the last reset.  Synchronises
+/* Number of bad queries decoded since creation or the last reset (no paper
+ * counterpart: the paper's queries are always valid).  Synchronises
  * the device.  Returns NTC_ERR_CUDA (and still writes *count) when a kernel
  * gave up one of its bounded waits since then (every mbarrier wait of the
  * tcgen05 kernels ends after 200 ms; the bucketing waits on nothing): that
@@ -292,14 +303,16 @@ NTC_API ntc_status ntc_reset_error_count(ntc_ctx *ctx);
  * faults, traps or hangs. */
 NTC_API ntc_status ntc_debug_wait_timeout(ntc_ctx *ctx, void *cuda_stream);
 
-/* Stage timing.  When enabled, ntc_decode records CUDA events on its stream
+/* Stage timing (no paper counterpart; Sec. 4.4 times whole kernels).  When
+ * enabled, ntc_decode records CUDA events on its stream
  * before bucketing, between bucketing and the gather-decode, and after it.
  * ntc_stage_times waits for the last decode and returns, in milliseconds,
  * times[0] = bucketing (0 in divergent mode) and times[1] = gather-decode. */
 NTC_API ntc_status ntc_set_stage_timing(ntc_ctx *ctx, int enable);
 NTC_API ntc_status ntc_stage_times(ntc_ctx *ctx, float times[2]);
 
-/* Kernels this context has launched since creation (host-side counter). */
+/* Kernels this context has launched since creation (host-side counter; no
+ * paper counterpart). */
 NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
 
 /* ------------------------------------------------------ allocation-free entry
@@ -360,7 +373,8 @@ NTC_API ntc_status ntc_kmeans_map(const float *h_features, uint32_t n, uint32_t 
                                   const uint32_t *h_init, uint32_t max_iters, uint32_t *h_map,
                                   double *h_centroids, uint32_t *iters_run);
 
-/* Human-readable message of the last failed call on this host thread. */
+/* Human-readable message of the last failed call on this host thread (no
+ * paper counterpart). */
 NTC_API const char *ntc_last_error(void);
 NTC_API const char *ntc_status_string(ntc_status s);
 
