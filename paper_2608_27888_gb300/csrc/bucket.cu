@@ -15,10 +15,13 @@
 //            the decoder totals into the segment starts and the tile starts,
 //            and decides from Eq. 1's score whether the records are copied
 //   k_place  per chunk: each query's rank among the equal decoders of its
-//            chunk (stable); its place = segment start + chunk offset + rank;
-//            the chunk is sorted in shared memory and copied out with
-//            coalesced stores: perm[] and, when k_scan chose to, the query
-//            records in bucket order (staged in shared memory by cp.async)
+//            chunk (stable); its place = segment start + chunk offset + rank.
+//            When k_scan chose to copy the records, the chunk is sorted in
+//            shared memory and copied out with coalesced stores: perm[] and
+//            the query records in bucket order (staged by cp.async).
+//            Otherwise each perm entry is stored straight to its place: the
+//            equal decoders of a 32-query group get consecutive places, so a
+//            single-decoder group's stores coalesce
 // Divergence-aware: when the score is low (a G-buffer: most 32-query groups
 // need one decoder) a decoder's queries lie in long runs of the caller's
 // array, and the decode reads query perm[i] there directly; only a scattered

@@ -14,15 +14,19 @@
 //     packed fp16 (the latents' own type) and stores the fp16/bf16 feature row
 //     [16] into its stage with tcgen05.st (warp q writes TMEM lanes
 //     32q..32q+31, exactly its rows).
-//   Consumer (one elected thread issues every MMA): layer 1 reads A from the
-//     stage and B (the decoder's weights, copied by a TMA bulk copy whenever
-//     the decoder changes) from shared memory; its completion frees the stage;
-//     the ReLU/convert epilogue goes TMEM -> registers -> TMEM; layers 2 and 3
-//     read their A operand from TMEM too; each layer's bias is one more K step
-//     whose A is a shared block with a 1 in K column 0.  Layer 3 accumulates
-//     in the consumer's own 16 output columns, so the next tile's layer 1 is
-//     issued before it completes; the sigmoid epilogue then scatters rows to
-//     out[perm[i]].
+//   Consumer: layer 1 reads A from the stage and B (the decoder's weights,
+//     copied by a TMA bulk copy whenever the decoder changes) from shared
+//     memory; its completion frees the stage; the ReLU/convert epilogue goes
+//     TMEM -> registers -> TMEM; layers 2 and 3 read their A operand from TMEM
+//     too; each layer's bias is one more K step whose A is a shared block with
+//     a 1 in K column 0.  Layer 3 accumulates in the consumer's own 16 output
+//     columns, so the next tile's layer 1 runs before the outputs are read;
+//     the sigmoid epilogue scatters rows to out[perm[i]] (fp32, or fp16 rows).
+//     At H = 64 (four consumers) one elected thread of the consumer issues its
+//     MMAs.  At H = 128 (two consumers, tensor memory for no more) two issuer
+//     warps per consumer issue them and hand over through named barriers, the
+//     four epilogue warps only convert and write outputs, and a tile's
+//     outputs are written while the next tile's layer 2 runs.
 // Shared-memory B operands use the no-swizzle K-major canonical layout: 8-row
 // x 16-byte core matrices, K-adjacent core matrices 128 B apart (LBO), 8-row
 // groups K*16 B apart (SBO).  Every wait is bounded by time; on expiry the
