@@ -247,10 +247,11 @@ __host__ __device__ constexpr bool issuer_warp() {
 
 // Named barriers between a consumer's epilogue warps (E) and its issuers A and
 // B (ids above the warpgroup barriers 1..NP+NC), with their thread counts:
-// T A hands a tile over to E and B (192), X E has converted layer 1's result
-// (A waits, 160), Y E has converted the first half of layer 2's result and
-// read the previous tile's outputs (B waits, 160), Z E has converted all of it
-// (A and B wait, 192).
+// T A hands a tile over to E and B (192), X E has converted layer 1's result,
+// or taken over a tile with nothing to multiply (A waits, 160), Y E has
+// converted the first half of layer 2's result and read the previous tile's
+// outputs (B waits, 160), Z E has converted all of it (A and B wait, 192).  X,
+// Y and Z of a tile with nothing to multiply: only X.
 constexpr int kIssT = 0, kIssX = 1, kIssY = 2, kIssZ = 3;
 constexpr int kIssTN = 192, kIssXN = 160, kIssYN = 160, kIssZN = 192;
 template <int NP, int NC>
@@ -736,16 +737,19 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
           opend = true;
           poi = oi;
           pgood = good;
-        } else if (epi) {  // a tile with nothing to multiply: write the waiting outputs now
-          if (opend) {
-            wait_bar(obar, oph);
-            oph ^= 1;
-            opend = false;
+        } else {  // a tile with nothing to multiply
+          named_arrive(bX, kIssXN);  // taken over: A may hand over the next tile
+          if (epi) {                 // write the waiting outputs now
+            if (opend) {
+              wait_bar(obar, oph);
+              oph ^= 1;
+              opend = false;
+            }
+            wg_bar(wgid);
+            fence_after();
+            out_rows(poi, pgood);
+            epi = false;
           }
-          wg_bar(wgid);
-          fence_after();
-          out_rows(poi, pgood);
-          epi = false;
         }
       }
       if (epi && !stopped) {  // the last tile's outputs
@@ -872,19 +876,29 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
       };
       uint32_t dec = D;
       bool swap = false;
-      uint32_t stop = c < K ? prepare(c, dec, swap) : 0;
-      for (uint32_t k = c; k < K; k += NC) {
-        const uint32_t jc = k / NC, s = c * SC + jc % SC;
+      // Hands tile k over on T: the decision to stop (after the weights, if
+      // the decoder changes) in the slot of the tile's parity.  An arrival on
+      // T always follows this issuer's wait on X of the previous tile, which
+      // the epilogue warps pass only after T of that tile has completed, so
+      // two arrivals of this warp never meet in one barrier phase.  (Handing
+      // the next tile over before Z was slower: the epilogue warps then poll
+      // layer 1's barrier instead of waiting on T.)
+      auto hand_over = [&](uint32_t k, uint32_t stop) -> uint32_t {
+        const uint32_t jc = k / NC;
         if (lane == 0) {
-          if (swap && !stop && !*abort_flag) {
-            load_weights(dec);
-            cur = dec;
-          }
+          if (swap && !stop && !*abort_flag) load_weights(dec);
           stop |= *abort_flag;
           stop_flag[2 * c + (jc & 1)] = stop;
         }
+        if (swap) cur = dec;
         stop = __shfl_sync(0xFFFFFFFFu, stop, 0);
         named_arrive(bT, kIssTN);
+        return stop;
+      };
+      uint32_t stop = c < K ? prepare(c, dec, swap) : 0;
+      for (uint32_t k = c; k < K; k += NC) {
+        const uint32_t jc = k / NC, s = c * SC + jc % SC;
+        stop = hand_over(k, stop);
         if (stop) break;
         const uint32_t tdec = dec;
         if (tdec < D) {
@@ -896,8 +910,12 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
             umma_commit(empty_bar(s));
           }
           issued = true;
-          __syncwarp();
-          named_sync(bX, kIssXN);
+        } else if (lane == 0) {
+          mbar_arrive(empty_bar(s));  // a tile of bad queries: nothing to multiply
+        }
+        __syncwarp();
+        named_sync(bX, kIssXN);  // layer 1's result converted (or the bad tile taken over)
+        if (tdec < D) {
           if (lane == 0) {
             fence_after();
 #pragma unroll
@@ -906,8 +924,6 @@ __global__ void __launch_bounds__((NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 
             umma_commit(mbar);
           }
           ++l3;
-        } else if (lane == 0) {
-          mbar_arrive(empty_bar(s));  // a tile of bad queries: nothing to multiply
         }
         __syncwarp();
         // the next tile, while layer 2's result is converted

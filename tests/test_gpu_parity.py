@@ -235,6 +235,28 @@ def test_bad_queries_nan_and_counted():
         dec.close()
 
 
+@pytest.mark.parametrize("precision,output", [("fp16", "fp32"), ("bf16", "fp32"), ("fp16", "fp16")])
+def test_tiles_of_bad_queries_at_hidden_128(precision, output):
+    """40 % of the queries have out-of-range set ids: their bucket (the last)
+    is about 200 tiles with nothing to multiply, so the issuer warps of the
+    H = 128 kernel hand over runs of such tiles back to back."""
+    w = small("gbuffer-2160p-x4-trilinear")
+    q = w.queries.copy()
+    i = np.arange(len(q))
+    q["set_id"][i % 5 < 2] = 1000 + (i[i % 5 < 2] % 7)
+    q["u"][3::211] = np.nan
+    ref, nbad = oracle.decode(w.assets, q)
+    assert nbad > 0.4 * len(q)
+    dec = ntc().Decoder(w.assets, precision, output=output)
+    got = dec.decode(dq(q)).float().cpu().numpy()
+    bad = np.isnan(ref).any(axis=1)
+    assert np.array_equal(np.isnan(got).any(axis=1), bad)
+    assert np.isnan(got[bad]).all()
+    check_tc(got[~bad], ref[~bad], f"{precision}/{output}")
+    assert dec.error_count() == nbad
+    dec.close()
+
+
 def test_decode_host_equals_device_decode():
     w = small("gbuffer-1080p", "identity")
     dec = decoder("gbuffer-1080p", "identity", "fp16")
