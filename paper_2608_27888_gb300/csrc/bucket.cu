@@ -106,18 +106,33 @@ __global__ void __launch_bounds__(kBucketThreads) k_count(Assets A, const ntc_qu
   }
   uint32_t *my = cnt + warp * DW;
   uint32_t div = 0;  // this warp's groups: distinct decoders - 1
+  uint32_t dv[kBucketItems];
 #pragma unroll
   for (int it = 0; it < kBucketItems; ++it) {
     const size_t j = wbase + it * 32 + lane;
     const uint32_t dl = lookup(A, s[it]);  // every lane: the lookup shuffles
-    const uint32_t d = j < n ? dl : D + 1;
-    if (dec_out && j < n) dec_out[j] = (DecT)d;
-    const uint32_t m = match_key(d, nbits);
-    const bool leader = lane == __ffs(m) - 1;
-    if (leader) my[d] += __popc(m);
-    const uint32_t runs = __popc(__ballot_sync(0xFFFFFFFFu, leader && d <= D));
-    div += runs ? runs - 1 : 0u;
-    __syncwarp();
+    dv[it] = j < n ? dl : D + 1;
+    if (dec_out && j < n) dec_out[j] = (DecT)dv[it];
+  }
+  // a warp whose 256 queries all need one decoder (most of a G-buffer's):
+  // one count, no divergence
+  const uint32_t d0 = __shfl_sync(0xFFFFFFFFu, dv[0], 0);
+  bool one = true;
+#pragma unroll
+  for (int it = 0; it < kBucketItems; ++it) one &= dv[it] == d0;
+  if (__all_sync(0xFFFFFFFFu, one)) {
+    if (lane == 0) my[d0] += kBucketItems * 32;
+  } else {
+#pragma unroll
+    for (int it = 0; it < kBucketItems; ++it) {
+      const uint32_t d = dv[it];
+      const uint32_t m = match_key(d, nbits);
+      const bool leader = lane == __ffs(m) - 1;
+      if (leader) my[d] += __popc(m);
+      const uint32_t runs = __popc(__ballot_sync(0xFFFFFFFFu, leader && d <= D));
+      div += runs ? runs - 1 : 0u;
+      __syncwarp();
+    }
   }
   if (lane == 0 && div) atomicAdd(&s_div, div);
   __syncthreads();
@@ -338,17 +353,29 @@ __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc
     }
     if (own_offset && threadIdx.x <= D && !last)
       next_off = __ldcg(offs + (size_t)threadIdx.x * chunks + c + gridDim.x);
-    // rank of each query among the equal decoders of this warp's run, in order
+    // rank of each query among the equal decoders of this warp's run, in
+    // order; a warp whose 256 queries all need one decoder ranks them at once
     uint32_t *my = cnt + warp * DW;
     uint32_t rank[kBucketItems];
+    const uint32_t d0 = __shfl_sync(0xFFFFFFFFu, dec[0], 0);
+    bool one = true;
 #pragma unroll
-    for (int it = 0; it < kBucketItems; ++it) {
-      const uint32_t d = dec[it];
-      const uint32_t m = match_key(d, nbits);
-      rank[it] = my[d] + __popc(m & lt);
+    for (int it = 0; it < kBucketItems; ++it) one &= dec[it] == d0;
+    if (__all_sync(0xFFFFFFFFu, one)) {
+#pragma unroll
+      for (int it = 0; it < kBucketItems; ++it) rank[it] = it * 32 + lane;  // my[d0] is 0: a fresh chunk
+      if (lane == 0) my[d0] = kBucketItems * 32;
       __syncwarp();
-      if (lane == __ffs(m) - 1) my[d] += __popc(m);
-      __syncwarp();
+    } else {
+#pragma unroll
+      for (int it = 0; it < kBucketItems; ++it) {
+        const uint32_t d = dec[it];
+        const uint32_t m = match_key(d, nbits);
+        rank[it] = my[d] + __popc(m & lt);
+        __syncwarp();
+        if (lane == __ffs(m) - 1) my[d] += __popc(m);
+        __syncwarp();
+      }
     }
     __syncthreads();
     // per decoder: warp prefix (in place), the chunk's count and its global base
