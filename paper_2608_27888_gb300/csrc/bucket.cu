@@ -361,7 +361,8 @@ __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc
     bool one = true;
 #pragma unroll
     for (int it = 0; it < kBucketItems; ++it) one &= dec[it] == d0;
-    if (__all_sync(0xFFFFFFFFu, one)) {
+    one = __all_sync(0xFFFFFFFFu, one);  // the warp's 256 queries need decoder d0
+    if (one) {
 #pragma unroll
       for (int it = 0; it < kBucketItems; ++it) rank[it] = it * 32 + lane;  // my[d0] is 0: a fresh chunk
       if (lane == 0) my[d0] = kBucketItems * 32;
@@ -397,10 +398,19 @@ __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc
       // consecutive places, so the stores of a group of one decoder (most of
       // a G-buffer's) coalesce without a local sort
       if (last) pdl_trigger();  // the decode may launch (it waits for this grid before reading)
+      if (one) {  // one decoder: 256 consecutive places from one base
+        if (d0 <= D) {
+          const uint32_t base = gbase[d0] + cnt[warp * DW + d0];
 #pragma unroll
-      for (int it = 0; it < kBucketItems; ++it) {
-        const uint32_t d = dec[it];
-        if (d <= D) perm[gbase[d] + cnt[warp * DW + d] + rank[it]] = (uint32_t)(cbase + wbase + it * 32 + lane);
+          for (int it = 0; it < kBucketItems; ++it)
+            perm[base + it * 32 + lane] = (uint32_t)(cbase + wbase + it * 32 + lane);
+        }
+      } else {
+#pragma unroll
+        for (int it = 0; it < kBucketItems; ++it) {
+          const uint32_t d = dec[it];
+          if (d <= D) perm[gbase[d] + cnt[warp * DW + d] + rank[it]] = (uint32_t)(cbase + wbase + it * 32 + lane);
+        }
       }
       __syncthreads();  // cnt and gbase are reused by the next chunk
       for (uint32_t i = threadIdx.x; i < kWarps * DW; i += blockDim.x) cnt[i] = 0;
