@@ -1002,7 +1002,7 @@ cudaError_t launch_tm_t(const Assets &A, const WeightImages &W, const Buckets &B
   const int vec_out = ((uintptr_t)out & (W.out_half ? 15 : 31)) == 0;
   const unsigned threads = (NP + NC) * 128 + (issuer_warp<H>() ? NC * 64 : 0);
   // launched as a programmatic dependent of the bucketing: its prologue overlaps
-  // the end of k_scatter
+  // the end of k_place
   cudaError_t e;
   if (c8)
     e = launch_pdl(k_decode_tm<H, BF16, TRI, WRAP, 8, NP, NC, SC, DBG>, dim3((unsigned)grid), dim3(threads), smem, st,

@@ -430,10 +430,11 @@ def test_bucketing_with_the_most_decoders():
 
 @pytest.mark.parametrize("pattern", ["random", "same", "bad", "sparse"])
 def test_bucketed_decode_writes_every_row(pattern):
-    """The tensor-core decode sorts with the look-back counting sort (chunks in
-    ticket order, totals and tickets cleared by the last CTA).  Every row of
-    the output must be written exactly as the oracle decodes it, over chunk
-    boundaries and ragged tails, on consecutive calls of varying sizes."""
+    """The tensor-core decode sorts with the three-kernel counting sort
+    (per-chunk counts, a scan whose last CTA clears the ticket, stable
+    placement).  Every row of the output must be written exactly as the
+    oracle decodes it, over chunk boundaries and ragged tails, on consecutive
+    calls of varying sizes."""
     S, D = 40, 13
     rng = np.random.default_rng(7)
     m = rng.integers(0, D, S).astype(np.uint32)
