@@ -508,8 +508,38 @@ def end_to_end(torch, dec, hq, n, C, ws, mode, reps):
         dec.decode_host(hq, hout, mode=mode)
         ts.append(time.perf_counter() - t0)
     ms = 1e3 * statistics.mean(ts)
+    link = host_link_ms(torch, hq, hout, reps)
     return {"value": n * ws / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": n * 16,
-            "d2h_bytes_per_step": n * C * (2 if half else 4), "ms_per_step": ms}
+            "d2h_bytes_per_step": n * C * (2 if half else 4), "ms_per_step": ms,
+            "host_link": {"copy_ms_per_step": link, "frac": link / ms,
+                          "what": "the same upload and download alone, issued together on two streams "
+                                  "(no decode): the bound of this end-to-end number"}}
+
+
+def host_link_ms(torch, hq, hout, reps):
+    """The host link's own time for one step's bytes: the query upload and the
+    row download of a decode_host call, as two plain copies on two streams."""
+    dq = torch.empty(hq.shape, dtype=hq.dtype, device="cuda")
+    dout = torch.zeros(hout.shape, dtype=hout.dtype, device="cuda")
+    up, down = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def once():
+        with torch.cuda.stream(up):
+            dq.copy_(hq, non_blocking=True)
+        with torch.cuda.stream(down):
+            hout.copy_(dout, non_blocking=True)
+        torch.cuda.synchronize()
+
+    once()
+    once()
+    ts = []
+    for _ in range(reps):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        once()
+        ts.append(time.perf_counter() - t0)
+    del dq, dout
+    return 1e3 * statistics.mean(ts)
 
 
 def time_decode(torch, dec, qd, out, mode, flush, flush_rd, reps=5, warm=2):

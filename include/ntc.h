@@ -196,7 +196,7 @@ NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n
 
 /* ntc_decode on HOST buffers: copies the queries to context-owned device
  * memory, decodes, copies the outputs back into h_out and synchronises before
- * returning.  The batch is split into up to 8 chunks (at least 2^18 queries
+ * returning.  The batch is split into up to 32 chunks (at least 2^18 queries
  * each) whose upload, decode and download overlap: uploads and downloads run
  * on two context-owned streams ordered after the work already queued on
  * `cuda_stream`, decodes on `cuda_stream`.  Each chunk is bucketed on its own;

@@ -14,7 +14,7 @@ using namespace ntc;
 
 // ntc_decode_host splits a batch into at most kHostChunks pipelined chunks of
 // at least kHostChunkMin queries.
-constexpr int kHostChunks = 8, kHostChunksMax = kHostChunks;
+constexpr int kHostChunks = 32;
 constexpr size_t kHostChunkMin = 1u << 18;
 
 struct ntc_ctx {
@@ -53,7 +53,7 @@ struct ntc_ctx {
   ntc_query *d_hq = nullptr;
   uint8_t *d_hout = nullptr;  // [cap_host][C] output elements of out_bytes each
   cudaStream_t s_up = nullptr, s_down = nullptr;
-  cudaEvent_t ev_begin = nullptr, ev_up[kHostChunksMax] = {}, ev_done[kHostChunksMax] = {};
+  cudaEvent_t ev_begin = nullptr, ev_up = nullptr, ev_done = nullptr;
   uint64_t launches = 0;
   // optional stage timing
   bool timing = false;
@@ -156,10 +156,8 @@ WeightImages weights_of(const ntc_ctx *c) {
 void release(ntc_ctx *c) {
   for (auto &e : c->ev)
     if (e) cudaEventDestroy(e);
-  for (int i = 0; i < kHostChunksMax; ++i) {
-    if (c->ev_up[i]) cudaEventDestroy(c->ev_up[i]);
-    if (c->ev_done[i]) cudaEventDestroy(c->ev_done[i]);
-  }
+  if (c->ev_up) cudaEventDestroy(c->ev_up);
+  if (c->ev_done) cudaEventDestroy(c->ev_done);
   if (c->ev_begin) cudaEventDestroy(c->ev_begin);
   if (c->s_up) cudaStreamDestroy(c->s_up);
   if (c->s_down) cudaStreamDestroy(c->s_down);
@@ -586,15 +584,14 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, void *vhou
     CK(cudaStreamCreateWithFlags(&c->s_up, cudaStreamNonBlocking), "copy stream");
     CK(cudaStreamCreateWithFlags(&c->s_down, cudaStreamNonBlocking), "copy stream");
     CK(cudaEventCreateWithFlags(&c->ev_begin, cudaEventDisableTiming), "chunk event");
-    for (int i = 0; i < kHostChunksMax; ++i) {
-      CK(cudaEventCreateWithFlags(&c->ev_up[i], cudaEventDisableTiming), "chunk event");
-      CK(cudaEventCreateWithFlags(&c->ev_done[i], cudaEventDisableTiming), "chunk event");
-    }
+    CK(cudaEventCreateWithFlags(&c->ev_up, cudaEventDisableTiming), "chunk event");
+    CK(cudaEventCreateWithFlags(&c->ev_done, cudaEventDisableTiming), "chunk event");
   }
   // Chunks pipeline the upload (s_up), the decode (the caller's stream) and the
   // download (s_down): chunk i+1 uploads and chunk i-1 downloads while chunk i
   // decodes.  Each chunk is bucketed on its own; every query's output is the
-  // same as in one call over all n.
+  // same as in one call over all n.  One event per direction serves every
+  // chunk: a stream wait takes the event's latest record when it is enqueued.
   size_t chunk = (n + kHostChunks - 1) / kHostChunks;
   if (chunk < kHostChunkMin) chunk = kHostChunkMin;
   chunk = (chunk + kBucketChunk - 1) / kBucketChunk * kBucketChunk;
@@ -607,16 +604,16 @@ ntc_status ntc_decode_host(ntc_ctx *c, const ntc_query *hq, size_t n, void *vhou
     const size_t off = i * chunk, m = n - off < chunk ? n - off : chunk;
     CK(cudaMemcpyAsync(c->d_hq + off, hq + off, m * sizeof(ntc_query), cudaMemcpyHostToDevice, c->s_up),
        "query upload");
-    CK(cudaEventRecord(c->ev_up[i], c->s_up), "chunk event");
-    CK(cudaStreamWaitEvent(st, c->ev_up[i], 0), "stream order");
+    CK(cudaEventRecord(c->ev_up, c->s_up), "chunk event");
+    CK(cudaStreamWaitEvent(st, c->ev_up, 0), "stream order");
     s = ntc_decode(c, c->d_hq + off, m, c->d_hout + off * row, stream, mode);
     if (s != NTC_OK) {
       cudaStreamSynchronize(c->s_up);
       cudaStreamSynchronize(c->s_down);
       return s;
     }
-    CK(cudaEventRecord(c->ev_done[i], st), "chunk event");
-    CK(cudaStreamWaitEvent(c->s_down, c->ev_done[i], 0), "stream order");
+    CK(cudaEventRecord(c->ev_done, st), "chunk event");
+    CK(cudaStreamWaitEvent(c->s_down, c->ev_done, 0), "stream order");
     CK(cudaMemcpyAsync(hout + off * row, c->d_hout + off * row, m * row, cudaMemcpyDeviceToHost, c->s_down),
        "output download");
   }
