@@ -559,6 +559,27 @@ def time_decode(torch, dec, qd, out, mode, flush, flush_rd, reps=5, warm=2):
     return statistics.mean(ts)
 
 
+def launch_floor_ms(torch, flush, flush_rd, reps=20):
+    """The step time of a kernel that does nothing (a one-element fill), timed
+    as time_decode times a decode: one launch between two events after the L2
+    flush.  No call that launches a kernel can take less, so for a small batch
+    it caps the fraction of the roofline that any decode could reach."""
+    tiny = torch.zeros(1, dtype=torch.float32, device="cuda")
+    for _ in range(3):
+        tiny.zero_()
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        flush_rd.sum()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        tiny.zero_()
+        e1.record()
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    return statistics.median(ts)
+
+
 def paper_mirror(ntc, torch, precision, sizes=(512, 1024, 2048, 4096, 8192), ds=(5, 10)):
     """The setting of the paper's Tables 5-6 on this GPU: an N x N texel-centre
     raster where every 32-query warp holds d distinct texture sets (32 sets of
@@ -695,6 +716,7 @@ def per_workload(ntc, torch, precision, headline=None):
     peak, _ = peaks()
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     flush_rd = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    floor_ms = launch_floor_ms(torch, flush, flush_rd)
     rows = []
     for name, variant in (("raster-256", None), ("uniform-4m", None), ("gbuffer-1080p", "identity"),
                           ("gbuffer-1080p", "clustered4"), ("gbuffer-1080p", "shared"), ("gbuffer-2160p", "128"),
@@ -733,6 +755,9 @@ def per_workload(ntc, torch, precision, headline=None):
             dec.close()
             del qd, out, w, a, q
             torch.cuda.empty_cache()
+        # the best fraction a decode taking no time at all would show
+        row["launch_floor_ms"] = floor_ms
+        row["frac_of_roofline_cap"] = min(1.0, row["queries"] / (floor_ms / 1e3) / row["roofline_rate"])
         if comp and comp["queries"] == row["queries"]:
             cpq = comp["compulsory_bytes_per_query_excluding_weights"]
             row["compulsory_bytes_per_query"] = cpq

@@ -82,6 +82,11 @@ def test_fp16_rows_full_size_headline():
     ref, _ = oracle.decode(w.assets, w.queries[rows])
     got = out16[torch.from_numpy(rows).to(out16.device)].cpu().numpy().astype(np.float64)
     assert np.abs(got - ref.astype(np.float16).astype(np.float64)).max() <= TC_MAX + HALF_STEP
+    # through host buffers: 32 pipelined chunks of ceil(n / 32) queries rounded
+    # up to the bucketing chunk, the last one ragged
+    hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
+    host = d16.decode_host(hq)
+    assert torch.equal(host.view(torch.int16), out16.cpu().view(torch.int16))
     d16.close()
 
 

@@ -266,6 +266,27 @@ def test_decode_host_equals_device_decode():
     assert np.array_equal(host, dev)
 
 
+@pytest.mark.parametrize("output", ["fp32", "fp16"])
+@pytest.mark.parametrize("n", [3 * 2 ** 18 + 777, 4 * 2 ** 20 - 5, 4 * 2 ** 20])
+def test_decode_host_over_many_chunks(n, output):
+    """ntc_decode_host pipelines chunks of at least 2^18 queries (up to 32 of
+    them), each bucketed on its own.  On a fully divergent stream (every chunk
+    copies its records) the rows must equal one device-buffer decode over all
+    n bit for bit, with the last chunk ragged or full."""
+    w = W.named("uniform-4m", "full")
+    q = w.queries[:n]
+    dec = ntc().Decoder(w.assets, "fp16", output=output)
+    dev = dec.decode(dq(q)).cpu()
+    hq = torch.from_numpy(np.ascontiguousarray(q).view(np.int32).reshape(-1, 4)).pin_memory()
+    host = dec.decode_host(hq)
+    bits = torch.int16 if output == "fp16" else torch.int32
+    assert torch.equal(host.view(bits), dev.view(bits))
+    # a second call reuses the staging and the events
+    host2 = dec.decode_host(hq)
+    assert torch.equal(host2.view(bits), dev.view(bits))
+    dec.close()
+
+
 def test_empty_and_invalid_calls():
     m = ntc()
     dec = decoder("raster-256", None, "fp16")
