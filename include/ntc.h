@@ -30,8 +30,8 @@
  * Memory: the context owns device copies of latents, weights and map.  Query
  * and output buffers of ntc_decode are DEVICE pointers owned by the caller.
  * Scratch (the permutation and a decoder id per query, 5 or 6 bytes per
- * query, 4 bytes per decoder and 2048 queries of chunk counts, and the tile
- * table) is owned by the context and grows on demand with cudaMallocAsync on
+ * query, 8 bytes per decoder and 2048 queries of chunk counts and offsets, and
+ * the tile table) is owned by the context and grows on demand with cudaMallocAsync on
  * the call's stream.  Every bucketed decode sorts with the same stable
  * counting sort that ntc_debug_bucket exports.  One context must not run two
  * decodes concurrently (on different streams or threads).
@@ -40,6 +40,13 @@
  * message is available from ntc_last_error().  A query whose set id is out of
  * range or whose u or v is not finite decodes to NaN in every channel and is
  * counted (ntc_get_error_count).  No kernel traps.
+ *
+ * Environment: the bucketing kernels and the tensor-core decode after them
+ * are launched as programmatic dependents of their predecessor on the stream
+ * (each starts while the one before is finishing and waits for its results).
+ * With NTC_NO_PDL set (any value, read once per process) they are ordinary
+ * launches instead; the results are the same.  Profilers that replay a single
+ * kernel of such a chain need it.
  */
 #ifndef NTC_H
 #define NTC_H
@@ -331,7 +338,7 @@ NTC_API uint64_t ntc_launch_count(const ntc_ctx *ctx);
  * d_perm and d_sorted are caller-owned device buffers (the query buffers
  * 16-byte aligned).  Its kernels wait on nothing (no barrier, flag or
  * timeout), so a call that was enqueued completes.  Its scratch is one
- * file-scope device array of 1,360,896 bytes that every GPU loading the
+ * file-scope device array of 2,409,472 bytes that every GPU loading the
  * library holds until the process exits, so:
  *   - num_sets <= 65536, num_decoders <= 4095 and
  *     (num_decoders + 1) * ceil(n / 2048) <= 262144 (larger calls return

@@ -11,7 +11,9 @@
 //            decoder, and the divergence of its 32-query groups (Eq. 1:
 //            distinct decoders in a group - 1, summed)
 //   k_scan   one CTA per decoder scans that decoder's per-chunk counts into
-//            the chunk offsets; the last CTA to finish (atomic ticket) scans
+//            the chunk offsets (an array of their own: the counts are only
+//            read, so the kernel can run again on them, as a profiler's
+//            replay does); the last CTA to finish (atomic ticket) scans
 //            the decoder totals into the segment starts and the tile starts,
 //            and decides from Eq. 1's score whether the records are copied
 //   k_place  per chunk: each query's rank among the equal decoders of its
@@ -174,23 +176,23 @@ __device__ __forceinline__ uint32_t block_scan_1024(uint32_t v, uint32_t &total,
   return excl;
 }
 
-// Scan `len` values in place (exclusive) with 1024 threads, 4 per thread per
-// round; returns the total.
-__device__ uint32_t block_scan_inplace(uint32_t *a, uint32_t len, uint32_t *ws) {
+// Exclusive scan of `len` values of src into dst (dst may be src) with 1024
+// threads, 4 per thread per round; returns the total.
+__device__ uint32_t block_scan_to(const uint32_t *src, uint32_t *dst, uint32_t len, uint32_t *ws) {
   uint32_t carry = 0;
   for (uint32_t b = 0; b < len; b += 4096) {
     uint32_t v[4], s = 0;
     const uint32_t i0 = b + threadIdx.x * 4;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      v[j] = i0 + j < len ? a[i0 + j] : 0u;
+      v[j] = i0 + j < len ? src[i0 + j] : 0u;
       s += v[j];
     }
     uint32_t tot;
     uint32_t e = block_scan_1024(s, tot, ws) + carry;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      if (i0 + j < len) a[i0 + j] = e;
+      if (i0 + j < len) dst[i0 + j] = e;
       e += v[j];
     }
     carry += tot;
@@ -201,15 +203,15 @@ __device__ uint32_t block_scan_inplace(uint32_t *a, uint32_t len, uint32_t *ws) 
 // meta layout: [0] num_tiles, [1 .. D+2] seg_start, [D+3 .. 2D+4] tile_start,
 // [2D+5] copied, [2D+6] divergence; then totals [D+1], the ticket and the
 // divergence sum of k_count (zero between calls).
-__global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks, uint32_t D, uint32_t *meta,
-                                               int force_copy) {
+__global__ void __launch_bounds__(1024) k_scan(const uint32_t *counts, uint32_t *offs, uint32_t chunks, uint32_t D,
+                                               uint32_t *meta, int force_copy) {
   __shared__ uint32_t ws[32];
   __shared__ bool last;
   const uint32_t d = blockIdx.x;
   uint32_t *totals = meta + meta_words(D), *ticket = totals + (D + 1), *div_sum = ticket + 1;
   pdl_wait();     // the per-chunk counts of k_count
   pdl_trigger();  // k_place may launch (it waits for this grid before reading)
-  const uint32_t tot = block_scan_inplace(counts + (size_t)d * chunks, chunks, ws);
+  const uint32_t tot = block_scan_to(counts + (size_t)d * chunks, offs + (size_t)d * chunks, chunks, ws);
   if (threadIdx.x == 0) {
     totals[d] = tot;
     __threadfence();
@@ -226,9 +228,9 @@ __global__ void __launch_bounds__(1024) k_scan(uint32_t *counts, uint32_t chunks
     tst[i] = (c + kTile - 1) / kTile;
   }
   __syncthreads();
-  const uint32_t ns = block_scan_inplace(seg, D + 1, ws);
+  const uint32_t ns = block_scan_to(seg, seg, D + 1, ws);
   __syncthreads();
-  const uint32_t nt = block_scan_inplace(tst, D + 1, ws);
+  const uint32_t nt = block_scan_to(tst, tst, D + 1, ws);
   if (threadIdx.x == 0) {
     seg[D + 1] = ns;  // == n
     tst[D + 1] = nt;
@@ -402,14 +404,17 @@ __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc
         if (d0 <= D) {
           const uint32_t base = gbase[d0] + cnt[warp * DW + d0];
 #pragma unroll
-          for (int it = 0; it < kBucketItems; ++it)
-            perm[base + it * 32 + lane] = (uint32_t)(cbase + wbase + it * 32 + lane);
+          for (int it = 0; it < kBucketItems; ++it) {
+            const uint32_t p = base + it * 32 + lane;
+            if (p < n) perm[p] = (uint32_t)(cbase + wbase + it * 32 + lane);
+          }
         }
       } else {
 #pragma unroll
         for (int it = 0; it < kBucketItems; ++it) {
           const uint32_t d = dec[it];
-          if (d <= D) perm[gbase[d] + cnt[warp * DW + d] + rank[it]] = (uint32_t)(cbase + wbase + it * 32 + lane);
+          const uint32_t p = d <= D ? gbase[d] + cnt[warp * DW + d] + rank[it] : 0xFFFFFFFFu;
+          if (p < n) perm[p] = (uint32_t)(cbase + wbase + it * 32 + lane);
         }
       }
       __syncthreads();  // cnt and gbase are reused by the next chunk
@@ -438,8 +443,10 @@ __global__ void __launch_bounds__(kBucketThreads, 5) k_place(Assets A, const ntc
     for (uint32_t i = threadIdx.x; i < valid; i += blockDim.x) {
       const uint32_t d = sdec[i], j = sidx[i];
       const uint32_t pos = gbase[d] + (i - loff[d]);
-      perm[pos] = (uint32_t)(cbase + j);
-      reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
+      if (pos < n) {
+        perm[pos] = (uint32_t)(cbase + j);
+        reinterpret_cast<uint4 *>(sorted)[pos] = srec[j];
+      }
     }
     __syncthreads();  // srec, sidx, sdec, loff and gbase are reused by the next chunk
     if (FROM_Q && !last) {
@@ -516,15 +523,17 @@ cudaError_t launch_bucket_t(const Assets &A, const ntc_query *q, size_t n, const
   DecT *dec = reinterpret_cast<DecT *>(s.dec);
   k_count<DecT><<<chunks, kBucketThreads, smem_count, st>>>(A, q, n, chunks, s.counts, div_sum, dec);
   e = cudaGetLastError();
-  if (e == cudaSuccess) e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, s.counts, chunks, D, s.meta, copy);
+  if (e == cudaSuccess)
+    e = launch_pdl(k_scan, dim3(D + 1), dim3(1024), 0, st, (const uint32_t *)s.counts, s.offs, chunks, D, s.meta,
+                   copy);
   if (e == cudaSuccess) {
     if (from_q)
       e = launch_pdl(k_place<DecT, true>, dim3(place_grid), dim3(kBucketThreads), smem_place, st, A, q,
-                     (const DecT *)nullptr, n, chunks, (const uint32_t *)s.counts, (const uint32_t *)s.meta,
+                     (const DecT *)nullptr, n, chunks, (const uint32_t *)s.offs, (const uint32_t *)s.meta,
                      s.perm, s.sorted);
     else
       e = launch_pdl(k_place<DecT, false>, dim3(place_grid), dim3(kBucketThreads), smem_place, st, A, q,
-                     (const DecT *)dec, n, chunks, (const uint32_t *)s.counts, (const uint32_t *)s.meta, s.perm,
+                     (const DecT *)dec, n, chunks, (const uint32_t *)s.offs, (const uint32_t *)s.meta, s.perm,
                      s.sorted);
   }
   if (e != cudaSuccess) return e;

@@ -8,8 +8,8 @@
 // counting sort by decoder id (the same kernels as ntc_decode and
 // ntc_debug_bucket) without a context and without allocating: a copy of the
 // set->decoder map, the tile table with the totals and the ticket, and the
-// per-chunk counts live in one file-scope device array of fixed size that
-// every GPU loading this library keeps until the process exits.
+// per-chunk counts and offsets live in one file-scope device array of fixed
+// size that every GPU loading this library keeps until the process exits.
 #include <mutex>
 
 #include "ntc_internal.cuh"
@@ -24,8 +24,8 @@ namespace {
 
 constexpr size_t kMapWords = 65536;    // set->decoder map copy
 constexpr size_t kMetaWords = 12544;   // tile table, totals, ticket, divergence sum (<= 12295 words for D <= 4095)
-constexpr size_t kCountWords = 262144; // (D+1) * ceil(n / 2048) per-chunk counts
-constexpr size_t kStaticWords = kMapWords + kMetaWords + kCountWords;  // 1,360,896 bytes
+constexpr size_t kCountWords = 262144; // (D+1) * ceil(n / 2048) per-chunk counts, and as many offsets
+constexpr size_t kStaticWords = kMapWords + kMetaWords + 2 * kCountWords;  // 2,409,472 bytes
 
 // The scratch.  In host code this name is only a host-side stand-in: kernels
 // receive the device address looked up with cudaGetSymbolAddress below.
@@ -82,6 +82,7 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
   uint32_t *map = base;
   uint32_t *meta = base + kMapWords;
   uint32_t *counts = meta + kMetaWords;
+  uint32_t *offs = counts + kCountWords;
   // the map copy, and the tile table, totals and ticket cleared (the ticket
   // must start at 0)
   cudaError_t e = cudaMemcpyAsync(map, h_set_to_decoder, (size_t)num_sets * 4, cudaMemcpyHostToDevice, st);
@@ -95,6 +96,7 @@ extern "C" NTC_API ntc_status ntc_bucket_static(const uint32_t *h_set_to_decoder
   s.perm = d_perm;
   s.meta = meta;
   s.counts = counts;
+  s.offs = offs;
   s.sorted = d_sorted;
   s.dec = nullptr;  // no room for a decoder per query: the placement reads the staged records
   int launches = 0;

@@ -2,6 +2,7 @@
 // copies of the assets, scratch management and the launch sequence of each
 // decode path.
 #include <stdarg.h>
+#include <stdlib.h>
 #include <stdio.h>
 #include <string.h>
 
@@ -73,6 +74,10 @@ static ntc_status fail(ntc_status s, const char *fmt, ...) {
 
 namespace ntc {
 void set_last_error(const char *msg) { snprintf(g_err, sizeof g_err, "%s", msg); }
+bool pdl_enabled() {
+  static const bool on = getenv("NTC_NO_PDL") == nullptr;
+  return on;
+}
 }  // namespace ntc
 
 static ntc_status cuda_fail(cudaError_t e, const char *what) {
@@ -187,8 +192,9 @@ size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 // Make sure the bucketing scratch holds n queries (stream-ordered
 // allocation): perm, the sorted query records and the decoder ids [n], the
-// per-chunk counts, and the tile table with the totals, the ticket and the
-// divergence sum (zeroed once; the bucketing leaves them at zero).
+// per-chunk counts and offsets (one allocation, offsets in its second half),
+// and the tile table with the totals, the ticket and the divergence sum
+// (zeroed once; the bucketing leaves them at zero).
 ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
   const size_t counts = bucket_count_words(c->D, n);
   if (!c->d_meta) {
@@ -200,7 +206,7 @@ ntc_status ensure_scratch(ntc_ctx *c, size_t n, cudaStream_t st) {
     if (c->d_counts) CK(cudaFreeAsync(c->d_counts, st), "scratch free");
     c->d_counts = nullptr;
     c->cap_counts = 0;
-    CK(cudaMallocAsync((void **)&c->d_counts, counts * 4, st), "scratch allocation");
+    CK(cudaMallocAsync((void **)&c->d_counts, 2 * counts * 4, st), "scratch allocation");
     c->cap_counts = counts;
   }
   if (n > c->cap_n) {
@@ -224,6 +230,7 @@ Scratch scratch_of(const ntc_ctx *c) {
   s.perm = c->d_perm;
   s.meta = c->d_meta;
   s.counts = c->d_counts;
+  s.offs = c->d_counts + c->cap_counts;
   s.sorted = c->d_sorted;
   s.dec = c->d_dec;
   return s;

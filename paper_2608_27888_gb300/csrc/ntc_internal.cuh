@@ -514,7 +514,10 @@ struct Scratch {
   uint32_t *meta;     // bucket_meta_words(D): the tile table, then the totals
                       // [D+1], a ticket and the divergence sum (zero between
                       // calls)
-  uint32_t *counts;   // [bucket_count_words(D, n)] per-chunk counts, then offsets
+  uint32_t *counts;   // [bucket_count_words(D, n)] per-chunk counts (k_count)
+  uint32_t *offs;     // [bucket_count_words(D, n)] per-chunk offsets (k_scan);
+                      // a separate array, so that running k_scan again (a
+                      // profiler's replay) reads the same counts
   void *dec;          // [n] decoder per query, bucket_dec_bytes(D) bytes each;
                       // null: k_place reads the decoders from the records, which
                       // it then always stages and copies (copy must be 1)
@@ -635,6 +638,12 @@ class PerDevice {
   }
 };
 
+// False when the environment variable NTC_NO_PDL is set (read once per
+// process): launch_pdl then makes ordinary launches, which start only after
+// their predecessor has ended.  The results are the same; a profiler that
+// replays one kernel of the chain needs it.
+bool pdl_enabled();
+
 // Launch with programmatic stream serialisation (see pdl_wait).
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
@@ -648,7 +657,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 

@@ -287,6 +287,46 @@ def test_decode_host_over_many_chunks(n, output):
     dec.close()
 
 
+NO_PDL_CASES = [("gbuffer-2160p-x4-trilinear", None), ("uniform-4m", None), ("gbuffer-1080p", "clustered4"),
+                ("gbuffer-1080p", "shared")]
+
+
+def test_ordinary_launches_give_the_same_rows(tmp_path):
+    """With NTC_NO_PDL set the bucketing and decode kernels are ordinary
+    launches instead of programmatic dependents; a process decoding that way
+    must produce the same bits, through device and host buffers."""
+    import os
+    import subprocess
+    import sys
+    import textwrap
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    script = textwrap.dedent(f"""
+        import sys
+        import numpy as np
+        import torch
+        sys.path.insert(0, {root!r})
+        from paper_2608_27888_gb300 import ntc, workloads as W
+        for i, (name, variant) in enumerate({NO_PDL_CASES!r}):
+            w = W.named(name, "small", variant)
+            dec = ntc.Decoder(w.assets, "fp16")
+            np.save({str(tmp_path)!r} + f"/dev{{i}}.npy", dec.decode(ntc.queries_to_device(w.queries)).cpu().numpy())
+            hq = torch.from_numpy(np.ascontiguousarray(w.queries).view(np.int32).reshape(-1, 4)).pin_memory()
+            np.save({str(tmp_path)!r} + f"/host{{i}}.npy", dec.decode_host(hq).numpy())
+            dec.close()
+    """)
+    env = dict(os.environ, NTC_NO_PDL="1")
+    r = subprocess.run([sys.executable, "-c", script], env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    for i, (name, variant) in enumerate(NO_PDL_CASES):
+        w = small(name, variant)
+        dec = ntc().Decoder(w.assets, "fp16")
+        got = dec.decode(dq(w.queries)).cpu().numpy()
+        dec.close()
+        for kind in ("dev", "host"):
+            other = np.load(tmp_path / f"{kind}{i}.npy")
+            assert np.array_equal(got.view(np.uint32), other.view(np.uint32)), (name, variant, kind)
+
+
 def test_empty_and_invalid_calls():
     m = ntc()
     dec = decoder("raster-256", None, "fp16")
