@@ -334,8 +334,12 @@ __global__ void __launch_bounds__(kTile) k_decode_mma(Assets A, WeightImages W, 
   }
 }
 
+// At most 128 registers a thread, so that four CTAs (16 warps) fit on an SM.
+// The warp MLP wants ~180 at H = 128 (both m-tiles of the hidden layer as A
+// fragments); the few spills cost less than the latency that eight warps
+// cannot hide (measured on config 5: 13.8 -> 11.2 ms; 3 CTAs: 14.0, 5: 18.2).
 template <int H, int NT3, bool BF16>
-__global__ void __launch_bounds__(128) k_decode_divergent(Assets A, WeightImages W,
+__global__ void __launch_bounds__(128, 4) k_decode_divergent(Assets A, WeightImages W,
                                                           const ntc_query *qs, size_t n,
                                                           float *out, unsigned long long *err) {
   using I = MmaImage<H>;
