@@ -80,8 +80,13 @@ __device__ __forceinline__ float2 dot8(const float (&w)[8], const float *x, floa
   return acc;
 }
 
+// Register cap: each lane holds its whole hidden vector, so the compiler takes
+// ~230 registers a thread at H = 128 (2 CTAs, 8 warps per SM) and ~140 at
+// H = 64.  Capping them for 4 (H = 128) or 3 (H = 64) CTAs per SM spills a
+// little and hides more of the gather latency; measured on config 5 158 -> 97
+// ms, on the 1080p G-buffer (H = 64) 1.24 -> 1.09 ms; more CTAs were slower.
 template <int H, int CP, typename T>
-__global__ void __launch_bounds__(128) k_decode_divergent_fma(Assets A, const uint8_t *img, size_t stride,
+__global__ void __launch_bounds__(128, H >= 128 ? 4 : 3) k_decode_divergent_fma(Assets A, const uint8_t *img, size_t stride,
                                                               uint32_t C, const ntc_query *qs, size_t n,
                                                               float *out, unsigned long long *err) {
   using E = Elem<T>;
