@@ -44,6 +44,30 @@ def test_static_bucketing_matches_the_oracle_on_consecutive_calls():
         assert torch.equal(perm, ref_perm)
 
 
+def test_static_bucketing_at_its_largest_size():
+    """4,095 decoders and 64 chunks of 2,048 queries: (4095 + 1) x 64 = 262,144
+    per-chunk counts, exactly what the static scratch holds (the offsets fill
+    the second half of it to its last word).  Out-of-range set ids form the
+    extra bucket.  Equal to the oracle bit for bit, twice in a row."""
+    from paper_2608_27888_gb300 import ntc
+    from tests.util import QD
+    D, n = 4095, 64 * 2048
+    rng = np.random.default_rng(23)
+    q = np.zeros(n, dtype=QD)
+    q["set_id"] = rng.integers(0, D + 40, n)  # ~1 % beyond the map
+    m = rng.permutation(D).astype(np.uint32)
+    qd = ntc.queries_to_device(q)
+    p, _, _, _ = oracle.bucket(q["set_id"], m, D)
+    for _ in range(2):
+        perm = torch.full((n,), -1, dtype=torch.int32, device="cuda")
+        srt = torch.zeros((n, 4), dtype=torch.int32, device="cuda")
+        ntc.ntc_bucket_static(m.ctypes.data, D, D, qd.data_ptr(), n, perm.data_ptr(), srt.data_ptr(),
+                              torch.cuda.current_stream().cuda_stream)
+        torch.cuda.synchronize()
+        assert np.array_equal(perm.cpu().numpy().astype(np.uint32), p)
+        assert torch.equal(srt, qd[perm.long()])
+
+
 def test_static_bucketing_rejects_sizes_beyond_its_scratch():
     from paper_2608_27888_gb300 import ntc
     w = W.named("raster-256", "small")
