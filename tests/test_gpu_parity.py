@@ -284,6 +284,12 @@ def test_decode_host_over_many_chunks(n, output):
     # a second call reuses the staging and the events
     host2 = dec.decode_host(hq)
     assert torch.equal(host2.view(bits), dev.view(bits))
+    # pageable buffers: the copies no longer overlap, the rows are the same
+    pq = torch.empty(hq.shape, dtype=hq.dtype)
+    pq.copy_(hq)
+    pout = torch.empty(dev.shape, dtype=dev.dtype)
+    dec.decode_host(pq, pout)
+    assert torch.equal(pout.view(bits), dev.view(bits))
     dec.close()
 
 
