@@ -192,12 +192,12 @@ NTC_API ntc_status ntc_create(const ntc_desc *desc, ntc_ctx **out);
  * of its texture set's group -- the per-pixel decode whose divergence Sec. 2
  * measures, with the decoder D_g shared by the sets i of group g = c(i)
  * (Sec. 3.1, Sec. 3.3): d_out[i][c] = channel c of D_{c(set_i)}(features of
- * query i), for c < out_dim, in the queries' original order.  d_queries: device array of n records (16-byte aligned); d_out:
- * device array of n*out_dim elements of the context's output format (floats,
- * 4-byte aligned; or IEEE halves, 2-byte aligned).  Asynchronous on
- * `cuda_stream` (a cudaStream_t; NULL is the legacy default stream); no host
- * synchronisation.  n = 0 is a no-op.  Output for a bad query is NaN in every
- * channel. */
+ * query i), for c < out_dim, in the queries' original order.
+ * d_queries: device array of n records (16-byte aligned).  d_out: device
+ * array of n*out_dim elements of the context's output format (floats, 4-byte
+ * aligned; or IEEE halves, 2-byte aligned).  Asynchronous on `cuda_stream` (a
+ * cudaStream_t; NULL is the legacy default stream); no host synchronisation.
+ * n = 0 is a no-op.  Output for a bad query is NaN in every channel. */
 NTC_API ntc_status ntc_decode(ntc_ctx *ctx, const ntc_query *d_queries, size_t n, void *d_out,
                       void *cuda_stream, ntc_mode mode);
 
@@ -242,7 +242,8 @@ NTC_API ntc_status ntc_debug_features(ntc_ctx *ctx, const ntc_query *d_queries, 
  * different decoders are what diverges; sorting by decoder leaves tiles of one
  * decoder), by the same kernels and the same scratch as ntc_decode's BUCKETED
  * mode.  d_perm[n]: query indices in (decoder, original index) order, where a
- * query with an out-of-range set id counts as decoder num_decoders.  d_counts (may be NULL): [num_decoders+1] queries per decoder.
+ * query with an out-of-range set id counts as decoder num_decoders.
+ * d_counts (may be NULL): [num_decoders+1] queries per decoder.
  * d_tiles (may be NULL): [ntc_max_tiles(ctx, n)][3] = (decoder, first position
  * in perm, length) of every 128-query tile, in decoder order; d_num_tiles (may
  * be NULL): [1] the number of tiles written.  d_divergence (may be NULL): [2]
